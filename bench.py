@@ -1,0 +1,394 @@
+"""Benchmark of the evicted decode step on GB300.
+
+Workload (default): Qwen2.5-Math-7B decode geometry (28 layers, 28 query /
+4 KV heads, head_dim 128, bf16), a batch of 64 independent sequences with
+prior context lengths drawn uniformly from [512, 16384], budget B=64 and
+recent window W=8.  The prompts are loaded with zero scores; the first decode
+step evicts each unit down to B+W (timed separately as `first_step_ms`);
+after that every step is the steady state: append, attend over B+W+1 rows,
+accumulate scores, evict one row per (sequence, layer, KV head).
+
+One "step" = one decode token for all 64 sequences and all 28 layers, run as
+one kvr_decode_step call over every layer.  `value` is steps/s with inputs
+resident in HBM; `e2e` is the same metric with the step's q/k/v copied from
+pinned host memory and its output copied back inside the timed region.
+
+`python bench.py --impl reference` times the fp64 CPU oracle on the same
+workload instead (a bounded sample: one of the 64 sequences per step,
+extrapolated to the whole batch).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2608_15797_gb300 import cost_model, inputs  # noqa: E402
+
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=4000)
+    p.add_argument("--warmup", type=int, default=50)
+    p.add_argument("--impl", default="kvr", choices=["kvr", "reference"])
+    p.add_argument("--workload", default="7b_s64_b64")
+    p.add_argument("--seed", type=int, default=0)
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--cpu-seconds", type=float, default=15.0)
+    return p.parse_args()
+
+
+def metric_name(w):
+    return (f"evicted decode steps/s at 7B geometry, B={w.budget}, W={w.window}"
+            f" ({w.n_seq} sequences x {w.n_layers} layers per step)")
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            return json.load(f), "measured"
+    return {"hbm_gbs": FALLBACK_HBM_GBS}, "fallback"
+
+
+# --------------------------------------------------------------------------
+# CPU oracle timing (the reference arm and the cpu_baseline field)
+# --------------------------------------------------------------------------
+
+def oracle_rate(w, seed, max_seconds, max_steps=None):
+    from oracle import oracle as orc
+    L, H, G, d = w.n_layers, w.n_kv_heads, w.group, w.head_dim
+    m = w.budget + w.window
+    o = orc.OracleCache(1, L, H, G, d, cap=m + 1)
+    k, v = inputs.prompt(w, seed, 0, m)
+    o.load(0, k, v, first_pos=16384 - m)
+    pre = [inputs.step_inputs(w, seed, i, 1) for i in range(8)]
+    o.step(*pre[0], B=w.budget, W=w.window)
+    spent, n = 0.0, 0
+    while spent < max_seconds and (max_steps is None or n < max_steps):
+        q, kn, vn = pre[(n + 1) % len(pre)]
+        t = time.perf_counter()
+        o.step(q, kn, vn, B=w.budget, W=w.window)
+        spent += time.perf_counter() - t
+        n += 1
+    per_seq_step = spent / n
+    # one step of the workload = n_seq sequences
+    return 1.0 / (per_seq_step * w.n_seq), n, spent
+
+
+# --------------------------------------------------------------------------
+# clocks sampled during the timed region
+# --------------------------------------------------------------------------
+
+class ClockSampler:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,"
+             "clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+             "clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,"
+             "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.lines = []
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.QUERY,
+                 "--format=csv,noheader,nounits", "-lms", "50"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+        t0 = time.time()
+        while not self.lines and time.time() - t0 < 5:
+            time.sleep(0.02)
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append((time.time(), line.strip()))
+
+    def mark(self):
+        return time.time()
+
+    def stop(self, t_begin, t_end):
+        if self.proc is None:
+            return None
+        time.sleep(0.1)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = [l for t, l in self.lines if t_begin <= t <= t_end + 0.05]
+        if not rows:
+            rows = [l for _, l in self.lines[-3:]]
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown",
+                 "sw_power_cap"]
+        for r in rows:
+            f = [x.strip() for x in r.split(",")]
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except (ValueError, IndexError):
+                continue
+            for nm, val in zip(names, f[5:9]):
+                if val.lower() == "active":
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": max(mx),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# --------------------------------------------------------------------------
+# the CUDA arm
+# --------------------------------------------------------------------------
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2608_15797_gb300", "csrc")
+    for fn in sorted(os.listdir(csrc)):
+        if fn.endswith((".cu", ".h")):
+            with open(os.path.join(csrc, fn), "rb") as f:
+                h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def committed_traffic(workload):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken
+    on the current kernel sources."""
+    path = os.path.join(ROOT, "profiles", f"decode_step_{workload}.json")
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        d = json.load(f)
+    if d.get("kernel_sources_sha") != kernel_source_hash():
+        return None
+    return d.get("dram_bytes_per_launch")
+
+
+def run_kvr(args, rank, world, local_rank):
+    import torch
+    from paper_2608_15797_gb300 import kvr
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    w = inputs.WORKLOADS[args.workload]
+    S, L, H, G, d = w.n_seq, w.n_layers, w.n_kv_heads, w.group, w.head_dim
+    B, W = w.budget, w.window
+    lens = inputs.prior_lengths(args.seed + 7919 * rank, S)
+    cap = int(lens.max()) + 1
+    cache = kvr.Cache(S, L, H, G, d, cap, kv_dtype="bf16", out_dtype="bf16",
+                      device=dev)
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(1_000_003 * (args.seed + 1) + rank)
+    for s in range(S):
+        n = int(lens[s])
+        k = (torch.randn(L, H, n, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+        v = (torch.randn(L, H, n, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+        cache.load(s, k, v)
+        del k, v
+    torch.cuda.synchronize()
+
+    n_pool = 16
+    pool = []
+    for _ in range(n_pool):
+        q = (torch.randn(S, L, H * G, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+        kn = (torch.randn(S, L, H, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+        vn = (torch.randn(S, L, H, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+        pool.append((q, kn, vn))
+    out = torch.empty(S, L, H * G, d, dtype=torch.bfloat16, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    # First step: evicts every unit from its prior length down to B + W.
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    kvr.kvr_decode_step(cache.handle, 0, L, *pool[0], out, B, W, stream)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    first_ms = ev0.elapsed_time(ev1)
+    cache.sync_status()
+    assert (cache.lengths() == B + W).all()
+
+    def step(i):
+        q, kn, vn = pool[i % n_pool]
+        kvr.kvr_decode_step(cache.handle, 0, L, q, kn, vn, out, B, W, stream)
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+
+    K = args.steps
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
+    sampler = ClockSampler(local_rank) if rank == 0 else None
+    if sampler:
+        sampler.start()
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    launches0 = cache.launch_count()
+    t_begin = time.time()
+    for i in range(K):
+        starts[i].record(stream)
+        step(i)
+        ends[i].record(stream)
+    torch.cuda.synchronize()
+    t_end = time.time()
+    launches = cache.launch_count() - launches0
+    if world > 1:
+        torch.distributed.barrier()
+    clocks = sampler.stop(t_begin, t_end) if sampler else None
+    total_ms = starts[0].elapsed_time(ends[-1])
+    per_launch_ms = sum(s.elapsed_time(e) for s, e in zip(starts, ends)) / K
+    cache.sync_status()
+
+    if world > 1:
+        t = torch.tensor([total_ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        total_ms = float(t.item())
+
+    # End to end through the public call: pinned host inputs in, output out.
+    hpool = [tuple(x.cpu().pin_memory() for x in p) for p in pool[:4]]
+    hout = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+    dq, dk, dv = (torch.empty_like(x) for x in pool[0])
+    bi = sum(x.numel() * x.element_size() for x in hpool[0])
+    bo = hout.numel() * hout.element_size()
+    Ke = max(1, min(K, 1000))
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for i in range(Ke):
+        hq, hk, hv = hpool[i % len(hpool)]
+        dq.copy_(hq, non_blocking=True)
+        dk.copy_(hk, non_blocking=True)
+        dv.copy_(hv, non_blocking=True)
+        kvr.kvr_decode_step(cache.handle, 0, L, dq, dk, dv, out, B, W, stream)
+        hout.copy_(out, non_blocking=True)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1)
+    cache.sync_status()
+
+    unit_bytes = cost_model.step_unit_bytes(B + W, d, G, 2, 2, B, W)
+    launch_bytes = unit_bytes * S * L * H
+    return dict(total_ms=total_ms, per_launch_ms=per_launch_ms, K=K,
+                first_ms=first_ms, clocks=clocks, e2e_ms=e2e_ms, Ke=Ke,
+                bi=bi, bo=bo, launch_bytes=launch_bytes, lens=lens,
+                launches=launches)
+
+
+def main():
+    args = parse()
+    w = inputs.WORKLOADS[args.workload]
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        if rank != 0:
+            return 0
+        budget = 60.0
+        rate, n, spent = oracle_rate(w, args.seed, budget,
+                                     max_steps=max(1, args.steps))
+        line = {
+            "impl": "reference", "metric": metric_name(w), "value": rate,
+            "unit": "steps/s", "n_gpus": args.gpus, "steps": n,
+            "warmup": args.warmup, "ms_per_step": 1e3 / rate,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "f64", "data": "synthetic",
+            "config": {"workload": args.workload, "n_seq": w.n_seq,
+                       "layers": w.n_layers, "kv_heads": w.n_kv_heads,
+                       "group": w.group, "head_dim": w.head_dim,
+                       "budget": w.budget, "window": w.window},
+            "cpu_baseline": {"value": rate, "unit": "steps/s", "cores": 1,
+                             "kind": "oracle",
+                             "sample": f"{n} steady-state steps of 1 of the "
+                                       f"{w.n_seq} sequences ({spent:.1f} s), "
+                                       f"scaled x{w.n_seq}"},
+            "e2e": {"value": rate, "unit": "steps/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0},
+        }
+        print(json.dumps(line))
+        return 0
+
+    import torch
+    if world > 1:
+        torch.distributed.init_process_group("nccl")
+    r = run_kvr(args, rank, world, local_rank)
+    if rank != 0:
+        if world > 1:
+            torch.distributed.destroy_process_group()
+        return 0
+
+    peaks, peak_kind = measured_peaks()
+    peak = float(peaks["hbm_gbs"])
+    steps_per_s = world * r["K"] / (r["total_ms"] / 1e3)
+    achieved = r["launch_bytes"] / (r["per_launch_ms"] / 1e3) / 1e9
+    cpu = None
+    if world == 1 and not args.no_cpu_baseline:
+        rate, n, spent = oracle_rate(w, args.seed, args.cpu_seconds)
+        cpu = {"value": rate, "unit": "steps/s", "cores": 1, "kind": "oracle",
+               "sample": f"{n} steady-state steps of 1 of the {w.n_seq} "
+                         f"sequences ({spent:.1f} s of fp64 oracle), scaled "
+                         f"x{w.n_seq}"}
+    line = {
+        "metric": metric_name(w), "value": steps_per_s, "unit": "steps/s",
+        "n_gpus": world, "steps": r["K"], "warmup": args.warmup,
+        "ms_per_step": r["total_ms"] / r["K"], "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic",
+        "config": {"workload": args.workload, "n_seq": w.n_seq,
+                   "layers": w.n_layers, "kv_heads": w.n_kv_heads,
+                   "group": w.group, "head_dim": w.head_dim,
+                   "budget": w.budget, "window": w.window,
+                   "prior_len": "U[512,16384]", "elem": "bf16",
+                   "l2": f"inputs larger than L2: {r['launch_bytes'] / 1e6:.0f} MB"
+                         " touched per step, no flush",
+                   "per_rank_sequences": w.n_seq},
+        "hbm_gbs": achieved,
+        "hbm_frac_of_8tbs": achieved / NOMINAL_HBM_GBS,
+        "first_step_ms": r["first_ms"],
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak,
+                     "unit": "GB/s", "frac": achieved / peak,
+                     "peak_kind": peak_kind,
+                     "traffic": committed_traffic(args.workload),
+                     "algorithmic_bytes_per_launch": r["launch_bytes"],
+                     "launch_ms": r["per_launch_ms"],
+                     "kernel": "kvr_decode_step (all layers, one call)"},
+        "e2e": {"value": world * r["Ke"] / (r["e2e_ms"] / 1e3),
+                "unit": "steps/s", "h2d_bytes_per_step": r["bi"],
+                "d2h_bytes_per_step": r["bo"]},
+        "gpu_launches": r["launches"],
+        "clocks": r["clocks"],
+        "cpu_baseline": cpu,
+    }
+    print(json.dumps(line))
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,160 @@
+/*
+ * kvr.h -- C ABI of libkvr: the evicted-KV decode step of KV-Rescue
+ * (arXiv 2608.15797) on one GB300 (sm_103a).
+ *
+ * The operation (Sec. 2.1, Eq. 1): at decode step t each layer keeps, per KV
+ * head, a budgeted cache C_t^B of key/value rows.  The step
+ *   1. appends the new token's (k_t, v_t),
+ *   2. computes Attn(q_t, C) for the G query heads that share the KV head
+ *      (grouped-query attention; softmax scale 1/sqrt(d) by default),
+ *   3. adds to every live row's importance score s_i ("accumulated attention",
+ *      Sec. 2.1) the mean over the G query heads of that row's probability,
+ *   4. once the live length exceeds B' = B + W (App. C: eviction "fires every
+ *      step once l > B'"), keeps the W most recent rows (the protected window
+ *      of Sec. 4.1 / App. Impl.) plus the B best-scored others (TopB of Eq. 1;
+ *      equal scores keep the lower position) and compacts K/V in place.
+ * Candidates (Sec. 2.2 Eq. 2, App. Impl. "Best-of-(N+N)") fork from one cache
+ * state, share its rows as a read-only prefix, decode a step each, and one of
+ * them is committed back (Algorithm 1, "retain the selected base fork").
+ *
+ * Conventions for every call below:
+ *  - A "unit" is one (sequence, layer, KV head).  Query head j of a layer
+ *    uses KV head j / G.
+ *  - Device pointers ("dev") are caller-owned CUDA device memory; host
+ *    pointers ("host") are caller-owned host memory.  The library never
+ *    allocates device memory: a handle owns only host metadata.
+ *  - Tensors are dense row-major with the shapes given; element type is the
+ *    descriptor's kv_dtype unless stated (out_dtype for outputs).
+ *  - "stream" is a cudaStream_t (NULL = legacy default stream).  Calls are
+ *    asynchronous and stream-ordered unless marked "synchronising".
+ *  - Errors are returned as kvr_status, never thrown; kvr_last_error() gives
+ *    a thread-local message for the last failing call.  Argument and capacity
+ *    errors are detected on the host before anything is enqueued (the handle
+ *    keeps a host mirror of every live length).  Errors found by a kernel
+ *    (non-finite logits, an inconsistent length) set a device error word that
+ *    kvr_sync_status() reports as KVR_EDEVICE.
+ *  - Slot order inside a unit is not part of the contract: rows are
+ *    identified by their position (token index).
+ */
+#ifndef KVR_H
+#define KVR_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  KVR_OK = 0,
+  KVR_EINVAL = 1,    /* bad argument (null pointer, range, unsupported shape) */
+  KVR_ENOMEM = 2,    /* caller-provided buffer smaller than required */
+  KVR_ECAPACITY = 3, /* appended rows would exceed the unit capacity */
+  KVR_ECUDA = 4,     /* a CUDA runtime call failed */
+  KVR_EDEVICE = 5,   /* a kernel set the device error word */
+  KVR_ESTATE = 6     /* call not valid in the handle's current state */
+} kvr_status;
+
+typedef enum { KVR_BF16 = 0, KVR_F32 = 1 } kvr_dtype;
+
+typedef struct {
+  int n_seq;           /* S, sequences in the batch (>= 1) */
+  int n_layers;        /* L (>= 1) */
+  int n_kv_heads;      /* H, KV heads per layer (>= 1) */
+  int group;           /* G = query heads per KV head, 1..8 */
+  int head_dim;        /* d: 64 or 128 */
+  int capacity;        /* rows per unit slab (>= 1) */
+  kvr_dtype kv_dtype;  /* K, V, q, k_new, v_new element type */
+  kvr_dtype out_dtype; /* attention output element type */
+  float softmax_scale; /* 0 selects 1/sqrt(d) */
+} kvr_cache_desc;
+
+typedef struct kvr_cache kvr_cache; /* opaque; host metadata only */
+typedef struct kvr_fork kvr_fork;   /* opaque; host metadata only */
+
+/* ---- cache lifetime ---------------------------------------------------- */
+
+/* Bytes of device memory a cache with this descriptor needs (0 if the
+ * descriptor is invalid).  The buffer holds, per unit, the K and V slabs
+ * [capacity][d], the fp32 scores and int32 positions [capacity], the live
+ * length and next position, a logit scratch area [G][capacity] fp32 used when
+ * a unit is too long for on-chip memory, and a device error word. */
+size_t kvr_cache_required_bytes(const kvr_cache_desc *desc);
+
+/* Create a cache over dev_buf (>= kvr_cache_required_bytes, 256-byte
+ * aligned; owned by the caller and must outlive the handle).  Every unit
+ * starts empty at position 0.  The initialisation is enqueued on stream. */
+kvr_status kvr_cache_create(const kvr_cache_desc *desc, void *dev_buf,
+                            size_t bytes, void *stream, kvr_cache **out);
+
+/* Free the handle's host metadata (not the device buffer). NULL is a no-op. */
+void kvr_cache_destroy(kvr_cache *cache);
+
+/* Load a prompt into sequence seq of every layer and KV head:
+ * k, v dev [L][H][n_rows][d].  Rows get positions first_pos..first_pos+n-1
+ * and score 0 (no prefill scoring: the first decode step supplies the first
+ * scores).  Replaces whatever the sequence held.  n_rows <= capacity. */
+kvr_status kvr_cache_load(kvr_cache *cache, int seq, const void *k,
+                          const void *v, int n_rows, int first_pos,
+                          void *stream);
+
+/* ---- the decode step --------------------------------------------------- */
+
+/* Steps 1-3 for layers [layer_begin, layer_end) of every sequence: append,
+ * attend, accumulate scores; no eviction.  nl = layer_end - layer_begin.
+ *   q     dev [S][nl][H*G][d]
+ *   k_new dev [S][nl][H][d], v_new dev [S][nl][H][d]
+ *   out   dev [S][nl][H*G][d] (out_dtype)
+ * Needs one free row per unit (KVR_ECAPACITY otherwise). */
+kvr_status kvr_decode_attend_score(kvr_cache *cache, int layer_begin,
+                                   int layer_end, const void *q,
+                                   const void *k_new, const void *v_new,
+                                   void *out, void *stream);
+
+/* Step 4 alone for layers [layer_begin, layer_end): every unit longer than
+ * budget + window is cut back to budget + window rows (window = the W most
+ * recent positions, always kept; TopB of the rest; ties keep the lower
+ * position), compacting K, V, scores and positions in place.
+ * budget >= 0, window >= 0, budget + window >= 1. */
+kvr_status kvr_evict_compact(kvr_cache *cache, int layer_begin, int layer_end,
+                             int budget, int window, void *stream);
+
+/* Steps 1-4 fused in one pass: equivalent to kvr_decode_attend_score
+ * followed by kvr_evict_compact, with the appended row written straight into
+ * the slot the eviction frees. */
+kvr_status kvr_decode_step(kvr_cache *cache, int layer_begin, int layer_end,
+                           const void *q, const void *k_new, const void *v_new,
+                           void *out, int budget, int window, void *stream);
+
+/* ---- inspection -------------------------------------------------------- */
+
+/* Synchronising: wait for stream, then copy sequence seq's state to host.
+ * host_k, host_v [L][H][capacity][d] (kv_dtype); host_score [L][H][capacity]
+ * fp32; host_pos [L][H][capacity] int32; host_len and host_next_pos [L][H]
+ * int32 (live length; position the next appended row will get).  Any pointer
+ * may be NULL.  Slots at or beyond a unit's length hold stale data. */
+kvr_status kvr_cache_export(const kvr_cache *cache, int seq, void *host_k,
+                            void *host_v, float *host_score, int32_t *host_pos,
+                            int32_t *host_len, int32_t *host_next_pos,
+                            void *stream);
+
+/* Host mirror of the live length of every (sequence, layer): host_len
+ * [S][L].  Not synchronising (the mirror is exact after every call). */
+kvr_status kvr_cache_lengths(const kvr_cache *cache, int32_t *host_len);
+
+/* Number of kernels this handle has launched since it was created (each
+ * call adds the kernels it enqueued; memsets are not counted). */
+kvr_status kvr_cache_launch_count(const kvr_cache *cache, uint64_t *count);
+
+/* Synchronising: wait for stream, read and clear the device error word.
+ * KVR_OK if no kernel reported an error since the last call. */
+kvr_status kvr_sync_status(kvr_cache *cache, void *stream);
+
+/* Message of the last failing call on this thread ("" if none). */
+const char *kvr_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* KVR_H */

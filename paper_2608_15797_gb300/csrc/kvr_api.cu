@@ -1,0 +1,362 @@
+// kvr_api.cu -- the C ABI of libkvr (include/kvr.h): argument validation,
+// the host mirror of every live length, carving of the caller's device
+// buffer, and kernel dispatch.  No device memory is allocated here.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "../../include/kvr.h"
+#include "kvr_internal.h"
+
+using kvr::CacheView;
+using kvr::StepArgs;
+
+namespace {
+
+thread_local std::string g_err;
+
+kvr_status fail(kvr_status st, const char *fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  g_err = buf;
+  return st;
+}
+
+kvr_status cuda_fail(const char *where, cudaError_t e) {
+  return fail(KVR_ECUDA, "%s: %s", where, cudaGetErrorString(e));
+}
+
+constexpr size_t kAlign = 256;
+size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+
+int esize(kvr_dtype t) { return t == KVR_BF16 ? 2 : 4; }
+
+bool desc_ok(const kvr_cache_desc *d) {
+  if (!d) return false;
+  if (d->n_seq < 1 || d->n_layers < 1 || d->n_kv_heads < 1) return false;
+  if (d->group < 1 || d->group > 8) return false;
+  if (d->head_dim != 64 && d->head_dim != 128) return false;
+  if (d->capacity < 1 || d->capacity > (1 << 24)) return false;
+  if (d->kv_dtype != KVR_BF16 && d->kv_dtype != KVR_F32) return false;
+  if (d->out_dtype != KVR_BF16 && d->out_dtype != KVR_F32) return false;
+  if (!(d->softmax_scale >= 0.f) || !std::isfinite(d->softmax_scale))
+    return false;
+  return true;
+}
+
+// Byte offsets of every array inside the cache buffer.
+struct Layout {
+  size_t K, V, score, pos, len, next_pos, err, logits, total;
+};
+
+Layout layout_of(const kvr_cache_desc *d) {
+  const size_t units = (size_t)d->n_seq * d->n_layers * d->n_kv_heads;
+  const size_t rows = units * (size_t)d->capacity;
+  Layout l{};
+  size_t off = 0;
+  l.K = off;
+  off = align_up(off + rows * d->head_dim * esize(d->kv_dtype));
+  l.V = off;
+  off = align_up(off + rows * d->head_dim * esize(d->kv_dtype));
+  l.score = off;
+  off = align_up(off + rows * sizeof(float));
+  l.pos = off;
+  off = align_up(off + rows * sizeof(int32_t));
+  l.len = off;
+  off = align_up(off + units * sizeof(int32_t));
+  l.next_pos = off;
+  off = align_up(off + units * sizeof(int32_t));
+  l.err = off;
+  off = align_up(off + 16);
+  l.logits = off;
+  off = align_up(off + rows * d->group * sizeof(float));
+  l.total = off;
+  return l;
+}
+
+}  // namespace
+
+struct kvr_cache {
+  kvr_cache_desc desc;
+  CacheView view;
+  std::vector<int32_t> len;       // host mirror [S][L]
+  std::vector<int32_t> next_pos;  // host mirror [S][L]
+  size_t bytes;
+  uint64_t launches = 0;          // kernels launched through this handle
+};
+
+namespace {
+
+cudaStream_t as_stream(void *s) { return reinterpret_cast<cudaStream_t>(s); }
+
+kvr_status check_layers(const kvr_cache *c, int lb, int le) {
+  if (lb < 0 || le > c->desc.n_layers || lb >= le)
+    return fail(KVR_EINVAL, "layer range [%d, %d) outside [0, %d)", lb, le,
+                c->desc.n_layers);
+  return KVR_OK;
+}
+
+// Largest live length over (all sequences) x (layers [lb, le)).
+int max_len(const kvr_cache *c, int lb, int le) {
+  int m = 0;
+  for (int s = 0; s < c->desc.n_seq; ++s)
+    for (int l = lb; l < le; ++l)
+      m = std::max(m, c->len[(size_t)s * c->desc.n_layers + l]);
+  return m;
+}
+
+kvr_status check_step(kvr_cache *c, int lb, int le, const void *q,
+                      const void *k_new, const void *v_new, void *out) {
+  if (!c) return fail(KVR_EINVAL, "null cache");
+  kvr_status st = check_layers(c, lb, le);
+  if (st != KVR_OK) return st;
+  if (!q || !k_new || !v_new || !out)
+    return fail(KVR_EINVAL, "null q, k_new, v_new or out");
+  const int m = max_len(c, lb, le);
+  if (m + 1 > c->desc.capacity)
+    return fail(KVR_ECAPACITY, "a unit holds %d rows; capacity %d is full", m,
+                c->desc.capacity);
+  for (int s = 0; s < c->desc.n_seq; ++s)
+    for (int l = lb; l < le; ++l)
+      if (c->next_pos[(size_t)s * c->desc.n_layers + l] == INT32_MAX)
+        return fail(KVR_ECAPACITY, "position counter exhausted");
+  return KVR_OK;
+}
+
+kvr_status check_evict(int budget, int window) {
+  if (budget < 0 || window < 0 || (long long)budget + window < 1 ||
+      (long long)budget + window > (1 << 24))
+    return fail(KVR_EINVAL, "bad budget %d / window %d", budget, window);
+  return KVR_OK;
+}
+
+void mirror_append(kvr_cache *c, int lb, int le) {
+  for (int s = 0; s < c->desc.n_seq; ++s)
+    for (int l = lb; l < le; ++l) {
+      const size_t i = (size_t)s * c->desc.n_layers + l;
+      c->len[i] += 1;
+      c->next_pos[i] += 1;
+    }
+}
+
+void mirror_evict(kvr_cache *c, int lb, int le, int budget, int window) {
+  for (int s = 0; s < c->desc.n_seq; ++s)
+    for (int l = lb; l < le; ++l) {
+      int32_t &n = c->len[(size_t)s * c->desc.n_layers + l];
+      n = std::min<long long>(n, (long long)budget + window);
+    }
+}
+
+StepArgs step_args(const kvr_cache *c, int lb, int le, const void *q,
+                   const void *k_new, const void *v_new, void *out) {
+  StepArgs a{};
+  a.lb = lb;
+  a.nl = le - lb;
+  a.q = q;
+  a.k_new = k_new;
+  a.v_new = v_new;
+  a.out = out;
+  a.max_rows = max_len(c, lb, le) + 1;
+  return a;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t kvr_cache_required_bytes(const kvr_cache_desc *desc) {
+  if (!desc_ok(desc)) return 0;
+  return layout_of(desc).total;
+}
+
+kvr_status kvr_cache_create(const kvr_cache_desc *desc, void *dev_buf,
+                            size_t bytes, void *stream, kvr_cache **out) {
+  if (!out) return fail(KVR_EINVAL, "null output handle");
+  *out = nullptr;
+  if (!desc_ok(desc)) return fail(KVR_EINVAL, "invalid cache descriptor");
+  if (!dev_buf) return fail(KVR_EINVAL, "null device buffer");
+  if (reinterpret_cast<uintptr_t>(dev_buf) % kAlign)
+    return fail(KVR_EINVAL, "device buffer not %zu-byte aligned", kAlign);
+  const Layout lay = layout_of(desc);
+  if (bytes < lay.total)
+    return fail(KVR_ENOMEM, "buffer of %zu bytes < required %zu", bytes,
+                lay.total);
+  kvr_cache *c = new (std::nothrow) kvr_cache();
+  if (!c) return fail(KVR_ENOMEM, "host allocation failed");
+  c->desc = *desc;
+  c->bytes = bytes;
+  char *b = static_cast<char *>(dev_buf);
+  CacheView &v = c->view;
+  v.K = b + lay.K;
+  v.V = b + lay.V;
+  v.score = reinterpret_cast<float *>(b + lay.score);
+  v.pos = reinterpret_cast<int32_t *>(b + lay.pos);
+  v.len = reinterpret_cast<int32_t *>(b + lay.len);
+  v.next_pos = reinterpret_cast<int32_t *>(b + lay.next_pos);
+  v.err = reinterpret_cast<unsigned *>(b + lay.err);
+  v.logits = reinterpret_cast<float *>(b + lay.logits);
+  v.S = desc->n_seq;
+  v.L = desc->n_layers;
+  v.H = desc->n_kv_heads;
+  v.G = desc->group;
+  v.d = desc->head_dim;
+  v.cap = desc->capacity;
+  v.scale = desc->softmax_scale > 0.f
+                ? desc->softmax_scale
+                : (float)(1.0 / std::sqrt((double)desc->head_dim));
+  v.kv_bf16 = desc->kv_dtype == KVR_BF16;
+  v.out_bf16 = desc->out_dtype == KVR_BF16;
+  c->len.assign((size_t)v.S * v.L, 0);
+  c->next_pos.assign((size_t)v.S * v.L, 0);
+  cudaError_t e = kvr::launch_init(v, as_stream(stream));
+  if (e != cudaSuccess) {
+    delete c;
+    return cuda_fail("kvr_cache_create", e);
+  }
+  *out = c;
+  return KVR_OK;
+}
+
+void kvr_cache_destroy(kvr_cache *cache) { delete cache; }
+
+kvr_status kvr_cache_load(kvr_cache *c, int seq, const void *k, const void *v,
+                          int n_rows, int first_pos, void *stream) {
+  if (!c) return fail(KVR_EINVAL, "null cache");
+  if (seq < 0 || seq >= c->desc.n_seq)
+    return fail(KVR_EINVAL, "sequence %d outside [0, %d)", seq, c->desc.n_seq);
+  if (n_rows < 0 || first_pos < 0 ||
+      (long long)first_pos + n_rows >= INT32_MAX)
+    return fail(KVR_EINVAL, "bad prompt length %d / first position %d", n_rows,
+                first_pos);
+  if (n_rows > c->desc.capacity)
+    return fail(KVR_ECAPACITY, "prompt of %d rows > capacity %d", n_rows,
+                c->desc.capacity);
+  if (n_rows > 0 && (!k || !v)) return fail(KVR_EINVAL, "null k or v");
+  if ((reinterpret_cast<uintptr_t>(k) | reinterpret_cast<uintptr_t>(v)) % 16)
+    return fail(KVR_EINVAL, "k and v must be 16-byte aligned");
+  cudaError_t e =
+      kvr::launch_load(c->view, seq, k, v, n_rows, first_pos, as_stream(stream));
+  if (e != cudaSuccess) return cuda_fail("kvr_cache_load", e);
+  c->launches += 1;
+  for (int l = 0; l < c->desc.n_layers; ++l) {
+    c->len[(size_t)seq * c->desc.n_layers + l] = n_rows;
+    c->next_pos[(size_t)seq * c->desc.n_layers + l] = first_pos + n_rows;
+  }
+  return KVR_OK;
+}
+
+kvr_status kvr_decode_attend_score(kvr_cache *c, int lb, int le, const void *q,
+                                   const void *k_new, const void *v_new,
+                                   void *out, void *stream) {
+  kvr_status st = check_step(c, lb, le, q, k_new, v_new, out);
+  if (st != KVR_OK) return st;
+  StepArgs a = step_args(c, lb, le, q, k_new, v_new, out);
+  cudaError_t e =
+      kvr::launch_attend_score_generic(c->view, a, as_stream(stream));
+  if (e != cudaSuccess) return cuda_fail("kvr_decode_attend_score", e);
+  c->launches += 1;
+  mirror_append(c, lb, le);
+  return KVR_OK;
+}
+
+kvr_status kvr_evict_compact(kvr_cache *c, int lb, int le, int budget,
+                             int window, void *stream) {
+  if (!c) return fail(KVR_EINVAL, "null cache");
+  kvr_status st = check_layers(c, lb, le);
+  if (st != KVR_OK) return st;
+  st = check_evict(budget, window);
+  if (st != KVR_OK) return st;
+  const int m = max_len(c, lb, le);
+  if (m <= budget + window) return KVR_OK;  // nothing exceeds B + W
+  cudaError_t e = kvr::launch_evict_generic(c->view, lb, le - lb, m, budget,
+                                            window, as_stream(stream));
+  if (e != cudaSuccess) return cuda_fail("kvr_evict_compact", e);
+  c->launches += 1;
+  mirror_evict(c, lb, le, budget, window);
+  return KVR_OK;
+}
+
+kvr_status kvr_decode_step(kvr_cache *c, int lb, int le, const void *q,
+                           const void *k_new, const void *v_new, void *out,
+                           int budget, int window, void *stream) {
+  kvr_status st = check_step(c, lb, le, q, k_new, v_new, out);
+  if (st != KVR_OK) return st;
+  st = check_evict(budget, window);
+  if (st != KVR_OK) return st;
+  st = kvr_decode_attend_score(c, lb, le, q, k_new, v_new, out, stream);
+  if (st != KVR_OK) return st;
+  return kvr_evict_compact(c, lb, le, budget, window, stream);
+}
+
+kvr_status kvr_cache_export(const kvr_cache *c, int seq, void *host_k,
+                            void *host_v, float *host_score, int32_t *host_pos,
+                            int32_t *host_len, int32_t *host_next_pos,
+                            void *stream) {
+  if (!c) return fail(KVR_EINVAL, "null cache");
+  if (seq < 0 || seq >= c->desc.n_seq)
+    return fail(KVR_EINVAL, "sequence %d outside [0, %d)", seq, c->desc.n_seq);
+  cudaError_t e = cudaStreamSynchronize(as_stream(stream));
+  if (e != cudaSuccess) return cuda_fail("kvr_cache_export: sync", e);
+  const CacheView &v = c->view;
+  const size_t units = (size_t)v.L * v.H, rows = units * v.cap;
+  const size_t ebytes = (size_t)v.d * esize(c->desc.kv_dtype);
+  struct {
+    void *dst;
+    const void *src;
+    size_t bytes;
+  } copies[] = {
+      {host_k, static_cast<char *>(v.K) + seq * rows * ebytes, rows * ebytes},
+      {host_v, static_cast<char *>(v.V) + seq * rows * ebytes, rows * ebytes},
+      {host_score, v.score + seq * rows, rows * sizeof(float)},
+      {host_pos, v.pos + seq * rows, rows * sizeof(int32_t)},
+      {host_len, v.len + seq * units, units * sizeof(int32_t)},
+      {host_next_pos, v.next_pos + seq * units, units * sizeof(int32_t)},
+  };
+  for (auto &cp : copies) {
+    if (!cp.dst) continue;
+    e = cudaMemcpy(cp.dst, cp.src, cp.bytes, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail("kvr_cache_export", e);
+  }
+  return KVR_OK;
+}
+
+kvr_status kvr_cache_lengths(const kvr_cache *c, int32_t *host_len) {
+  if (!c || !host_len) return fail(KVR_EINVAL, "null argument");
+  std::memcpy(host_len, c->len.data(), c->len.size() * sizeof(int32_t));
+  return KVR_OK;
+}
+
+kvr_status kvr_cache_launch_count(const kvr_cache *c, uint64_t *count) {
+  if (!c || !count) return fail(KVR_EINVAL, "null argument");
+  *count = c->launches;
+  return KVR_OK;
+}
+
+kvr_status kvr_sync_status(kvr_cache *c, void *stream) {
+  if (!c) return fail(KVR_EINVAL, "null cache");
+  cudaError_t e = cudaStreamSynchronize(as_stream(stream));
+  if (e != cudaSuccess) return cuda_fail("kvr_sync_status: sync", e);
+  unsigned word = 0;
+  e = cudaMemcpy(&word, c->view.err, sizeof word, cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail("kvr_sync_status: read", e);
+  if (!word) return KVR_OK;
+  e = cudaMemset(c->view.err, 0, sizeof word);
+  if (e != cudaSuccess) return cuda_fail("kvr_sync_status: clear", e);
+  return fail(KVR_EDEVICE, "device error word 0x%x (%s%s%s)", word,
+              word & kvr::ERR_CAPACITY ? "capacity " : "",
+              word & kvr::ERR_NONFINITE ? "non-finite " : "",
+              word & kvr::ERR_LENGTH ? "length" : "");
+}
+
+const char *kvr_last_error(void) { return g_err.c_str(); }
+
+}  // extern "C"

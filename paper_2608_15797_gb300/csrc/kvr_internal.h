@@ -1,0 +1,56 @@
+// kvr_internal.h -- shared between the C-ABI host code and the kernels of
+// libkvr.  Not installed; not part of the ABI.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace kvr {
+
+// Device error word bits (set with atomicOr, read by kvr_sync_status).
+enum : unsigned {
+  ERR_CAPACITY = 1u,   // a unit had no free row for the append
+  ERR_NONFINITE = 2u,  // a softmax normaliser was not finite
+  ERR_LENGTH = 4u,     // an eviction produced an unexpected live length
+};
+
+// Device view of one cache: every pointer points into the caller's buffer.
+struct CacheView {
+  void *K;          // [S][L][H][cap][d] kv element type
+  void *V;          // [S][L][H][cap][d]
+  float *score;     // [S][L][H][cap]
+  int32_t *pos;     // [S][L][H][cap]
+  int32_t *len;     // [S][L][H]
+  int32_t *next_pos;// [S][L][H]
+  unsigned *err;    // device error word
+  float *logits;    // [S][L][H][G][cap] scratch for units beyond on-chip size
+  int S, L, H, G, d, cap;
+  float scale;      // softmax scale (1/sqrt(d) by default)
+  int kv_bf16;      // 1: bf16 elements, 0: fp32
+  int out_bf16;     // 1: bf16 output, 0: fp32
+};
+
+// Work description of one decode call over layers [lb, lb + nl).
+struct StepArgs {
+  int lb, nl;
+  const void *q;      // [S][nl][H*G][d]
+  const void *k_new;  // [S][nl][H][d]
+  const void *v_new;  // [S][nl][H][d]
+  void *out;          // [S][nl][H*G][d]
+  int max_rows;       // largest live length after the append over the units
+  int budget, window; // eviction target (evict only when evict != 0)
+  int evict;
+};
+
+// Generic kernels (any d in {64,128}, G <= 8, fp32 or bf16): one CTA per unit.
+cudaError_t launch_attend_score_generic(const CacheView &c, const StepArgs &a,
+                                        cudaStream_t st);
+cudaError_t launch_evict_generic(const CacheView &c, int lb, int nl,
+                                 int max_rows, int budget, int window,
+                                 cudaStream_t st);
+cudaError_t launch_load(const CacheView &c, int seq, const void *k,
+                        const void *v, int n_rows, int first_pos,
+                        cudaStream_t st);
+cudaError_t launch_init(const CacheView &c, cudaStream_t st);
+
+}  // namespace kvr

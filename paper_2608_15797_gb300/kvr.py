@@ -1,0 +1,268 @@
+"""Thin Python binding of libkvr (include/kvr.h) over ctypes.
+
+Argument marshalling only: every step of the decode path runs in the CUDA
+kernels of libkvr.so.  Functions keep the C names; torch tensors are passed by
+their data pointers, and the stream defaults to torch's current CUDA stream.
+Importing this module fails loudly if libkvr.so has not been built.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libkvr.so")
+
+if not os.path.exists(LIB_PATH):
+    raise ImportError(
+        f"libkvr.so not found at {LIB_PATH}: build it with "
+        "`python -c 'import __graft_entry__ as g; g.build()'` (there is no "
+        "fallback implementation)")
+
+lib = ctypes.CDLL(LIB_PATH)
+
+KVR_OK, KVR_EINVAL, KVR_ENOMEM, KVR_ECAPACITY, KVR_ECUDA, KVR_EDEVICE, \
+    KVR_ESTATE = range(7)
+STATUS_NAMES = {0: "KVR_OK", 1: "KVR_EINVAL", 2: "KVR_ENOMEM",
+                3: "KVR_ECAPACITY", 4: "KVR_ECUDA", 5: "KVR_EDEVICE",
+                6: "KVR_ESTATE"}
+KVR_BF16, KVR_F32 = 0, 1
+DTYPES = {"bf16": KVR_BF16, "f32": KVR_F32}
+TORCH_DTYPES = {"bf16": torch.bfloat16, "f32": torch.float32}
+
+
+class KvrError(RuntimeError):
+    def __init__(self, status: int, where: str, msg: str):
+        super().__init__(f"{where}: {STATUS_NAMES.get(status, status)}: {msg}")
+        self.status = status
+
+
+class kvr_cache_desc(ctypes.Structure):
+    _fields_ = [("n_seq", ctypes.c_int), ("n_layers", ctypes.c_int),
+                ("n_kv_heads", ctypes.c_int), ("group", ctypes.c_int),
+                ("head_dim", ctypes.c_int), ("capacity", ctypes.c_int),
+                ("kv_dtype", ctypes.c_int), ("out_dtype", ctypes.c_int),
+                ("softmax_scale", ctypes.c_float)]
+
+
+_P = ctypes.c_void_p
+_I = ctypes.c_int
+_S = ctypes.c_int
+
+_SIGS = {
+    "kvr_cache_required_bytes": (ctypes.c_size_t, [ctypes.POINTER(kvr_cache_desc)]),
+    "kvr_cache_create": (_S, [ctypes.POINTER(kvr_cache_desc), _P, ctypes.c_size_t,
+                              _P, ctypes.POINTER(_P)]),
+    "kvr_cache_destroy": (None, [_P]),
+    "kvr_cache_load": (_S, [_P, _I, _P, _P, _I, _I, _P]),
+    "kvr_decode_attend_score": (_S, [_P, _I, _I, _P, _P, _P, _P, _P]),
+    "kvr_evict_compact": (_S, [_P, _I, _I, _I, _I, _P]),
+    "kvr_decode_step": (_S, [_P, _I, _I, _P, _P, _P, _P, _I, _I, _P]),
+    "kvr_cache_export": (_S, [_P, _I, _P, _P, _P, _P, _P, _P, _P]),
+    "kvr_cache_lengths": (_S, [_P, _P]),
+    "kvr_cache_launch_count": (_S, [_P, _P]),
+    "kvr_sync_status": (_S, [_P, _P]),
+    "kvr_last_error": (ctypes.c_char_p, []),
+}
+for _name, (_res, _args) in _SIGS.items():
+    _f = getattr(lib, _name)
+    _f.restype = _res
+    _f.argtypes = _args
+
+
+def kvr_last_error() -> str:
+    return lib.kvr_last_error().decode()
+
+
+def _check(status: int, where: str):
+    if status != KVR_OK:
+        raise KvrError(status, where, kvr_last_error())
+
+
+def _stream(stream):
+    if stream is None:
+        return ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    if isinstance(stream, torch.cuda.Stream):
+        return ctypes.c_void_p(stream.cuda_stream)
+    return ctypes.c_void_p(int(stream))
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    if isinstance(t, torch.Tensor):
+        if not t.is_contiguous():
+            raise ValueError("tensors passed to libkvr must be contiguous")
+        return ctypes.c_void_p(t.data_ptr())
+    if isinstance(t, np.ndarray):
+        if not t.flags["C_CONTIGUOUS"]:
+            raise ValueError("arrays passed to libkvr must be C-contiguous")
+        return t.ctypes.data_as(ctypes.c_void_p)
+    return ctypes.c_void_p(int(t))
+
+
+def make_desc(n_seq, n_layers, n_kv_heads, group, head_dim, capacity,
+              kv_dtype="bf16", out_dtype="bf16", softmax_scale=0.0):
+    return kvr_cache_desc(n_seq, n_layers, n_kv_heads, group, head_dim,
+                          capacity, DTYPES[kv_dtype], DTYPES[out_dtype],
+                          float(softmax_scale))
+
+
+def kvr_cache_required_bytes(desc: kvr_cache_desc) -> int:
+    return int(lib.kvr_cache_required_bytes(ctypes.byref(desc)))
+
+
+def kvr_cache_create(desc, dev_buf, nbytes, stream=None):
+    h = ctypes.c_void_p()
+    _check(lib.kvr_cache_create(ctypes.byref(desc), _ptr(dev_buf), nbytes,
+                                _stream(stream), ctypes.byref(h)),
+           "kvr_cache_create")
+    return h
+
+
+def kvr_cache_destroy(h):
+    lib.kvr_cache_destroy(h)
+
+
+def kvr_cache_load(h, seq, k, v, n_rows, first_pos=0, stream=None):
+    _check(lib.kvr_cache_load(h, seq, _ptr(k), _ptr(v), n_rows, first_pos,
+                              _stream(stream)), "kvr_cache_load")
+
+
+def kvr_decode_attend_score(h, layer_begin, layer_end, q, k_new, v_new, out,
+                            stream=None):
+    _check(lib.kvr_decode_attend_score(h, layer_begin, layer_end, _ptr(q),
+                                       _ptr(k_new), _ptr(v_new), _ptr(out),
+                                       _stream(stream)),
+           "kvr_decode_attend_score")
+
+
+def kvr_evict_compact(h, layer_begin, layer_end, budget, window, stream=None):
+    _check(lib.kvr_evict_compact(h, layer_begin, layer_end, budget, window,
+                                 _stream(stream)), "kvr_evict_compact")
+
+
+def kvr_decode_step(h, layer_begin, layer_end, q, k_new, v_new, out, budget,
+                    window, stream=None):
+    _check(lib.kvr_decode_step(h, layer_begin, layer_end, _ptr(q), _ptr(k_new),
+                               _ptr(v_new), _ptr(out), budget, window,
+                               _stream(stream)), "kvr_decode_step")
+
+
+def kvr_cache_export(h, seq, host_k, host_v, host_score, host_pos, host_len,
+                     host_next_pos, stream=None):
+    _check(lib.kvr_cache_export(h, seq, _ptr(host_k), _ptr(host_v),
+                                _ptr(host_score), _ptr(host_pos),
+                                _ptr(host_len), _ptr(host_next_pos),
+                                _stream(stream)), "kvr_cache_export")
+
+
+def kvr_cache_lengths(h, host_len):
+    _check(lib.kvr_cache_lengths(h, _ptr(host_len)), "kvr_cache_lengths")
+
+
+def kvr_cache_launch_count(h) -> int:
+    n = ctypes.c_uint64()
+    _check(lib.kvr_cache_launch_count(h, ctypes.byref(n)),
+           "kvr_cache_launch_count")
+    return int(n.value)
+
+
+def kvr_sync_status(h, stream=None):
+    _check(lib.kvr_sync_status(h, _stream(stream)), "kvr_sync_status")
+
+
+class Cache:
+    """Owner of one kvr_cache handle and the torch buffer it lives in."""
+
+    def __init__(self, n_seq, n_layers, n_kv_heads, group, head_dim, capacity,
+                 kv_dtype="bf16", out_dtype="bf16", softmax_scale=0.0,
+                 device="cuda", stream=None):
+        self.desc = make_desc(n_seq, n_layers, n_kv_heads, group, head_dim,
+                              capacity, kv_dtype, out_dtype, softmax_scale)
+        self.S, self.L, self.H, self.G, self.d = (n_seq, n_layers, n_kv_heads,
+                                                  group, head_dim)
+        self.cap = capacity
+        self.kv_dtype, self.out_dtype = kv_dtype, out_dtype
+        self.nbytes = kvr_cache_required_bytes(self.desc)
+        if self.nbytes == 0:
+            raise KvrError(KVR_EINVAL, "Cache", "invalid descriptor")
+        self.buf = torch.empty(self.nbytes, dtype=torch.uint8, device=device)
+        self.handle = kvr_cache_create(self.desc, self.buf, self.nbytes, stream)
+
+    def __del__(self):
+        h = getattr(self, "handle", None)
+        if h:
+            kvr_cache_destroy(h)
+            self.handle = None
+
+    @property
+    def kv_torch_dtype(self):
+        return TORCH_DTYPES[self.kv_dtype]
+
+    @property
+    def out_torch_dtype(self):
+        return TORCH_DTYPES[self.out_dtype]
+
+    def load(self, seq, k, v, first_pos=0, stream=None):
+        k = k.contiguous()
+        v = v.contiguous()
+        kvr_cache_load(self.handle, seq, k, v, k.shape[2], first_pos, stream)
+
+    def _layers(self, layers):
+        return (0, self.L) if layers is None else layers
+
+    def new_out(self, nl):
+        return torch.empty(self.S, nl, self.H * self.G, self.d,
+                           dtype=self.out_torch_dtype, device=self.buf.device)
+
+    def attend_score(self, q, k_new, v_new, out=None, layers=None, stream=None):
+        lb, le = self._layers(layers)
+        out = self.new_out(le - lb) if out is None else out
+        kvr_decode_attend_score(self.handle, lb, le, q, k_new, v_new, out,
+                                stream)
+        return out
+
+    def evict(self, budget, window, layers=None, stream=None):
+        lb, le = self._layers(layers)
+        kvr_evict_compact(self.handle, lb, le, budget, window, stream)
+
+    def step(self, q, k_new, v_new, budget, window, out=None, layers=None,
+             stream=None):
+        lb, le = self._layers(layers)
+        out = self.new_out(le - lb) if out is None else out
+        kvr_decode_step(self.handle, lb, le, q, k_new, v_new, out, budget,
+                        window, stream)
+        return out
+
+    def lengths(self):
+        a = np.zeros((self.S, self.L), np.int32)
+        kvr_cache_lengths(self.handle, a)
+        return a
+
+    def export(self, seq, kv=True, stream=None):
+        """Host copy of one sequence: dict of numpy arrays (K/V as float32)."""
+        rows = (self.L, self.H, self.cap)
+        score = np.zeros(rows, np.float32)
+        pos = np.zeros(rows, np.int32)
+        ln = np.zeros(rows[:2], np.int32)
+        npos = np.zeros(rows[:2], np.int32)
+        hk = hv = None
+        if kv:
+            hk = torch.empty(*rows, self.d, dtype=self.kv_torch_dtype).contiguous()
+            hv = torch.empty_like(hk)
+        kvr_cache_export(self.handle, seq, hk, hv, score, pos, ln, npos, stream)
+        res = {"score": score, "pos": pos, "len": ln, "next_pos": npos}
+        if kv:
+            res["K"] = hk.float().numpy()
+            res["V"] = hv.float().numpy()
+        return res
+
+    def launch_count(self):
+        return kvr_cache_launch_count(self.handle)
+
+    def sync_status(self, stream=None):
+        kvr_sync_status(self.handle, stream)

@@ -1,0 +1,66 @@
+"""Drivers that run the CUDA path and the fp64 oracle side by side.
+
+Test infrastructure: used by the GPU parity tests and by
+``__graft_entry__.smoke()``.  Inputs come from the seeded generators of
+``paper_2608_15797_gb300.inputs``; the CUDA path is driven through the C ABI
+(via the ctypes binding), the oracle through ``oracle.oracle``.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from oracle import oracle as orc
+from oracle import parity
+from paper_2608_15797_gb300 import inputs, kvr
+
+
+def dev(x: np.ndarray, dtype: str) -> torch.Tensor:
+    """Element-type-exact float32 host values -> device tensor of dtype."""
+    return torch.from_numpy(np.ascontiguousarray(x)).to(
+        device="cuda", dtype=kvr.TORCH_DTYPES[dtype])
+
+
+def make_pair(w: inputs.Workload, seed: int, S: int, cap: int,
+              prompt_lens=None, out_dtype="f32", first_pos=None):
+    """A CUDA cache and an oracle cache loaded with the same prompts."""
+    c = kvr.Cache(S, w.n_layers, w.n_kv_heads, w.group, w.head_dim, cap,
+                  kv_dtype=w.dtype, out_dtype=out_dtype)
+    o = orc.OracleCache(S, w.n_layers, w.n_kv_heads, w.group, w.head_dim, cap)
+    lens = [w.prompt] * S if prompt_lens is None else list(prompt_lens)
+    for s in range(S):
+        k, v = inputs.prompt(w, seed, s, int(lens[s]))
+        fp = 0 if first_pos is None else int(first_pos[s])
+        c.load(s, dev(k, w.dtype), dev(v, w.dtype), first_pos=fp)
+        o.load(s, k, v, first_pos=fp)
+    return c, o
+
+
+def lockstep(c: kvr.Cache, o: orc.OracleCache, w: inputs.Workload, seed: int,
+             steps: int, budget: int, window: int, fused: bool = True,
+             step0: int = 0, layers=None, evict: bool = True) -> parity.Stats:
+    """Run `steps` decode steps on both sides, checking after every step."""
+    S = c.S
+    stats = parity.Stats()
+    lb, le = (0, c.L) if layers is None else layers
+    for t in range(step0, step0 + steps):
+        q, kn, vn = inputs.step_inputs(w, seed, t, S, n_layers=le - lb)
+        qd, kd, vd = (dev(a, w.dtype) for a in (q, kn, vn))
+        if not evict:
+            out = c.attend_score(qd, kd, vd, layers=(lb, le))
+        elif fused:
+            out = c.step(qd, kd, vd, budget, window, layers=(lb, le))
+        else:
+            out = c.attend_score(qd, kd, vd, layers=(lb, le))
+            c.evict(budget, window, layers=(lb, le))
+        ref = o.step(q, kn, vn, evict=False, layer_begin=lb, layer_end=le)
+        torch.cuda.synchronize()
+        stats.max_out_excess = max(stats.max_out_excess, parity.check_out(
+            out.float().cpu().numpy(), ref, what=f"out at step {t}"))
+        exports = [c.export(s, kv=False) for s in range(S)]
+        st = parity.check_and_adopt(o, exports, budget, window, evict=evict,
+                                    layers=(lb, le))
+        stats.merge(st)
+        stats.steps = t - step0 + 1
+    c.sync_status()
+    return stats

@@ -1,0 +1,160 @@
+"""Parity of the CUDA decode step (through the C ABI) with the fp64 oracle.
+
+Tolerances (oracle/parity.py): outputs |d| <= 2e-3 + 1e-2 |ref|; scores of
+retained rows 1e-4 relative; retained sets exact up to swaps of oracle
+near-ties (1e-4 relative), ties to the lower position.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import oracle as orc
+from oracle import parity
+from paper_2608_15797_gb300 import inputs, kvr
+from tests import harness
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(autouse=True)
+def _cuda():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA device")
+    torch.cuda.set_device(0)
+
+
+def test_tiny_workload_full_run():
+    """Tiny: 1 layer, 4 q / 2 kv heads, d=64, fp32, prompt 128 (5% heavy
+    keys) then 256 steps at B=16, W=8; the first step evicts 105 rows."""
+    w = inputs.WORKLOADS["tiny"]
+    c, o = harness.make_pair(w, 0, 1, cap=w.prompt + 1)
+    st = harness.lockstep(c, o, w, 0, w.steps, w.budget, w.window)
+    assert st.steps == 256
+    assert (c.lengths() == w.budget + w.window).all()
+
+
+def test_7b_geometry_lockstep():
+    """Qwen2.5-Math-7B decode geometry (28 layers, G=7, d=128, bf16,
+    N(0,1)/sqrt(128)), prompt 512, B=64, W=8: 48 steps in lock-step."""
+    w = inputs.WORKLOADS["7b_b64"]
+    c, o = harness.make_pair(w, 2, 1, cap=w.prompt + 1)
+    st = harness.lockstep(c, o, w, 2, 48, w.budget, w.window)
+    assert st.units == 48 * 28 * 4
+
+
+def test_7b_unscaled_selection_exercised():
+    """Unscaled N(0,1) q/k: attention is peaked, so TopB decisions are far
+    from ties and must match the oracle exactly."""
+    w = inputs.WORKLOADS["7b_unscaled"]
+    c, o = harness.make_pair(w, 3, 2, cap=w.prompt + 1, prompt_lens=[512, 301])
+    st = harness.lockstep(c, o, w, 3, 24, w.budget, w.window)
+    assert st.adoptions == 0
+
+
+@pytest.mark.parametrize("G,d,dtype", [(1, 128, "bf16"), (8, 128, "bf16"),
+                                       (3, 64, "bf16"), (5, 64, "f32"),
+                                       (7, 128, "f32")])
+def test_group_sizes_and_dims(G, d, dtype):
+    w = inputs.Workload("g", 2, 3, G, d, dtype, 9, 3, 33, 10, sigma=1.0)
+    c, o = harness.make_pair(w, 4, 2, cap=40, prompt_lens=[33, 5])
+    harness.lockstep(c, o, w, 4, 10, w.budget, w.window)
+
+
+@pytest.mark.parametrize("B,W", [(1, 0), (0, 2), (5, 0), (1, 1), (30, 8)])
+def test_budget_window_edges(B, W):
+    w = inputs.Workload("e", 1, 2, 2, 128, "bf16", B, W, 20, 8, sigma=1.0)
+    c, o = harness.make_pair(w, 5, 2, cap=40, prompt_lens=[20, 1])
+    harness.lockstep(c, o, w, 5, 8, B, W)
+
+
+def test_empty_prompt_and_single_row():
+    """Decoding from an empty cache: the first step attends to its own row
+    only (out = v_new)."""
+    w = inputs.Workload("z", 1, 2, 3, 128, "bf16", 2, 1, 0, 6, sigma=1.0)
+    c, o = harness.make_pair(w, 6, 1, cap=8, prompt_lens=[0])
+    q, kn, vn = inputs.step_inputs(w, 6, 0, 1)
+    out = c.step(*(harness.dev(a, "bf16") for a in (q, kn, vn)), 2, 1)
+    np.testing.assert_allclose(out.float().cpu().numpy()[0, 0],
+                               np.repeat(vn[0, 0], 3, axis=0), rtol=0, atol=0)
+    o.step(q, kn, vn, B=2, W=1)
+    harness.lockstep(c, o, w, 6, 5, 2, 1, step0=1)
+
+
+def test_no_eviction_is_full_attention():
+    """B >= length: nothing is evicted and the output is full attention."""
+    w = inputs.Workload("f", 3, 2, 4, 128, "bf16", 1000, 8, 70, 20, sigma=1.0)
+    c, o = harness.make_pair(w, 7, 2, cap=100, prompt_lens=[70, 45])
+    harness.lockstep(c, o, w, 7, 20, w.budget, w.window)
+    assert c.lengths().tolist() == [[90] * 3, [65] * 3]
+
+
+def test_long_first_eviction():
+    """Prompts of ~[512, 16384] rows (the throughput workload's prior
+    lengths), first step evicting thousands of rows per unit; the longest
+    unit's logits exceed on-chip memory and go through the scratch area."""
+    w = inputs.Workload("long", 2, 2, 7, 128, "bf16", 64, 8, 0, 3, sigma=1.0)
+    lens = [9001, 600, 16384]
+    c, o = harness.make_pair(w, 8, 3, cap=16385, prompt_lens=lens)
+    st = harness.lockstep(c, o, w, 8, 3, 64, 8)
+    assert (c.lengths() == 72).all()
+
+
+def test_fused_equals_unfused_bitwise():
+    w = inputs.Workload("u", 3, 2, 7, 128, "bf16", 16, 4, 50, 6, sigma=1.0)
+    c1, _ = harness.make_pair(w, 9, 2, cap=60, prompt_lens=[50, 31])
+    c2, _ = harness.make_pair(w, 9, 2, cap=60, prompt_lens=[50, 31])
+    for t in range(6):
+        q, kn, vn = (harness.dev(a, "bf16") for a in inputs.step_inputs(w, 9, t, 2))
+        o1 = c1.step(q, kn, vn, 16, 4)
+        o2 = c2.attend_score(q, kn, vn)
+        c2.evict(16, 4)
+        assert torch.equal(o1, o2)
+        for s in range(2):
+            e1, e2 = c1.export(s), c2.export(s)
+            for l in range(3):
+                for h in range(2):
+                    n = e1["len"][l, h]
+                    a = dict(zip(e1["pos"][l, h, :n], e1["score"][l, h, :n]))
+                    b = dict(zip(e2["pos"][l, h, :n], e2["score"][l, h, :n]))
+                    assert a == b
+
+
+def test_selection_exact_on_kernel_scores():
+    """Given the kernel's own fp32 scores, TopB must be exactly the oracle's
+    selection on those same scores (no tolerance)."""
+    w = inputs.Workload("x", 2, 4, 7, 128, "bf16", 20, 5, 90, 5, sigma=1.0)
+    c, _ = harness.make_pair(w, 10, 2, cap=96, prompt_lens=[90, 60])
+    for t in range(5):
+        q, kn, vn = (harness.dev(a, "bf16") for a in inputs.step_inputs(w, 10, t, 2))
+        c.attend_score(q, kn, vn)
+        pre = [c.export(s, kv=False) for s in range(2)]
+        c.evict(20, 5)
+        post = [c.export(s, kv=False) for s in range(2)]
+        for s in range(2):
+            for l in range(2):
+                for h in range(4):
+                    n = pre[s]["len"][l, h]
+                    pos = pre[s]["pos"][l, h, :n]
+                    keep = orc.select_unit(pre[s]["score"][l, h, :n].astype(np.float64),
+                                           pos, 20, 5)
+                    m = post[s]["len"][l, h]
+                    assert set(post[s]["pos"][l, h, :m].tolist()) == set(pos[keep].tolist())
+
+
+def test_capacity_and_argument_errors():
+    w = inputs.Workload("c", 1, 1, 2, 64, "bf16", 4, 1, 3, 2)
+    c, _ = harness.make_pair(w, 11, 1, cap=4)
+    q, kn, vn = (harness.dev(a, "bf16") for a in inputs.step_inputs(w, 11, 0, 1))
+    c.attend_score(q, kn, vn)  # 4 rows: full
+    with pytest.raises(kvr.KvrError) as e:
+        c.attend_score(q, kn, vn)
+    assert e.value.status == kvr.KVR_ECAPACITY
+    with pytest.raises(kvr.KvrError) as e:
+        c.evict(0, 0)
+    assert e.value.status == kvr.KVR_EINVAL
+    with pytest.raises(kvr.KvrError) as e:
+        c.attend_score(q, kn, vn, layers=(0, 2))
+    assert e.value.status == kvr.KVR_EINVAL
+    c.evict(2, 1)
+    assert c.lengths().tolist() == [[3]]
+    c.sync_status()
