@@ -127,6 +127,38 @@ kvr_status kvr_decode_step(kvr_cache *cache, int layer_begin, int layer_end,
                            const void *q, const void *k_new, const void *v_new,
                            void *out, int budget, int window, void *stream);
 
+/* ---- the same step for callers that cannot allocate -------------------- */
+
+/* The paper has no counterpart to this call: it is a deployment variant.
+ *
+ * Some callers cannot allocate device memory for a call at all: a plug-in
+ * running inside a host program that owns every device allocation and hands
+ * the plug-in only the tensors of a call, or a service that fixes its device
+ * footprint at start-up and may not allocate afterwards.  This entry point
+ * does exactly what kvr_decode_attend_score does (same arguments, same
+ * results), but keeps the per-unit logits in a static device array inside
+ * the library instead of the cache buffer's scratch area, and calls no
+ * allocator (no cudaMalloc, cudaFree or allocating library routine).
+ *  - Limit: the call needs S x (layer_end - layer_begin) x H x G x
+ *    (longest live length + 1) x 4 bytes of logits; more than
+ *    KVR_NOALLOC_SCRATCH_BYTES is rejected with KVR_EINVAL before anything
+ *    is enqueued.
+ *  - Every GPU that loads the library holds the array until the process
+ *    exits.
+ *  - The first call on each device looks up the array's device address
+ *    (cudaGetSymbolAddress, with that device current); make that first call
+ *    before any stream capture.
+ *  - All calls share the array and it keeps the previous call's contents:
+ *    every logit is written before it is read, so nothing needs clearing,
+ *    but calls that overlap on the GPU (other streams or host threads) race
+ *    on it; serialise them. */
+#define KVR_NOALLOC_SCRATCH_BYTES (4u << 20)
+kvr_status kvr_decode_attend_score_noalloc(kvr_cache *cache, int layer_begin,
+                                           int layer_end, const void *q,
+                                           const void *k_new,
+                                           const void *v_new, void *out,
+                                           void *stream);
+
 /* ---- inspection -------------------------------------------------------- */
 
 /* Synchronising: wait for stream, then copy sequence seq's state to host.

@@ -268,6 +268,41 @@ kvr_status kvr_decode_attend_score(kvr_cache *c, int lb, int le, const void *q,
   return KVR_OK;
 }
 
+}  // extern "C"
+
+int kvr::report_cuda_error(const char *where, cudaError_t e) {
+  return cuda_fail(where, e);
+}
+
+int kvr::decode_attend_score_ext(kvr_cache *c, int lb, int le, const void *q,
+                                 const void *k_new, const void *v_new,
+                                 void *out, float *ext, size_t ext_floats,
+                                 void *stream) {
+  kvr_status st = check_step(c, lb, le, q, k_new, v_new, out);
+  if (st != KVR_OK) return st;
+  if (!ext) return fail(KVR_EINVAL, "null scratch");
+  StepArgs a = step_args(c, lb, le, q, k_new, v_new, out);
+  const size_t need =
+      (size_t)c->desc.n_seq * a.nl * c->desc.n_kv_heads * c->desc.group *
+      (size_t)a.max_rows;
+  if (need > ext_floats)
+    return fail(KVR_EINVAL,
+                "this call needs %zu bytes of logit scratch (%d seq x %d layers"
+                " x %d heads x G=%d x %d rows x 4 B); the static scratch holds "
+                "%zu bytes",
+                need * sizeof(float), c->desc.n_seq, a.nl,
+                c->desc.n_kv_heads, c->desc.group, a.max_rows,
+                ext_floats * sizeof(float));
+  cudaError_t e = kvr::launch_attend_score_ext_scratch(c->view, a, ext,
+                                                       as_stream(stream));
+  if (e != cudaSuccess) return cuda_fail("kvr_decode_attend_score_noalloc", e);
+  c->launches += 1;
+  mirror_append(c, lb, le);
+  return KVR_OK;
+}
+
+extern "C" {
+
 kvr_status kvr_evict_compact(kvr_cache *c, int lb, int le, int budget,
                              int window, void *stream) {
   if (!c) return fail(KVR_EINVAL, "null cache");

@@ -76,9 +76,12 @@ __host__ __device__ constexpr int attend_fixed_floats(int D) {
          + 2 * kMaxG;                        // max and 1/sum per head
 }
 
-template <typename T, typename O, int D>
+// kExtScratch: logits always go to `ext`, one [G][max_rows] block per CTA,
+// instead of shared memory or the cache's own scratch area.
+template <typename T, typename O, int D, bool kExtScratch = false>
 __global__ void __launch_bounds__(kThreads)
-    attend_score_kernel(CacheView c, StepArgs a, int logits_in_smem) {
+    attend_score_kernel(CacheView c, StepArgs a, int logits_in_smem,
+                        float *ext) {
   extern __shared__ float smem[];
   constexpr int P = D / 2;         // dimension pairs
   constexpr int R = kThreads / P;  // row groups of the PV pass
@@ -122,8 +125,10 @@ __global__ void __launch_bounds__(kThreads)
   }
   __syncthreads();
 
-  float *lg = logits_in_smem ? lg_s : c.logits + x.u * (size_t)G * c.cap;
-  const int ls = logits_in_smem ? a.max_rows : c.cap;
+  float *lg = kExtScratch ? ext + (size_t)blockIdx.x * G * a.max_rows
+              : logits_in_smem ? lg_s
+                               : c.logits + x.u * (size_t)G * c.cap;
+  const int ls = (kExtScratch || logits_in_smem) ? a.max_rows : c.cap;
 
   // Logits l_{g,i} = scale * <q_g, k_i>: one warp per row.
   for (int i = warp; i < n; i += kWarps) {
@@ -396,7 +401,19 @@ cudaError_t attend_dispatch(const CacheView &c, const StepArgs &a,
       kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
   if (e != cudaSuccess) return e;
   const int grid = c.S * a.nl * c.H;
-  kern<<<grid, kThreads, bytes, st>>>(c, a, in_smem);
+  kern<<<grid, kThreads, bytes, st>>>(c, a, in_smem, nullptr);
+  return cudaGetLastError();
+}
+
+template <typename T, typename O, int D>
+cudaError_t attend_ext_dispatch(const CacheView &c, const StepArgs &a,
+                                float *ext, cudaStream_t st) {
+  const size_t bytes = attend_fixed_floats(D) * sizeof(float);
+  auto kern = attend_score_kernel<T, O, D, true>;
+  cudaError_t e = cudaFuncSetAttribute(
+      kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+  if (e != cudaSuccess) return e;
+  kern<<<c.S * a.nl * c.H, kThreads, bytes, st>>>(c, a, 0, ext);
   return cudaGetLastError();
 }
 
@@ -432,6 +449,28 @@ cudaError_t launch_attend_score_generic(const CacheView &c, const StepArgs &a,
                       : attend_dispatch<float, float, 128>(c, a, st);
   return c.out_bf16 ? attend_dispatch<float, __nv_bfloat16, 64>(c, a, st)
                     : attend_dispatch<float, float, 64>(c, a, st);
+}
+
+cudaError_t launch_attend_score_ext_scratch(const CacheView &c,
+                                            const StepArgs &a, float *ext,
+                                            cudaStream_t st) {
+  if (c.kv_bf16) {
+    if (c.d == 128)
+      return c.out_bf16 ? attend_ext_dispatch<__nv_bfloat16, __nv_bfloat16,
+                                              128>(c, a, ext, st)
+                        : attend_ext_dispatch<__nv_bfloat16, float, 128>(
+                              c, a, ext, st);
+    return c.out_bf16
+               ? attend_ext_dispatch<__nv_bfloat16, __nv_bfloat16, 64>(c, a,
+                                                                        ext, st)
+               : attend_ext_dispatch<__nv_bfloat16, float, 64>(c, a, ext, st);
+  }
+  if (c.d == 128)
+    return c.out_bf16
+               ? attend_ext_dispatch<float, __nv_bfloat16, 128>(c, a, ext, st)
+               : attend_ext_dispatch<float, float, 128>(c, a, ext, st);
+  return c.out_bf16 ? attend_ext_dispatch<float, __nv_bfloat16, 64>(c, a, ext, st)
+                    : attend_ext_dispatch<float, float, 64>(c, a, ext, st);
 }
 
 cudaError_t launch_evict_generic(const CacheView &c, int lb, int nl,

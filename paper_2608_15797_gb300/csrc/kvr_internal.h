@@ -45,6 +45,11 @@ struct StepArgs {
 // Generic kernels (any d in {64,128}, G <= 8, fp32 or bf16): one CTA per unit.
 cudaError_t launch_attend_score_generic(const CacheView &c, const StepArgs &a,
                                         cudaStream_t st);
+// The attend kernel with its logits always in `ext` (one [G][max_rows] fp32
+// block per (sequence, layer, KV head) of the launch, in launch order).
+cudaError_t launch_attend_score_ext_scratch(const CacheView &c,
+                                            const StepArgs &a, float *ext,
+                                            cudaStream_t st);
 cudaError_t launch_evict_generic(const CacheView &c, int lb, int nl,
                                  int max_rows, int budget, int window,
                                  cudaStream_t st);
@@ -53,4 +58,15 @@ cudaError_t launch_load(const CacheView &c, int seq, const void *k,
                         cudaStream_t st);
 cudaError_t launch_init(const CacheView &c, cudaStream_t st);
 
+}  // namespace kvr
+
+struct kvr_cache;
+namespace kvr {
+// kvr_decode_attend_score with the logit scratch supplied by the caller of
+// this internal function (ext, ext_floats) instead of the cache buffer.
+int decode_attend_score_ext(kvr_cache *c, int lb, int le, const void *q,
+                            const void *k_new, const void *v_new, void *out,
+                            float *ext, size_t ext_floats, void *stream);
+// Record a CUDA failure as the thread's last error; returns KVR_ECUDA.
+int report_cuda_error(const char *where, cudaError_t e);
 }  // namespace kvr

@@ -59,6 +59,7 @@ _SIGS = {
     "kvr_cache_destroy": (None, [_P]),
     "kvr_cache_load": (_S, [_P, _I, _P, _P, _I, _I, _P]),
     "kvr_decode_attend_score": (_S, [_P, _I, _I, _P, _P, _P, _P, _P]),
+    "kvr_decode_attend_score_noalloc": (_S, [_P, _I, _I, _P, _P, _P, _P, _P]),
     "kvr_evict_compact": (_S, [_P, _I, _I, _I, _I, _P]),
     "kvr_decode_step": (_S, [_P, _I, _I, _P, _P, _P, _P, _I, _I, _P]),
     "kvr_cache_export": (_S, [_P, _I, _P, _P, _P, _P, _P, _P, _P]),
@@ -138,6 +139,15 @@ def kvr_decode_attend_score(h, layer_begin, layer_end, q, k_new, v_new, out,
                                        _ptr(k_new), _ptr(v_new), _ptr(out),
                                        _stream(stream)),
            "kvr_decode_attend_score")
+
+
+def kvr_decode_attend_score_noalloc(h, layer_begin, layer_end, q, k_new,
+                                    v_new, out, stream=None):
+    _check(lib.kvr_decode_attend_score_noalloc(h, layer_begin, layer_end,
+                                               _ptr(q), _ptr(k_new),
+                                               _ptr(v_new), _ptr(out),
+                                               _stream(stream)),
+           "kvr_decode_attend_score_noalloc")
 
 
 def kvr_evict_compact(h, layer_begin, layer_end, budget, window, stream=None):
