@@ -127,6 +127,13 @@ kvr_status kvr_decode_step(kvr_cache *cache, int layer_begin, int layer_end,
                            const void *q, const void *k_new, const void *v_new,
                            void *out, int budget, int window, void *stream);
 
+/* Choose whether kvr_decode_attend_score / kvr_decode_step may use the
+ * fused single-pass kernel (bf16, head_dim 128, G <= 8, at most 128 live rows
+ * per unit, at most one eviction per unit; the default) or must use the
+ * generic kernels for every shape.  Both compute the same step; this exists
+ * for testing and measurement.  enable: 0 or 1. */
+kvr_status kvr_cache_set_fused(kvr_cache *cache, int enable);
+
 /* ---- the same step for callers that cannot allocate -------------------- */
 
 /* The paper has no counterpart to this call: it is a deployment variant.

@@ -1,9 +1,14 @@
 // kvr_api.cu -- the C ABI of libkvr (include/kvr.h): argument validation,
 // the host mirror of every live length, carving of the caller's device
 // buffer, and kernel dispatch.  No device memory is allocated here.
+#include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <map>
+#include <mutex>
+#include <utility>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -55,12 +60,13 @@ bool desc_ok(const kvr_cache_desc *d) {
 
 // Byte offsets of every array inside the cache buffer.
 struct Layout {
-  size_t K, V, score, pos, len, next_pos, err, logits, total;
+  size_t K, V, score, pos, state, err, logits, total;
 };
 
 Layout layout_of(const kvr_cache_desc *d) {
   const size_t units = (size_t)d->n_seq * d->n_layers * d->n_kv_heads;
   const size_t rows = units * (size_t)d->capacity;
+  const size_t srows = units * (size_t)kvr::round_up16(d->capacity);
   Layout l{};
   size_t off = 0;
   l.K = off;
@@ -68,13 +74,11 @@ Layout layout_of(const kvr_cache_desc *d) {
   l.V = off;
   off = align_up(off + rows * d->head_dim * esize(d->kv_dtype));
   l.score = off;
-  off = align_up(off + rows * sizeof(float));
+  off = align_up(off + srows * sizeof(float));
   l.pos = off;
-  off = align_up(off + rows * sizeof(int32_t));
-  l.len = off;
-  off = align_up(off + units * sizeof(int32_t));
-  l.next_pos = off;
-  off = align_up(off + units * sizeof(int32_t));
+  off = align_up(off + srows * sizeof(int32_t));
+  l.state = off;
+  off = align_up(off + units * 4 * sizeof(int32_t));
   l.err = off;
   off = align_up(off + 16);
   l.logits = off;
@@ -92,7 +96,47 @@ struct kvr_cache {
   std::vector<int32_t> next_pos;  // host mirror [S][L]
   size_t bytes;
   uint64_t launches = 0;          // kernels launched through this handle
+  bool fused = true;              // use the fused kernel where it applies
+  int sm_count = 0;               // of the device, queried on first use
+  int smem_optin = 0;
+  std::map<int, std::pair<CUtensorMap, CUtensorMap>> tmaps;  // by staged rows
 };
+
+namespace {
+
+// cuTensorMapEncodeTiled through the runtime's driver entry point (the
+// library links no driver stub, so it also loads on hosts without a GPU).
+PFN_cuTensorMapEncodeTiled_v12000 encode_tiled() {
+  static std::once_flag once;
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  std::call_once(once, [] {
+    void *p = nullptr;
+    cudaDriverEntryPointQueryResult q{};
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000,
+                                         cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// 2-D view of a K or V slab: [units * cap rows][128 bf16], boxes of
+// 64 columns x R rows, 128-byte swizzle (conflict-free ldmatrix).
+bool encode_slab(CUtensorMap *m, void *base, size_t rows, int R) {
+  auto fn = encode_tiled();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {128, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {256};
+  cuuint32_t box[2] = {64, (cuuint32_t)R};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace
 
 namespace {
 
@@ -171,6 +215,76 @@ StepArgs step_args(const kvr_cache *c, int lb, int le, const void *q,
 
 }  // namespace
 
+namespace {
+
+bool aligned16(const void *p) {
+  return reinterpret_cast<uintptr_t>(p) % 16 == 0;
+}
+
+// Launch the fused kernel if this call qualifies; returns false (and does
+// nothing) if it does not, true with *err set otherwise.
+bool try_fused(kvr_cache *c, const StepArgs &a, bool evict, int budget,
+               int window, cudaStream_t stream, cudaError_t *err) {
+  const CacheView &v = c->view;
+  if (!c->fused || !v.kv_bf16 || v.d != 128 || v.G > 8) return false;
+  if (a.max_rows > 128) return false;
+  if (evict && (long long)a.max_rows > (long long)budget + window + 1)
+    return false;
+  const size_t rows = (size_t)v.S * v.L * v.H * v.cap;
+  if (rows >= (size_t)INT32_MAX) return false;
+  if (!aligned16(a.q) || !aligned16(a.k_new) || !aligned16(a.v_new) ||
+      !aligned16(a.out))
+    return false;
+  if (!c->sm_count) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&c->sm_count, cudaDevAttrMultiProcessorCount,
+                               dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&c->smem_optin,
+                               cudaDevAttrMaxSharedMemoryPerBlockOptin,
+                               dev) != cudaSuccess) {
+      c->sm_count = 0;
+      return false;
+    }
+  }
+  const int R = kvr::round_up16(a.max_rows);
+  const int stage = kvr::fused_stage_bytes(R);
+  const int avail = c->smem_optin - 1024 /*alignment*/ - 512 /*static*/;
+  const int n_stages = std::min(8, avail / stage);
+  if (n_stages < 2) return false;
+  auto it = c->tmaps.find(R);
+  if (it == c->tmaps.end()) {
+    std::pair<CUtensorMap, CUtensorMap> maps;
+    if (!encode_slab(&maps.first, v.K, rows, R) ||
+        !encode_slab(&maps.second, v.V, rows, R))
+      return false;
+    it = c->tmaps.emplace(R, maps).first;
+  }
+  kvr::FusedParams p{};
+  p.c = v;
+  p.q = static_cast<const __nv_bfloat16 *>(a.q);
+  p.k_new = static_cast<const __nv_bfloat16 *>(a.k_new);
+  p.v_new = static_cast<const __nv_bfloat16 *>(a.v_new);
+  p.out = a.out;
+  p.lb = a.lb;
+  p.nl = a.nl;
+  p.R = R;
+  p.n_stages = n_stages;
+  p.n_consumers = std::min(4, n_stages - 1);
+  p.budget = budget;
+  p.window = window;
+  p.evict = evict ? 1 : 0;
+  p.scale_log2e = v.scale * 1.4426950408889634f;
+  p.inv_g = 1.f / (float)v.G;
+  const int units = v.S * a.nl * v.H;
+  const int grid = std::min(c->sm_count, units);
+  *err = kvr::launch_fused_step(it->second.first, it->second.second, p, grid,
+                                n_stages * stage + 1024, stream);
+  return true;
+}
+
+}  // namespace
+
 extern "C" {
 
 size_t kvr_cache_required_bytes(const kvr_cache_desc *desc) {
@@ -200,8 +314,7 @@ kvr_status kvr_cache_create(const kvr_cache_desc *desc, void *dev_buf,
   v.V = b + lay.V;
   v.score = reinterpret_cast<float *>(b + lay.score);
   v.pos = reinterpret_cast<int32_t *>(b + lay.pos);
-  v.len = reinterpret_cast<int32_t *>(b + lay.len);
-  v.next_pos = reinterpret_cast<int32_t *>(b + lay.next_pos);
+  v.state = reinterpret_cast<int32_t *>(b + lay.state);
   v.err = reinterpret_cast<unsigned *>(b + lay.err);
   v.logits = reinterpret_cast<float *>(b + lay.logits);
   v.S = desc->n_seq;
@@ -210,6 +323,7 @@ kvr_status kvr_cache_create(const kvr_cache_desc *desc, void *dev_buf,
   v.G = desc->group;
   v.d = desc->head_dim;
   v.cap = desc->capacity;
+  v.sstride = kvr::round_up16(desc->capacity);
   v.scale = desc->softmax_scale > 0.f
                 ? desc->softmax_scale
                 : (float)(1.0 / std::sqrt((double)desc->head_dim));
@@ -260,11 +374,18 @@ kvr_status kvr_decode_attend_score(kvr_cache *c, int lb, int le, const void *q,
   kvr_status st = check_step(c, lb, le, q, k_new, v_new, out);
   if (st != KVR_OK) return st;
   StepArgs a = step_args(c, lb, le, q, k_new, v_new, out);
-  cudaError_t e =
-      kvr::launch_attend_score_generic(c->view, a, as_stream(stream));
+  cudaError_t e = cudaSuccess;
+  if (!try_fused(c, a, false, 0, 0, as_stream(stream), &e))
+    e = kvr::launch_attend_score_generic(c->view, a, as_stream(stream));
   if (e != cudaSuccess) return cuda_fail("kvr_decode_attend_score", e);
   c->launches += 1;
   mirror_append(c, lb, le);
+  return KVR_OK;
+}
+
+kvr_status kvr_cache_set_fused(kvr_cache *c, int enable) {
+  if (!c) return fail(KVR_EINVAL, "null cache");
+  c->fused = enable != 0;
   return KVR_OK;
 }
 
@@ -327,6 +448,15 @@ kvr_status kvr_decode_step(kvr_cache *c, int lb, int le, const void *q,
   if (st != KVR_OK) return st;
   st = check_evict(budget, window);
   if (st != KVR_OK) return st;
+  StepArgs a = step_args(c, lb, le, q, k_new, v_new, out);
+  cudaError_t e = cudaSuccess;
+  if (try_fused(c, a, true, budget, window, as_stream(stream), &e)) {
+    if (e != cudaSuccess) return cuda_fail("kvr_decode_step", e);
+    c->launches += 1;
+    mirror_append(c, lb, le);
+    mirror_evict(c, lb, le, budget, window);
+    return KVR_OK;
+  }
   st = kvr_decode_attend_score(c, lb, le, q, k_new, v_new, out, stream);
   if (st != KVR_OK) return st;
   return kvr_evict_compact(c, lb, le, budget, window, stream);
@@ -351,15 +481,33 @@ kvr_status kvr_cache_export(const kvr_cache *c, int seq, void *host_k,
   } copies[] = {
       {host_k, static_cast<char *>(v.K) + seq * rows * ebytes, rows * ebytes},
       {host_v, static_cast<char *>(v.V) + seq * rows * ebytes, rows * ebytes},
-      {host_score, v.score + seq * rows, rows * sizeof(float)},
-      {host_pos, v.pos + seq * rows, rows * sizeof(int32_t)},
-      {host_len, v.len + seq * units, units * sizeof(int32_t)},
-      {host_next_pos, v.next_pos + seq * units, units * sizeof(int32_t)},
   };
   for (auto &cp : copies) {
     if (!cp.dst) continue;
     e = cudaMemcpy(cp.dst, cp.src, cp.bytes, cudaMemcpyDeviceToHost);
     if (e != cudaSuccess) return cuda_fail("kvr_cache_export", e);
+  }
+  // Scores and positions: [units][sstride] on the device, [units][cap] out.
+  struct {
+    void *dst;
+    const void *src;
+  } rowwise[] = {{host_score, v.score + seq * units * v.sstride},
+                 {host_pos, v.pos + seq * units * v.sstride}};
+  for (auto &cp : rowwise) {
+    if (!cp.dst) continue;
+    e = cudaMemcpy2D(cp.dst, (size_t)v.cap * 4, cp.src, (size_t)v.sstride * 4,
+                     (size_t)v.cap * 4, units, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail("kvr_cache_export", e);
+  }
+  if (host_len || host_next_pos) {
+    std::vector<int32_t> st(units * 4);
+    e = cudaMemcpy(st.data(), v.state + seq * units * 4,
+                   st.size() * sizeof(int32_t), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail("kvr_cache_export", e);
+    for (size_t i = 0; i < units; ++i) {
+      if (host_len) host_len[i] = st[4 * i];
+      if (host_next_pos) host_next_pos[i] = st[4 * i + 1];
+    }
   }
   return KVR_OK;
 }

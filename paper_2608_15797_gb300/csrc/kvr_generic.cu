@@ -96,7 +96,7 @@ __global__ void __launch_bounds__(kThreads)
   const Unit x = unit_of(c, a.lb, a.nl);
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
 
-  const int n0 = c.len[x.u];
+  const int n0 = c.state[4 * x.u];
   if (n0 + 1 > c.cap) {
     if (tid == 0) atomicOr(c.err, ERR_CAPACITY);
     return;
@@ -104,8 +104,8 @@ __global__ void __launch_bounds__(kThreads)
   const int n = n0 + 1;
   T *Ku = reinterpret_cast<T *>(c.K) + x.u * (size_t)c.cap * D;
   T *Vu = reinterpret_cast<T *>(c.V) + x.u * (size_t)c.cap * D;
-  float *su = c.score + x.u * (size_t)c.cap;
-  int32_t *pu = c.pos + x.u * (size_t)c.cap;
+  float *su = c.score + x.u * (size_t)c.sstride;
+  int32_t *pu = c.pos + x.u * (size_t)c.sstride;
   const size_t kv_row = ((size_t)x.s * a.nl + x.lr) * c.H + x.h;
   const size_t q_row = kv_row * G;
   const T *qg = reinterpret_cast<const T *>(a.q) + q_row * D;
@@ -118,7 +118,7 @@ __global__ void __launch_bounds__(kThreads)
     Ku[(size_t)n0 * D + i] = kn[i];
     Vu[(size_t)n0 * D + i] = vn[i];
   }
-  const int newest = c.next_pos[x.u];
+  const int newest = c.state[4 * x.u + 1];
   if (tid == 0) {
     pu[n0] = newest;
     su[n0] = 0.f;
@@ -214,8 +214,8 @@ __global__ void __launch_bounds__(kThreads)
     st1(og + i, o);
   }
   if (tid == 0) {
-    c.len[x.u] = n;
-    c.next_pos[x.u] = newest + 1;
+    c.state[4 * x.u] = n;
+    c.state[4 * x.u + 1] = newest + 1;
   }
 }
 
@@ -267,15 +267,15 @@ __global__ void __launch_bounds__(kThreads)
 
   const Unit x = unit_of(c, lb, nl);
   const int tid = threadIdx.x;
-  const int n = c.len[x.u];
+  const int n = c.state[4 * x.u];
   if (n <= B + W) return;
   T *Ku = reinterpret_cast<T *>(c.K) + x.u * (size_t)c.cap * D;
   T *Vu = reinterpret_cast<T *>(c.V) + x.u * (size_t)c.cap * D;
-  float *su = c.score + x.u * (size_t)c.cap;
-  int32_t *pu = c.pos + x.u * (size_t)c.cap;
+  float *su = c.score + x.u * (size_t)c.sstride;
+  int32_t *pu = c.pos + x.u * (size_t)c.sstride;
   // The W most recent positions are protected; a row is a candidate iff its
   // position is at most newest - W.
-  const int wlo = c.next_pos[x.u] - 1 - W;
+  const int wlo = c.state[4 * x.u + 1] - 1 - W;
 
   // Radix select (8 passes of 8 bits) of the B-th largest candidate key.
   unsigned long long thr = ~0ull;
@@ -353,7 +353,7 @@ __global__ void __launch_bounds__(kThreads)
       pu[dst] = pu[src];
     }
   }
-  if (tid == 0) c.len[x.u] = nk;
+  if (tid == 0) c.state[4 * x.u] = nk;
 }
 
 // Copy one sequence's prompt rows [L][H][n][d] into its slabs.
@@ -377,12 +377,12 @@ __global__ void load_kernel(CacheView c, int seq, const T *k, const T *v,
         reinterpret_cast<const int4 *>(vs + r * D)[cidx];
   }
   for (int r = r0 + threadIdx.x; r < r1; r += blockDim.x) {
-    c.score[u * c.cap + r] = 0.f;
-    c.pos[u * c.cap + r] = first_pos + r;
+    c.score[u * c.sstride + r] = 0.f;
+    c.pos[u * c.sstride + r] = first_pos + r;
   }
   if (blockIdx.y == 0 && threadIdx.x == 0) {
-    c.len[u] = n;
-    c.next_pos[u] = first_pos + n;
+    c.state[4 * u] = n;
+    c.state[4 * u + 1] = first_pos + n;
   }
 }
 
@@ -513,9 +513,7 @@ cudaError_t launch_load(const CacheView &c, int seq, const void *k,
 
 cudaError_t launch_init(const CacheView &c, cudaStream_t st) {
   const size_t units = (size_t)c.S * c.L * c.H;
-  cudaError_t e = cudaMemsetAsync(c.len, 0, units * sizeof(int32_t), st);
-  if (e == cudaSuccess)
-    e = cudaMemsetAsync(c.next_pos, 0, units * sizeof(int32_t), st);
+  cudaError_t e = cudaMemsetAsync(c.state, 0, units * 4 * sizeof(int32_t), st);
   if (e == cudaSuccess) e = cudaMemsetAsync(c.err, 0, 16, st);
   return e;
 }

@@ -2,6 +2,8 @@
 // libkvr.  Not installed; not part of the ABI.
 #pragma once
 
+#include <cuda.h>
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -12,19 +14,23 @@ enum : unsigned {
   ERR_CAPACITY = 1u,   // a unit had no free row for the append
   ERR_NONFINITE = 2u,  // a softmax normaliser was not finite
   ERR_LENGTH = 4u,     // an eviction produced an unexpected live length
+  ERR_TIMEOUT = 8u,    // a bounded wait on an asynchronous copy gave up
 };
 
+__host__ __device__ inline int round_up16(int x) { return (x + 15) & ~15; }
+
 // Device view of one cache: every pointer points into the caller's buffer.
+// A unit u = (s * L + l) * H + h.
 struct CacheView {
-  void *K;          // [S][L][H][cap][d] kv element type
-  void *V;          // [S][L][H][cap][d]
-  float *score;     // [S][L][H][cap]
-  int32_t *pos;     // [S][L][H][cap]
-  int32_t *len;     // [S][L][H]
-  int32_t *next_pos;// [S][L][H]
+  void *K;          // [u][cap][d] kv element type
+  void *V;          // [u][cap][d]
+  float *score;     // [u][sstride]
+  int32_t *pos;     // [u][sstride]
+  int32_t *state;   // [u][4]: live length, next position, 0, 0
   unsigned *err;    // device error word
-  float *logits;    // [S][L][H][G][cap] scratch for units beyond on-chip size
+  float *logits;    // [u][G][cap] scratch for units beyond on-chip size
   int S, L, H, G, d, cap;
+  int sstride;      // cap rounded up to 16 (64-byte aligned score/pos rows)
   float scale;      // softmax scale (1/sqrt(d) by default)
   int kv_bf16;      // 1: bf16 elements, 0: fp32
   int out_bf16;     // 1: bf16 output, 0: fp32
@@ -57,6 +63,25 @@ cudaError_t launch_load(const CacheView &c, int seq, const void *k,
                         const void *v, int n_rows, int first_pos,
                         cudaStream_t st);
 cudaError_t launch_init(const CacheView &c, cudaStream_t st);
+
+// Fused steady-state step (kvr_fused.cu): bf16, d = 128, G <= 8, at most 128
+// live rows per unit after the append, at most one eviction per unit.
+struct FusedParams {
+  CacheView c;
+  const __nv_bfloat16 *q;      // [S][nl][H*G][128]
+  const __nv_bfloat16 *k_new;  // [S][nl][H][128]
+  const __nv_bfloat16 *v_new;  // [S][nl][H][128]
+  void *out;                   // [S][nl][H*G][128]
+  int lb, nl;
+  int R;                       // staged rows per unit (multiple of 16, <= 128)
+  int n_stages, n_consumers;   // shared-memory ring depth, consumer warps
+  int budget, window, evict;
+  float scale_log2e, inv_g;
+};
+int fused_stage_bytes(int R);
+cudaError_t launch_fused_step(const CUtensorMap &tmK, const CUtensorMap &tmV,
+                              const FusedParams &p, int grid, int smem_bytes,
+                              cudaStream_t st);
 
 }  // namespace kvr
 

@@ -65,6 +65,7 @@ _SIGS = {
     "kvr_cache_export": (_S, [_P, _I, _P, _P, _P, _P, _P, _P, _P]),
     "kvr_cache_lengths": (_S, [_P, _P]),
     "kvr_cache_launch_count": (_S, [_P, _P]),
+    "kvr_cache_set_fused": (_S, [_P, _I]),
     "kvr_sync_status": (_S, [_P, _P]),
     "kvr_last_error": (ctypes.c_char_p, []),
 }
@@ -181,6 +182,10 @@ def kvr_cache_launch_count(h) -> int:
     return int(n.value)
 
 
+def kvr_cache_set_fused(h, enable: bool):
+    _check(lib.kvr_cache_set_fused(h, 1 if enable else 0), "kvr_cache_set_fused")
+
+
 def kvr_sync_status(h, stream=None):
     _check(lib.kvr_sync_status(h, _stream(stream)), "kvr_sync_status")
 
@@ -270,6 +275,9 @@ class Cache:
             res["K"] = hk.float().numpy()
             res["V"] = hv.float().numpy()
         return res
+
+    def set_fused(self, enable: bool):
+        kvr_cache_set_fused(self.handle, enable)
 
     def launch_count(self):
         return kvr_cache_launch_count(self.handle)

@@ -33,20 +33,25 @@ def test_tiny_workload_full_run():
     assert (c.lengths() == w.budget + w.window).all()
 
 
-def test_7b_geometry_lockstep():
+@pytest.mark.parametrize("fused", [True, False])
+def test_7b_geometry_lockstep(fused):
     """Qwen2.5-Math-7B decode geometry (28 layers, G=7, d=128, bf16,
-    N(0,1)/sqrt(128)), prompt 512, B=64, W=8: 48 steps in lock-step."""
+    N(0,1)/sqrt(128)), prompt 512, B=64, W=8: 48 steps in lock-step.  The
+    first step (513 rows) runs the generic kernels; the steady state runs the
+    fused kernel unless it is disabled."""
     w = inputs.WORKLOADS["7b_b64"]
-    c, o = harness.make_pair(w, 2, 1, cap=w.prompt + 1)
+    c, o = harness.make_pair(w, 2, 1, cap=w.prompt + 1, fused=fused)
     st = harness.lockstep(c, o, w, 2, 48, w.budget, w.window)
     assert st.units == 48 * 28 * 4
 
 
-def test_7b_unscaled_selection_exercised():
+@pytest.mark.parametrize("fused", [True, False])
+def test_7b_unscaled_selection_exercised(fused):
     """Unscaled N(0,1) q/k: attention is peaked, so TopB decisions are far
     from ties and must match the oracle exactly."""
     w = inputs.WORKLOADS["7b_unscaled"]
-    c, o = harness.make_pair(w, 3, 2, cap=w.prompt + 1, prompt_lens=[512, 301])
+    c, o = harness.make_pair(w, 3, 2, cap=w.prompt + 1, prompt_lens=[512, 301],
+                             fused=fused)
     st = harness.lockstep(c, o, w, 3, 24, w.budget, w.window)
     assert st.adoptions == 0
 
@@ -60,11 +65,26 @@ def test_group_sizes_and_dims(G, d, dtype):
     harness.lockstep(c, o, w, 4, 10, w.budget, w.window)
 
 
+@pytest.mark.parametrize("fused", [True, False])
 @pytest.mark.parametrize("B,W", [(1, 0), (0, 2), (5, 0), (1, 1), (30, 8)])
-def test_budget_window_edges(B, W):
+def test_budget_window_edges(B, W, fused):
     w = inputs.Workload("e", 1, 2, 2, 128, "bf16", B, W, 20, 8, sigma=1.0)
-    c, o = harness.make_pair(w, 5, 2, cap=40, prompt_lens=[20, 1])
+    c, o = harness.make_pair(w, 5, 2, cap=40, prompt_lens=[20, 1], fused=fused)
     harness.lockstep(c, o, w, 5, 8, B, W)
+
+
+@pytest.mark.parametrize("G", [1, 4, 7, 8])
+@pytest.mark.parametrize("B,W", [(64, 8), (100, 19), (3, 5)])
+def test_fused_steady_state_shapes(G, B, W):
+    """The fused kernel across group sizes and staged-row counts (the last
+    16-row tile ragged or full), bf16 output, starting at B+W rows."""
+    w = inputs.Workload("s", 2, 2, G, 128, "bf16", B, W, B + W, 6, sigma=1.0)
+    c, o = harness.make_pair(w, 12, 3, cap=B + W + 1,
+                             prompt_lens=[B + W, B + W, max(1, B + W - 9)],
+                             out_dtype="bf16")
+    n0 = c.launch_count()
+    harness.lockstep(c, o, w, 12, 6, B, W)
+    assert c.launch_count() - n0 == 6  # one fused launch per step
 
 
 def test_empty_prompt_and_single_row():
