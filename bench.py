@@ -51,6 +51,10 @@ def parse():
     p.add_argument("--seed", type=int, default=0)
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=15.0)
+    p.add_argument("--prior-min", type=int, default=inputs.PRIOR_LEN_RANGE[0],
+                   help="shortest prior context (profiling uses a small case)")
+    p.add_argument("--prior-max", type=int, default=inputs.PRIOR_LEN_RANGE[1])
+    p.add_argument("--e2e-steps", type=int, default=1000)
     return p.parse_args()
 
 
@@ -197,7 +201,8 @@ def run_kvr(args, rank, world, local_rank):
     w = inputs.WORKLOADS[args.workload]
     S, L, H, G, d = w.n_seq, w.n_layers, w.n_kv_heads, w.group, w.head_dim
     B, W = w.budget, w.window
-    lens = inputs.prior_lengths(args.seed + 7919 * rank, S)
+    lens = inputs.prior_lengths(args.seed + 7919 * rank, S, args.prior_min,
+                                args.prior_max)
     cap = int(lens.max()) + 1
     cache = kvr.Cache(S, L, H, G, d, cap, kv_dtype="bf16", out_dtype="bf16",
                       device=dev)
@@ -275,7 +280,7 @@ def run_kvr(args, rank, world, local_rank):
     dq, dk, dv = (torch.empty_like(x) for x in pool[0])
     bi = sum(x.numel() * x.element_size() for x in hpool[0])
     bo = hout.numel() * hout.element_size()
-    Ke = max(1, min(K, 1000))
+    Ke = max(1, min(K, args.e2e_steps))
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     torch.cuda.synchronize()
     e0.record(stream)
@@ -363,7 +368,8 @@ def main():
                    "layers": w.n_layers, "kv_heads": w.n_kv_heads,
                    "group": w.group, "head_dim": w.head_dim,
                    "budget": w.budget, "window": w.window,
-                   "prior_len": "U[512,16384]", "elem": "bf16",
+                   "prior_len": f"U[{args.prior_min},{args.prior_max}]",
+                   "elem": "bf16",
                    "l2": f"inputs larger than L2: {r['launch_bytes'] / 1e6:.0f} MB"
                          " touched per step, no flush",
                    "per_rank_sequences": w.n_seq},

@@ -99,7 +99,7 @@ struct kvr_cache {
   bool fused = true;              // use the fused kernel where it applies
   int sm_count = 0;               // of the device, queried on first use
   int smem_optin = 0;
-  std::map<int, std::pair<CUtensorMap, CUtensorMap>> tmaps;  // by staged rows
+  std::map<int, std::pair<CUtensorMap, CUtensorMap>> tmaps;  // by box rows
 };
 
 namespace {
@@ -248,17 +248,22 @@ bool try_fused(kvr_cache *c, const StepArgs &a, bool evict, int budget,
     }
   }
   const int R = kvr::round_up16(a.max_rows);
+  const int Rb = std::max(8, (a.max_rows - 1 + 7) / 8 * 8);
+  const int U = kvr::fused_group_warps(R);
   const int stage = kvr::fused_stage_bytes(R);
   const int avail = c->smem_optin - 1024 /*alignment*/ - 512 /*static*/;
   const int n_stages = std::min(8, avail / stage);
-  if (n_stages < 2) return false;
-  auto it = c->tmaps.find(R);
+  if (U < 1 || n_stages < 2) return false;
+  const int n_groups = std::min(
+      {4, n_stages - 1, (kvr::fused_max_threads() / 32 - 1) / U});
+  if (n_groups < 1) return false;
+  auto it = c->tmaps.find(Rb);
   if (it == c->tmaps.end()) {
     std::pair<CUtensorMap, CUtensorMap> maps;
-    if (!encode_slab(&maps.first, v.K, rows, R) ||
-        !encode_slab(&maps.second, v.V, rows, R))
+    if (!encode_slab(&maps.first, v.K, rows, Rb) ||
+        !encode_slab(&maps.second, v.V, rows, Rb))
       return false;
-    it = c->tmaps.emplace(R, maps).first;
+    it = c->tmaps.emplace(Rb, maps).first;
   }
   kvr::FusedParams p{};
   p.c = v;
@@ -269,8 +274,9 @@ bool try_fused(kvr_cache *c, const StepArgs &a, bool evict, int budget,
   p.lb = a.lb;
   p.nl = a.nl;
   p.R = R;
+  p.Rb = Rb;
   p.n_stages = n_stages;
-  p.n_consumers = std::min(4, n_stages - 1);
+  p.n_groups = n_groups;
   p.budget = budget;
   p.window = window;
   p.evict = evict ? 1 : 0;

@@ -34,7 +34,10 @@ namespace kvr {
 namespace {
 
 constexpr int kMaxStages = 8;
-constexpr int kMaxConsumers = 4;
+constexpr int kMaxGroups = 4;      // units in flight on the consumer side
+constexpr int kMaxGroupWarps = 8;  // warps sharing one unit
+constexpr int kMaxThreads = 544;   // 16 consumer warps + the producer
+constexpr int kXsWords = 20;       // exchange words per warp of a group
 constexpr int kQPitch = 272;  // bytes per staged query row (256 + 16 padding)
 constexpr uint64_t kWaitNs = 2000000000ull;
 
@@ -138,9 +141,13 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   return *reinterpret_cast<uint32_t *>(&v);
 }
 
-// Byte offsets inside one stage (R rows).
+__device__ __forceinline__ void group_bar(int id, int threads) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
+}
+
+// Byte offsets inside one stage of R staged rows.
 struct StageLayout {
-  uint32_t k0, k1, v0, v1, q, kn, vn, sc, ps, st, bytes;
+  uint32_t k0, k1, v0, v1, q, kn, vn, sc, ps, st, xs, bytes;
   __host__ __device__ explicit StageLayout(int R) {
     k0 = 0;
     k1 = k0 + R * 128;
@@ -152,7 +159,8 @@ struct StageLayout {
     sc = vn + 256;
     ps = sc + 4 * R;
     st = ps + 4 * R;
-    bytes = ((st + 16) + 1023) / 1024 * 1024;
+    xs = st + 16;  // group exchange: kXsWords words per warp
+    bytes = ((xs + 4 * kXsWords * kMaxGroupWarps) + 1023) / 1024 * 1024;
   }
 };
 
@@ -172,7 +180,8 @@ __device__ __forceinline__ UnitIdx unit_idx(const FusedParams &p, int idx) {
   return x;
 }
 
-// Producer: enqueue every copy of one unit into a stage.
+// Producer: enqueue every copy of one unit into a stage.  K and V come as
+// two 128B-swizzled boxes of Rb rows each (columns 0-63, 64-127).
 __device__ void issue_unit(const FusedParams &p, const CUtensorMap *tmK,
                            const CUtensorMap *tmV, unsigned char *stage,
                            uint32_t bar, int idx) {
@@ -180,8 +189,8 @@ __device__ void issue_unit(const FusedParams &p, const CUtensorMap *tmK,
   const UnitIdx x = unit_idx(p, idx);
   const int G = p.c.G;
   const uint32_t s0 = smem_u32(stage);
-  const uint32_t tx = 4u * p.R * 128u + (uint32_t)G * 256u + 512u +
-                      8u * p.R + 16u;
+  const uint32_t tx = 4u * p.Rb * 128u + (uint32_t)G * 256u + 512u +
+                      8u * p.Rb + 16u;
   mbar_expect_tx(bar, tx);
   const int row0 = (int)(x.ug * (size_t)p.c.cap);
   tma_load_2d(s0 + L.k0, tmK, 0, row0, bar);
@@ -193,46 +202,54 @@ __device__ void issue_unit(const FusedParams &p, const CUtensorMap *tmK,
     bulk_load(s0 + L.q + g * kQPitch, q + g * 128, 256, bar);
   bulk_load(s0 + L.kn, p.k_new + x.krow * 128, 256, bar);
   bulk_load(s0 + L.vn, p.v_new + x.krow * 128, 256, bar);
-  bulk_load(s0 + L.sc, p.c.score + x.ug * p.c.sstride, 4u * p.R, bar);
-  bulk_load(s0 + L.ps, p.c.pos + x.ug * p.c.sstride, 4u * p.R, bar);
+  bulk_load(s0 + L.sc, p.c.score + x.ug * p.c.sstride, 4u * p.Rb, bar);
+  bulk_load(s0 + L.ps, p.c.pos + x.ug * p.c.sstride, 4u * p.Rb, bar);
   bulk_load(s0 + L.st, p.c.state + x.ug * 4, 16, bar);
 }
 
-// Consumer: one warp computes one unit held in a stage.
-template <bool kOutBf16>
+// One group of U warps computes one unit held in a stage.  The unit has
+// T = R / 16 row tiles; warp w of the group owns tiles w, w + U, ...
+// Exchange words per warp (XS): [0,8) column max, [8,16) column sum,
+// [16,18) argmin key, 18 argmin row, 19 wait flag.
+template <int T, int U, bool kOutBf16>
 __device__ void process_unit(const FusedParams &p, unsigned char *stage,
-                             int idx, int lane) {
-  const StageLayout L(p.R);
+                             int idx, int w, int lane, int bar_id) {
+  constexpr int TW = (T + U - 1) / U;  // tiles per warp (at most)
+  constexpr int R = 16 * T;
+  constexpr int GT = 32 * U;           // threads of the group
+  const StageLayout L(R);
   const UnitIdx x = unit_idx(p, idx);
   const int G = p.c.G;
+  const int gt = w * 32 + lane;
   unsigned char *K0 = stage + L.k0, *K1 = stage + L.k1;
   unsigned char *V0 = stage + L.v0, *V1 = stage + L.v1;
   const unsigned char *KN = stage + L.kn, *VN = stage + L.vn;
   float *SC = reinterpret_cast<float *>(stage + L.sc);
   const int32_t *PS = reinterpret_cast<const int32_t *>(stage + L.ps);
   const int32_t *ST = reinterpret_cast<const int32_t *>(stage + L.st);
+  float *XS = reinterpret_cast<float *>(stage + L.xs);
   const int m = ST[0], t = ST[1], n = m + 1;
-  if (m < 0 || n > p.R) {  // the staged rows cannot hold this unit
-    if (lane == 0) atomicOr(p.c.err, ERR_LENGTH);
+  if (m < 0 || n > R) {  // same decision in every warp of the group
+    if (gt == 0) atomicOr(p.c.err, ERR_LENGTH);
     return;
   }
 
-  // 1. Insert the new row as logical row m (128B-swizzled like the TMA
-  //    boxes) and zero V beyond it, so padded rows contribute 0, not NaN.
-  {
+  // 1. Insert the new row as logical row m (swizzled like the TMA boxes)
+  //    and zero V beyond it, so padded rows contribute 0, not NaN.
+  if (w == 0) {
     const int chunk = lane & 15, half = chunk >> 3, cc = chunk & 7;
     const uint32_t off = m * 128 + ((cc ^ (m & 7)) << 4);
     unsigned char *dst = lane < 16 ? (half ? K1 : K0) : (half ? V1 : V0);
     const unsigned char *src = lane < 16 ? KN : VN;
     *reinterpret_cast<int4 *>(dst + off) =
         *reinterpret_cast<const int4 *>(src + chunk * 16);
-    const int4 z = make_int4(0, 0, 0, 0);
-    for (int r = m + 1 + (lane >> 4); r < p.R; r += 2) {
-      const int c16 = lane & 15;
-      *reinterpret_cast<int4 *>((c16 < 8 ? V0 : V1) + r * 128 + (c16 & 7) * 16) = z;
-    }
   }
-  __syncwarp();
+  for (int i = gt; i < (R - m - 1) * 16; i += GT) {
+    const int r = m + 1 + (i >> 4), c16 = i & 15;
+    *reinterpret_cast<int4 *>((c16 < 8 ? V0 : V1) + r * 128 + (c16 & 7) * 16) =
+        make_int4(0, 0, 0, 0);
+  }
+  group_bar(bar_id, GT);
 
   // 2. Query heads as the MMA B operand (k = head dim, n = query head).
   uint32_t qb[8][2];
@@ -245,12 +262,12 @@ __device__ void process_unit(const FusedParams &p, unsigned char *stage,
               qb[2 * i + 1][1]);
   }
 
-  // 3. Logits: one m16n8 tile per 16 rows, 8 k-steps over the head dim.
-  const int T = (n + 15) >> 4;
-  float acc[8][4];
+  // 3. Logits of the owned tiles: m16n8 per 16 rows, 8 k-steps.
+  float acc[TW][4];
 #pragma unroll
-  for (int tt = 0; tt < 8; ++tt) {
-    acc[tt][0] = acc[tt][1] = acc[tt][2] = acc[tt][3] = 0.f;
+  for (int j = 0; j < TW; ++j) {
+    acc[j][0] = acc[j][1] = acc[j][2] = acc[j][3] = 0.f;
+    const int tt = w + j * U;
     if (tt < T) {
       const int row = tt * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
       const uint32_t b0 = smem_u32(K0) + row * 128, b1 = smem_u32(K1) + row * 128;
@@ -260,103 +277,125 @@ __device__ void process_unit(const FusedParams &p, unsigned char *stage,
         const uint32_t addr = (ks >> 2 ? b1 : b0) + ((cc ^ (row & 7)) << 4);
         uint32_t a0, a1, a2, a3;
         ldsm_x4(addr, a0, a1, a2, a3);
-        mma_bf16(acc[tt], a0, a1, a2, a3, qb[ks][0], qb[ks][1]);
+        mma_bf16(acc[j], a0, a1, a2, a3, qb[ks][0], qb[ks][1]);
       }
     }
   }
 
-  // 4. Softmax per query head (columns c2, c2+1 of this lane).
+  // 4. Softmax per query head: this lane holds columns c2 and c2 + 1.
   const int r0 = lane >> 2, c2 = (lane & 3) * 2;
   float mx0 = -INFINITY, mx1 = -INFINITY;
 #pragma unroll
-  for (int tt = 0; tt < 8; ++tt) {
-    if (tt < T) {
-      const int ra = tt * 16 + r0, rb = ra + 8;
-      acc[tt][0] = ra < n ? acc[tt][0] * p.scale_log2e : -INFINITY;
-      acc[tt][1] = ra < n ? acc[tt][1] * p.scale_log2e : -INFINITY;
-      acc[tt][2] = rb < n ? acc[tt][2] * p.scale_log2e : -INFINITY;
-      acc[tt][3] = rb < n ? acc[tt][3] * p.scale_log2e : -INFINITY;
-      mx0 = fmaxf(mx0, fmaxf(acc[tt][0], acc[tt][2]));
-      mx1 = fmaxf(mx1, fmaxf(acc[tt][1], acc[tt][3]));
-    }
+  for (int j = 0; j < TW; ++j) {
+    const int ra = (w + j * U) * 16 + r0, rb = ra + 8;  // rows >= n masked
+    acc[j][0] = ra < n ? acc[j][0] * p.scale_log2e : -INFINITY;
+    acc[j][1] = ra < n ? acc[j][1] * p.scale_log2e : -INFINITY;
+    acc[j][2] = rb < n ? acc[j][2] * p.scale_log2e : -INFINITY;
+    acc[j][3] = rb < n ? acc[j][3] * p.scale_log2e : -INFINITY;
+    mx0 = fmaxf(mx0, fmaxf(acc[j][0], acc[j][2]));
+    mx1 = fmaxf(mx1, fmaxf(acc[j][1], acc[j][3]));
   }
 #pragma unroll
   for (int o = 4; o < 32; o <<= 1) {
     mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
     mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
   }
+  if (U > 1) {
+    if (lane < 4) {
+      XS[w * kXsWords + c2] = mx0;
+      XS[w * kXsWords + c2 + 1] = mx1;
+    }
+    group_bar(bar_id, GT);
+#pragma unroll
+    for (int v = 0; v < U; ++v) {
+      mx0 = fmaxf(mx0, XS[v * kXsWords + c2]);
+      mx1 = fmaxf(mx1, XS[v * kXsWords + c2 + 1]);
+    }
+  }
   float z0 = 0.f, z1 = 0.f;
 #pragma unroll
-  for (int tt = 0; tt < 8; ++tt) {
-    if (tt < T) {
-      acc[tt][0] = exp2f(acc[tt][0] - mx0);
-      acc[tt][1] = exp2f(acc[tt][1] - mx1);
-      acc[tt][2] = exp2f(acc[tt][2] - mx0);
-      acc[tt][3] = exp2f(acc[tt][3] - mx1);
-      z0 += acc[tt][0] + acc[tt][2];
-      z1 += acc[tt][1] + acc[tt][3];
-    }
+  for (int j = 0; j < TW; ++j) {
+    acc[j][0] = exp2f(acc[j][0] - mx0);
+    acc[j][1] = exp2f(acc[j][1] - mx1);
+    acc[j][2] = exp2f(acc[j][2] - mx0);
+    acc[j][3] = exp2f(acc[j][3] - mx1);
+    z0 += acc[j][0] + acc[j][2];
+    z1 += acc[j][1] + acc[j][3];
   }
 #pragma unroll
   for (int o = 4; o < 32; o <<= 1) {
     z0 += __shfl_xor_sync(0xffffffffu, z0, o);
     z1 += __shfl_xor_sync(0xffffffffu, z1, o);
   }
-  if (lane == 0 && (!(z0 >= 1.f) || !(z0 < INFINITY)))
+  if (U > 1) {
+    if (lane < 4) {
+      XS[w * kXsWords + 8 + c2] = z0;
+      XS[w * kXsWords + 8 + c2 + 1] = z1;
+    }
+    group_bar(bar_id, GT);
+    z0 = z1 = 0.f;
+#pragma unroll
+    for (int v = 0; v < U; ++v) {
+      z0 += XS[v * kXsWords + 8 + c2];
+      z1 += XS[v * kXsWords + 8 + c2 + 1];
+    }
+  }
+  if (gt == 0 && (!(z0 >= 1.f) || !(z0 < INFINITY)))
     atomicOr(p.c.err, ERR_NONFINITE);
   const float i0 = 1.f / z0, i1 = 1.f / z1;
 
-  // 5. Accumulated attention: score += mean over the G heads (staged copy).
+  // 5. Accumulated attention: score += mean over the G heads (staged copy;
+  //    every row belongs to exactly one warp).
   const bool g0 = c2 < G, g1 = c2 + 1 < G;
 #pragma unroll
-  for (int tt = 0; tt < 8; ++tt) {
-    if (tt < T) {
-      acc[tt][0] *= i0;
-      acc[tt][2] *= i0;
-      acc[tt][1] *= i1;
-      acc[tt][3] *= i1;
-      float sa = (g0 ? acc[tt][0] : 0.f) + (g1 ? acc[tt][1] : 0.f);
-      float sb = (g0 ? acc[tt][2] : 0.f) + (g1 ? acc[tt][3] : 0.f);
-      sa += __shfl_xor_sync(0xffffffffu, sa, 1);
-      sb += __shfl_xor_sync(0xffffffffu, sb, 1);
-      sa += __shfl_xor_sync(0xffffffffu, sa, 2);
-      sb += __shfl_xor_sync(0xffffffffu, sb, 2);
-      if ((lane & 3) == 0) {
-        const int ra = tt * 16 + r0, rb = ra + 8;
-        if (ra < m) SC[ra] += sa * p.inv_g;
-        else if (ra == m) SC[ra] = sa * p.inv_g;
-        if (rb < m) SC[rb] += sb * p.inv_g;
-        else if (rb == m) SC[rb] = sb * p.inv_g;
-      }
+  for (int j = 0; j < TW; ++j) {
+    acc[j][0] *= i0;
+    acc[j][2] *= i0;
+    acc[j][1] *= i1;
+    acc[j][3] *= i1;
+    float sa = (g0 ? acc[j][0] : 0.f) + (g1 ? acc[j][1] : 0.f);
+    float sb = (g0 ? acc[j][2] : 0.f) + (g1 ? acc[j][3] : 0.f);
+    sa += __shfl_xor_sync(0xffffffffu, sa, 1);
+    sb += __shfl_xor_sync(0xffffffffu, sb, 1);
+    sa += __shfl_xor_sync(0xffffffffu, sa, 2);
+    sb += __shfl_xor_sync(0xffffffffu, sb, 2);
+    if ((lane & 3) == 0) {
+      const int ra = (w + j * U) * 16 + r0, rb = ra + 8;
+      if (ra < m) SC[ra] += sa * p.inv_g;
+      else if (ra == m) SC[ra] = sa * p.inv_g;
+      if (rb < m) SC[rb] += sb * p.inv_g;
+      else if (rb == m) SC[rb] = sb * p.inv_g;
     }
   }
 
   // 6. P as the PV B operand, split into two bf16 terms (hi + lo carries
-  //    ~16 mantissa bits: a single bf16 P would cost up to 2^-9 relative per
-  //    probability), each 8x8 block transposed in registers.
-  uint32_t bp[8][2], bl[8][2];
+  //    ~16 mantissa bits; a single bf16 P would cost up to 2^-9 relative
+  //    per probability), each 8x8 block transposed in registers.
+  uint32_t bp[TW][2], bl[TW][2];
 #pragma unroll
-  for (int tt = 0; tt < 8; ++tt) {
-    const uint32_t h0 = pack_bf16(acc[tt][0], acc[tt][1]);
-    const uint32_t h1 = pack_bf16(acc[tt][2], acc[tt][3]);
+  for (int j = 0; j < TW; ++j) {
+    const uint32_t h0 = pack_bf16(acc[j][0], acc[j][1]);
+    const uint32_t h1 = pack_bf16(acc[j][2], acc[j][3]);
     const __nv_bfloat162 hb0 = *reinterpret_cast<const __nv_bfloat162 *>(&h0);
     const __nv_bfloat162 hb1 = *reinterpret_cast<const __nv_bfloat162 *>(&h1);
-    const uint32_t l0 = pack_bf16(acc[tt][0] - __low2float(hb0),
-                                  acc[tt][1] - __high2float(hb0));
-    const uint32_t l1 = pack_bf16(acc[tt][2] - __low2float(hb1),
-                                  acc[tt][3] - __high2float(hb1));
-    bp[tt][0] = movm_t(h0);
-    bp[tt][1] = movm_t(h1);
-    bl[tt][0] = movm_t(l0);
-    bl[tt][1] = movm_t(l1);
+    const uint32_t l0 = pack_bf16(acc[j][0] - __low2float(hb0),
+                                  acc[j][1] - __high2float(hb0));
+    const uint32_t l1 = pack_bf16(acc[j][2] - __low2float(hb1),
+                                  acc[j][3] - __high2float(hb1));
+    bp[j][0] = movm_t(h0);
+    bp[j][1] = movm_t(h1);
+    bl[j][0] = movm_t(l0);
+    bl[j][1] = movm_t(l1);
   }
 
-  // 7. out^T = V^T P^T: M = head dim (8 tiles of 16), K = rows, N = heads.
+  // 7. Partial out^T = V^T P^T over the owned tiles: M = head dim (8 tiles
+  //    of 16), K = rows, N = query heads.
   float o[8][4];
 #pragma unroll
   for (int mt = 0; mt < 8; ++mt) o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.f;
 #pragma unroll
-  for (int tt = 0; tt < 8; ++tt) {
+  for (int j = 0; j < TW; ++j) {
+    const int tt = w + j * U;
     if (tt < T) {
       const int row = tt * 16 + (lane & 7) + ((lane >> 4) << 3);
       const uint32_t b0 = smem_u32(V0) + row * 128, b1 = smem_u32(V1) + row * 128;
@@ -366,50 +405,72 @@ __device__ void process_unit(const FusedParams &p, unsigned char *stage,
         const uint32_t addr = (c16 >> 3 ? b1 : b0) + (((c16 & 7) ^ (row & 7)) << 4);
         uint32_t a0, a1, a2, a3;
         ldsm_x4_t(addr, a0, a1, a2, a3);
-        mma_bf16(o[mt], a0, a1, a2, a3, bp[tt][0], bp[tt][1]);
-        mma_bf16(o[mt], a0, a1, a2, a3, bl[tt][0], bl[tt][1]);
+        mma_bf16(o[mt], a0, a1, a2, a3, bp[j][0], bp[j][1]);
+        mma_bf16(o[mt], a0, a1, a2, a3, bl[j][0], bl[j][1]);
       }
     }
   }
 
-  // 8. Output rows: stage them in the (now free) K area, then 16-byte stores.
-  __syncwarp();
-  {
-    constexpr int osz = kOutBf16 ? 2 : 4;
-    constexpr int pitch = 128 * osz + 16;
-    unsigned char *OUT = K0;
+  // 8. Sum the partials across the group (K area, free since every warp has
+  //    passed the softmax exchange), stage the output rows in the V area
+  //    (free once every warp has finished PV) and store them.
+  constexpr int osz = kOutBf16 ? 2 : 4;
+  const int pitch = 128 * osz + (G * (128 * osz + 16) <= 2 * R * 128 ? 16 : 0);
+  unsigned char *OUT = V0;
+  if (U > 1) {
+    float *XO = reinterpret_cast<float *>(K0);
+#pragma unroll
+    for (int mt = 0; mt < 8; ++mt)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) XO[((w * 8 + mt) * 4 + e) * 32 + lane] = o[mt][e];
+    group_bar(bar_id, GT);
 #pragma unroll
     for (int mt = 0; mt < 8; ++mt) {
-      const int d0 = 16 * mt + r0;
-      if (kOutBf16) {
-        __nv_bfloat16 *o0 = reinterpret_cast<__nv_bfloat16 *>(OUT + c2 * pitch);
-        __nv_bfloat16 *o1 = reinterpret_cast<__nv_bfloat16 *>(OUT + (c2 + 1) * pitch);
-        if (g0) {
-          o0[d0] = __float2bfloat16_rn(o[mt][0]);
-          o0[d0 + 8] = __float2bfloat16_rn(o[mt][2]);
-        }
-        if (g1) {
-          o1[d0] = __float2bfloat16_rn(o[mt][1]);
-          o1[d0 + 8] = __float2bfloat16_rn(o[mt][3]);
-        }
-      } else {
-        float *o0 = reinterpret_cast<float *>(OUT + c2 * pitch);
-        float *o1 = reinterpret_cast<float *>(OUT + (c2 + 1) * pitch);
-        if (g0) {
-          o0[d0] = o[mt][0];
-          o0[d0 + 8] = o[mt][2];
-        }
-        if (g1) {
-          o1[d0] = o[mt][1];
-          o1[d0 + 8] = o[mt][3];
+      if (mt % U == w) {
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          float sum = 0.f;
+#pragma unroll
+          for (int v = 0; v < U; ++v) sum += XO[((v * 8 + mt) * 4 + e) * 32 + lane];
+          o[mt][e] = sum;
         }
       }
     }
-    __syncwarp();
+  }
+#pragma unroll
+  for (int mt = 0; mt < 8; ++mt) {
+    if (mt % U != w) continue;
+    const int d0 = 16 * mt + r0;
+    if (kOutBf16) {
+      __nv_bfloat16 *o0 = reinterpret_cast<__nv_bfloat16 *>(OUT + c2 * pitch);
+      __nv_bfloat16 *o1 = reinterpret_cast<__nv_bfloat16 *>(OUT + (c2 + 1) * pitch);
+      if (g0) {
+        o0[d0] = __float2bfloat16_rn(o[mt][0]);
+        o0[d0 + 8] = __float2bfloat16_rn(o[mt][2]);
+      }
+      if (g1) {
+        o1[d0] = __float2bfloat16_rn(o[mt][1]);
+        o1[d0 + 8] = __float2bfloat16_rn(o[mt][3]);
+      }
+    } else {
+      float *o0 = reinterpret_cast<float *>(OUT + c2 * pitch);
+      float *o1 = reinterpret_cast<float *>(OUT + (c2 + 1) * pitch);
+      if (g0) {
+        o0[d0] = o[mt][0];
+        o0[d0 + 8] = o[mt][2];
+      }
+      if (g1) {
+        o1[d0] = o[mt][1];
+        o1[d0 + 8] = o[mt][3];
+      }
+    }
+  }
+  group_bar(bar_id, GT);
+  {
     constexpr int cpr = 128 * osz / 16;  // 16-byte chunks per output row
     unsigned char *gout = reinterpret_cast<unsigned char *>(p.out) +
                           x.krow * G * 128 * osz;
-    for (int i = lane; i < G * cpr; i += 32) {
+    for (int i = gt; i < G * cpr; i += GT) {
       const int g = i / cpr, ch = i % cpr;
       *reinterpret_cast<int4 *>(gout + (size_t)g * 128 * osz + ch * 16) =
           *reinterpret_cast<const int4 *>(OUT + g * pitch + ch * 16);
@@ -422,7 +483,7 @@ __device__ void process_unit(const FusedParams &p, unsigned char *stage,
     const int wlo = t - p.window;
     unsigned long long best = ~0ull;
     int bi = -1;
-    for (int i = lane; i < n; i += 32) {
+    for (int i = gt; i < n; i += GT) {
       const int pi = i < m ? PS[i] : t;
       if (pi <= wlo) {
         const unsigned long long key =
@@ -443,37 +504,57 @@ __device__ void process_unit(const FusedParams &p, unsigned char *stage,
         bi = oi;
       }
     }
+    if (U > 1) {
+      uint32_t *XW = reinterpret_cast<uint32_t *>(XS);
+      if (lane == 0) {
+        XW[w * kXsWords + 16] = (uint32_t)best;
+        XW[w * kXsWords + 17] = (uint32_t)(best >> 32);
+        XW[w * kXsWords + 18] = (uint32_t)bi;
+      }
+      group_bar(bar_id, GT);
+#pragma unroll
+      for (int v = 0; v < U; ++v) {
+        const unsigned long long kb =
+            ((unsigned long long)XW[v * kXsWords + 17] << 32) | XW[v * kXsWords + 16];
+        if (kb < best) {
+          best = kb;
+          bi = (int)XW[v * kXsWords + 18];
+        }
+      }
+    }
     victim = bi;
   }
 
-  // 10. Write back: scores of the kept rows, the new row into the freed slot
-  //     (or the first free slot when nothing is evicted), length and position.
+  // 10. Write back the kept rows' scores, the new row into the freed slot (or
+  //     the first free slot when nothing is evicted), length and position.
   float *gsc = p.c.score + x.ug * p.c.sstride;
   int32_t *gps = p.c.pos + x.ug * p.c.sstride;
   const float new_score = SC[m];
-  for (int i = lane; i < m; i += 32) gsc[i] = i == victim ? new_score : SC[i];
+  for (int i = gt; i < m; i += GT) gsc[i] = i == victim ? new_score : SC[i];
   const int slot = victim < 0 ? m : (victim < m ? victim : -1);
-  if (slot >= 0) {
-    const int chunk = lane & 15;
-    __nv_bfloat16 *dst =
-        reinterpret_cast<__nv_bfloat16 *>(lane < 16 ? p.c.K : p.c.V) +
-        (x.ug * (size_t)p.c.cap + slot) * 128;
-    const unsigned char *src = lane < 16 ? KN : VN;
-    reinterpret_cast<int4 *>(dst)[chunk] =
-        *reinterpret_cast<const int4 *>(src + chunk * 16);
-    if (lane == 0) {
-      gps[slot] = t;
-      if (slot == m) gsc[m] = new_score;
+  if (w == 0) {
+    if (slot >= 0) {
+      const int chunk = lane & 15;
+      __nv_bfloat16 *dst =
+          reinterpret_cast<__nv_bfloat16 *>(lane < 16 ? p.c.K : p.c.V) +
+          (x.ug * (size_t)p.c.cap + slot) * 128;
+      const unsigned char *src = lane < 16 ? KN : VN;
+      reinterpret_cast<int4 *>(dst)[chunk] =
+          *reinterpret_cast<const int4 *>(src + chunk * 16);
+      if (lane == 0) {
+        gps[slot] = t;
+        if (slot == m) gsc[m] = new_score;
+      }
     }
-  }
-  if (lane == 0) {
-    p.c.state[4 * x.ug] = victim < 0 ? m + 1 : m;
-    p.c.state[4 * x.ug + 1] = t + 1;
+    if (lane == 0) {
+      p.c.state[4 * x.ug] = victim < 0 ? m + 1 : m;
+      p.c.state[4 * x.ug + 1] = t + 1;
+    }
   }
 }
 
-template <bool kOutBf16>
-__global__ void __launch_bounds__(32 * (kMaxConsumers + 1), 1)
+template <int T, int U, bool kOutBf16>
+__global__ void __launch_bounds__(kMaxThreads, 1)
     fused_step_kernel(const __grid_constant__ CUtensorMap tmK,
                       const __grid_constant__ CUtensorMap tmV,
                       const FusedParams p) {
@@ -483,6 +564,7 @@ __global__ void __launch_bounds__(32 * (kMaxConsumers + 1), 1)
   __shared__ int issued_k[kMaxStages];
   __shared__ int consumed_k[kMaxStages];
   __shared__ volatile int s_abort;
+  __shared__ volatile int s_ok[kMaxGroups];
   unsigned char *smem = reinterpret_cast<unsigned char *>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -490,7 +572,8 @@ __global__ void __launch_bounds__(32 * (kMaxConsumers + 1), 1)
   const int mine = (int)blockIdx.x < n_units
                        ? (n_units - 1 - (int)blockIdx.x) / (int)gridDim.x + 1
                        : 0;
-  const StageLayout L(p.R);
+  const StageLayout L(16 * T);
+  const int consumers = p.n_groups * U;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < p.n_stages; ++s) {
@@ -512,7 +595,7 @@ __global__ void __launch_bounds__(32 * (kMaxConsumers + 1), 1)
   fence_proxy_async();
   __syncthreads();
 
-  if (warp == p.n_consumers) {
+  if (warp == consumers) {
     if (lane == 0) {
       for (int k = 0; k < mine; ++k) {
         const int s = k % p.n_stages;
@@ -527,22 +610,32 @@ __global__ void __launch_bounds__(32 * (kMaxConsumers + 1), 1)
         issued_k[s] = k;
       }
     }
-  } else if (warp < p.n_consumers) {
-    for (int k = warp; k < mine; k += p.n_consumers) {
+  } else if (warp < consumers) {
+    const int grp = warp / U, w = warp % U, bar_id = 1 + grp;
+    for (int k = grp; k < mine; k += p.n_groups) {
       const int s = k % p.n_stages;
       const uint32_t ph = (uint32_t)(k / p.n_stages) & 1u;
-      if (!mbar_wait(smem_u32(&full_bar[s]), ph, &s_abort)) {
+      // One warp waits (bounded) and tells the group, so that every warp
+      // of the group takes the same branch before the next named barrier.
+      if (w == 0) {
+        const bool ok = mbar_wait(smem_u32(&full_bar[s]), ph, &s_abort);
         if (lane == 0) {
-          atomicOr(p.c.err, ERR_TIMEOUT);
-          s_abort = 1;
+          s_ok[grp] = ok ? 1 : 0;
+          if (!ok) {
+            atomicOr(p.c.err, ERR_TIMEOUT);
+            s_abort = 1;
+          }
         }
-        break;
       }
-      process_unit<kOutBf16>(p, smem + s * L.bytes,
-                             (int)blockIdx.x + k * (int)gridDim.x, lane);
+      group_bar(bar_id, 32 * U);
+      if (!s_ok[grp]) break;
+      mbar_try_wait(smem_u32(&full_bar[s]), ph);  // acquire for this thread
+      process_unit<T, U, kOutBf16>(p, smem + s * L.bytes,
+                                   (int)blockIdx.x + k * (int)gridDim.x, w,
+                                   lane, bar_id);
       fence_proxy_async();
-      __syncwarp();
-      if (lane == 0) {
+      group_bar(bar_id, 32 * U);
+      if (w == 0 && lane == 0) {
         consumed_k[s] = k;
         mbar_arrive(smem_u32(&empty_bar[s]));
       }
@@ -561,29 +654,56 @@ __global__ void __launch_bounds__(32 * (kMaxConsumers + 1), 1)
   }
 }
 
+template <int T, int U, bool kOutBf16>
+cudaError_t launch_tu(const CUtensorMap &tmK, const CUtensorMap &tmV,
+                      const FusedParams &p, int grid, int smem_bytes,
+                      cudaStream_t st) {
+  auto kern = fused_step_kernel<T, U, kOutBf16>;
+  cudaError_t e = cudaFuncSetAttribute(
+      kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
+  if (e != cudaSuccess) return e;
+  const int threads = 32 * (p.n_groups * U + 1);
+  kern<<<grid, threads, smem_bytes, st>>>(tmK, tmV, p);
+  return cudaGetLastError();
+}
+
+template <bool kOutBf16>
+cudaError_t launch_t(const CUtensorMap &tmK, const CUtensorMap &tmV,
+                     const FusedParams &p, int grid, int smem_bytes,
+                     cudaStream_t st) {
+  switch (p.R / 16) {
+    case 1: return launch_tu<1, 1, kOutBf16>(tmK, tmV, p, grid, smem_bytes, st);
+    case 2: return launch_tu<2, 2, kOutBf16>(tmK, tmV, p, grid, smem_bytes, st);
+    case 3: return launch_tu<3, 3, kOutBf16>(tmK, tmV, p, grid, smem_bytes, st);
+    case 4: return launch_tu<4, 4, kOutBf16>(tmK, tmV, p, grid, smem_bytes, st);
+    case 5: return launch_tu<5, 5, kOutBf16>(tmK, tmV, p, grid, smem_bytes, st);
+    case 6: return launch_tu<6, 3, kOutBf16>(tmK, tmV, p, grid, smem_bytes, st);
+    case 7: return launch_tu<7, 4, kOutBf16>(tmK, tmV, p, grid, smem_bytes, st);
+    case 8: return launch_tu<8, 4, kOutBf16>(tmK, tmV, p, grid, smem_bytes, st);
+  }
+  return cudaErrorInvalidValue;
+}
+
 }  // namespace
 
 int fused_stage_bytes(int R) { return (int)StageLayout(R).bytes; }
 
+int fused_group_warps(int R) {
+  static const int u[9] = {0, 1, 2, 3, 4, 5, 3, 4, 4};
+  return (R % 16 == 0 && R >= 16 && R <= 128) ? u[R / 16] : 0;
+}
+
+int fused_max_threads() { return kMaxThreads; }
+
 cudaError_t launch_fused_step(const CUtensorMap &tmK, const CUtensorMap &tmV,
                               const FusedParams &p, int grid, int smem_bytes,
                               cudaStream_t st) {
-  const int threads = 32 * (p.n_consumers + 1);
-  cudaError_t e;
-  if (p.c.out_bf16) {
-    e = cudaFuncSetAttribute(fused_step_kernel<true>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             smem_bytes);
-    if (e != cudaSuccess) return e;
-    fused_step_kernel<true><<<grid, threads, smem_bytes, st>>>(tmK, tmV, p);
-  } else {
-    e = cudaFuncSetAttribute(fused_step_kernel<false>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             smem_bytes);
-    if (e != cudaSuccess) return e;
-    fused_step_kernel<false><<<grid, threads, smem_bytes, st>>>(tmK, tmV, p);
-  }
-  return cudaGetLastError();
+  if (fused_group_warps(p.R) == 0 || p.n_groups < 1 ||
+      p.n_groups > kMaxGroups || p.n_stages > kMaxStages ||
+      32 * (p.n_groups * fused_group_warps(p.R) + 1) > kMaxThreads)
+    return cudaErrorInvalidValue;
+  return p.c.out_bf16 ? launch_t<true>(tmK, tmV, p, grid, smem_bytes, st)
+                      : launch_t<false>(tmK, tmV, p, grid, smem_bytes, st);
 }
 
 }  // namespace kvr

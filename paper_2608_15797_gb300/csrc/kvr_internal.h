@@ -74,11 +74,14 @@ struct FusedParams {
   void *out;                   // [S][nl][H*G][128]
   int lb, nl;
   int R;                       // staged rows per unit (multiple of 16, <= 128)
-  int n_stages, n_consumers;   // shared-memory ring depth, consumer warps
+  int Rb;                      // rows copied from a slab (multiple of 8, <= R)
+  int n_stages, n_groups;      // ring depth; units computed at once
   int budget, window, evict;
   float scale_log2e, inv_g;
 };
 int fused_stage_bytes(int R);
+int fused_group_warps(int R);  // warps that share one unit of R staged rows
+int fused_max_threads();
 cudaError_t launch_fused_step(const CUtensorMap &tmK, const CUtensorMap &tmV,
                               const FusedParams &p, int grid, int smem_bytes,
                               cudaStream_t st);
