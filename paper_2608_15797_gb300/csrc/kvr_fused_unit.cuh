@@ -1,0 +1,367 @@
+// kvr_fused_unit.cuh -- the per-unit body of the fused decode-step kernel
+// (included by kvr_fused.cu only).
+//
+// One group of U warps computes one (sequence, layer, KV head) unit held in
+// a shared-memory stage.  The unit has T = R / 16 row tiles; warp w of the
+// group owns tiles w, w + U, ... and everything about their rows: inserting
+// the new row if it falls in an owned tile, the logits, probabilities,
+// accumulated-attention scores, eviction candidates and the PV partial sums.
+// The group meets at two named barriers per unit: one to merge the softmax
+// statistics and one to sum the PV partials and agree on the evicted row.
+//
+// Exchange words per warp (XS): [0,8) column max, [8,16) column sum under
+// that max, [16,18) argmin key, 18 argmin row.
+
+template <int T, int U, bool kOutBf16>
+__device__ void process_unit(const FusedParams &p, unsigned char *stage,
+                             int idx, int w, int lane, int bar_id) {
+  constexpr int TW = (T + U - 1) / U;  // tiles per warp (at most)
+  constexpr int R = 16 * T;
+  constexpr int GT = 32 * U;           // threads of the group
+  const StageLayout L(R);
+  const UnitIdx x = unit_idx(p, idx);
+  const int G = p.c.G;
+  unsigned char *K0 = stage + L.k0, *K1 = stage + L.k1;
+  unsigned char *V0 = stage + L.v0, *V1 = stage + L.v1;
+  const unsigned char *KN = stage + L.kn, *VN = stage + L.vn;
+  const float *SC = reinterpret_cast<const float *>(stage + L.sc);
+  const int32_t *PS = reinterpret_cast<const int32_t *>(stage + L.ps);
+  const int32_t *ST = reinterpret_cast<const int32_t *>(stage + L.st);
+  float *XS = reinterpret_cast<float *>(stage + L.xs);
+  const int m = ST[0], t = ST[1], n = m + 1;
+  if (m < 0 || n > R) {  // same decision in every warp of the group
+    if (w == 0 && lane == 0) atomicOr(p.c.err, ERR_LENGTH);
+    return;
+  }
+  const bool own_new = ((m >> 4) % U) == w;  // this warp owns row m's tile
+
+  // 1. Insert the new row as logical row m (swizzled like the TMA boxes) and
+  //    zero V beyond it in the owned tiles, so padded rows contribute 0.
+  if (own_new) {
+    const int chunk = lane & 15, half = chunk >> 3, cc = chunk & 7;
+    const uint32_t off = m * 128 + ((cc ^ (m & 7)) << 4);
+    unsigned char *dst = lane < 16 ? (half ? K1 : K0) : (half ? V1 : V0);
+    const unsigned char *src = lane < 16 ? KN : VN;
+    *reinterpret_cast<int4 *>(dst + off) =
+        *reinterpret_cast<const int4 *>(src + chunk * 16);
+  }
+#pragma unroll
+  for (int j = 0; j < TW; ++j) {
+    const int tt = w + j * U;
+    const int r_lo = max(tt * 16, m + 1), r_hi = tt * 16 + 16;
+    if (tt < T && r_lo < r_hi)
+      for (int i = lane; i < (r_hi - r_lo) * 16; i += 32) {
+        const int r = r_lo + (i >> 4), c16 = i & 15;
+        *reinterpret_cast<int4 *>((c16 < 8 ? V0 : V1) + r * 128 +
+                                  (c16 & 7) * 16) = make_int4(0, 0, 0, 0);
+      }
+  }
+  __syncwarp();
+
+  // 2. Query heads as the MMA B operand (k = head dim, n = query head).
+  uint32_t qb[8][2];
+  {
+    const uint32_t qa = smem_u32(stage + L.q) + (lane & 7) * kQPitch +
+                        (lane >> 3) * 16;
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+      ldsm_x4(qa + i * 64, qb[2 * i][0], qb[2 * i][1], qb[2 * i + 1][0],
+              qb[2 * i + 1][1]);
+  }
+
+  // 3. Logits of the owned tiles: m16n8 per 16 rows, 8 k-steps split over
+  //    two accumulator chains.
+  float acc[TW][4];
+#pragma unroll
+  for (int j = 0; j < TW; ++j) {
+    float a2[4] = {0.f, 0.f, 0.f, 0.f};
+    acc[j][0] = acc[j][1] = acc[j][2] = acc[j][3] = 0.f;
+    const int tt = w + j * U;
+    if (tt < T) {
+      const int row = tt * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+      const uint32_t b0 = smem_u32(K0) + row * 128, b1 = smem_u32(K1) + row * 128;
+#pragma unroll
+      for (int ks = 0; ks < 8; ++ks) {
+        const int cc = ((ks & 3) << 1) + (lane >> 4);
+        const uint32_t addr = (ks >> 2 ? b1 : b0) + ((cc ^ (row & 7)) << 4);
+        uint32_t a0, a1, a2r, a3;
+        ldsm_x4(addr, a0, a1, a2r, a3);
+        if (ks & 1)
+          mma_bf16(a2, a0, a1, a2r, a3, qb[ks][0], qb[ks][1]);
+        else
+          mma_bf16(acc[j], a0, a1, a2r, a3, qb[ks][0], qb[ks][1]);
+      }
+#pragma unroll
+      for (int e = 0; e < 4; ++e) acc[j][e] += a2[e];
+    }
+  }
+
+  // 4. Softmax per query head (this lane holds columns c2 and c2 + 1): the
+  //    warp's (max, sum) per column, merged across the group in one round.
+  const int r0 = lane >> 2, c2 = (lane & 3) * 2;
+  float mx0 = -INFINITY, mx1 = -INFINITY;
+#pragma unroll
+  for (int j = 0; j < TW; ++j) {
+    const int ra = (w + j * U) * 16 + r0, rb = ra + 8;  // rows >= n masked
+    acc[j][0] = ra < n ? acc[j][0] * p.scale_log2e : -INFINITY;
+    acc[j][1] = ra < n ? acc[j][1] * p.scale_log2e : -INFINITY;
+    acc[j][2] = rb < n ? acc[j][2] * p.scale_log2e : -INFINITY;
+    acc[j][3] = rb < n ? acc[j][3] * p.scale_log2e : -INFINITY;
+    mx0 = fmaxf(mx0, fmaxf(acc[j][0], acc[j][2]));
+    mx1 = fmaxf(mx1, fmaxf(acc[j][1], acc[j][3]));
+  }
+#pragma unroll
+  for (int o = 4; o < 32; o <<= 1) {
+    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
+    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
+  }
+  // A warp whose rows are all padding has max -inf: use 0 as its reference
+  // so that exp2(-inf - 0) = 0 instead of NaN.
+  const float ref0 = mx0 == -INFINITY ? 0.f : mx0;
+  const float ref1 = mx1 == -INFINITY ? 0.f : mx1;
+  float z0 = 0.f, z1 = 0.f;
+#pragma unroll
+  for (int j = 0; j < TW; ++j) {
+    acc[j][0] = exp2f(acc[j][0] - ref0);
+    acc[j][1] = exp2f(acc[j][1] - ref1);
+    acc[j][2] = exp2f(acc[j][2] - ref0);
+    acc[j][3] = exp2f(acc[j][3] - ref1);
+    z0 += acc[j][0] + acc[j][2];
+    z1 += acc[j][1] + acc[j][3];
+  }
+#pragma unroll
+  for (int o = 4; o < 32; o <<= 1) {
+    z0 += __shfl_xor_sync(0xffffffffu, z0, o);
+    z1 += __shfl_xor_sync(0xffffffffu, z1, o);
+  }
+  float f0 = 1.f / z0, f1 = 1.f / z1;  // this warp's rescale factors
+  if (U > 1) {
+    if (lane < 4) {
+      XS[w * kXsWords + c2] = ref0;
+      XS[w * kXsWords + c2 + 1] = ref1;
+      XS[w * kXsWords + 8 + c2] = z0;
+      XS[w * kXsWords + 8 + c2 + 1] = z1;
+    }
+    group_bar(bar_id, GT);
+    // Warps with no live row (z = 0) take no part in the merge.
+    float M0 = -INFINITY, M1 = -INFINITY;
+#pragma unroll
+    for (int v = 0; v < U; ++v) {
+      if (XS[v * kXsWords + 8 + c2] > 0.f) M0 = fmaxf(M0, XS[v * kXsWords + c2]);
+      if (XS[v * kXsWords + 8 + c2 + 1] > 0.f)
+        M1 = fmaxf(M1, XS[v * kXsWords + c2 + 1]);
+    }
+    float Z0 = 0.f, Z1 = 0.f;
+#pragma unroll
+    for (int v = 0; v < U; ++v) {
+      const float za = XS[v * kXsWords + 8 + c2], zb = XS[v * kXsWords + 8 + c2 + 1];
+      if (za > 0.f) Z0 += za * exp2f(XS[v * kXsWords + c2] - M0);
+      if (zb > 0.f) Z1 += zb * exp2f(XS[v * kXsWords + c2 + 1] - M1);
+    }
+    f0 = z0 > 0.f ? exp2f(ref0 - M0) / Z0 : 0.f;
+    f1 = z1 > 0.f ? exp2f(ref1 - M1) / Z1 : 0.f;
+    z0 = Z0;  // >= 1: the warp holding the maximum contributes exp2(0)
+  }
+  if (w == 0 && lane == 0 && !(z0 >= 1.f && z0 < INFINITY))
+    atomicOr(p.c.err, ERR_NONFINITE);
+
+  // 5. Probabilities; accumulated attention of the owned rows (score += mean
+  //    over the G heads), written back at once except for the new row; the
+  //    warp's eviction candidate (lowest (score, -position) outside the
+  //    window).
+  const bool g0 = c2 < G, g1 = c2 + 1 < G;
+  const int wlo = t - p.window;  // a row is a candidate iff pos <= wlo
+  float *gsc = p.c.score + x.ug * p.c.sstride;
+  unsigned long long best = ~0ull;
+  int bi = -1;
+  float new_score = 0.f;
+#pragma unroll
+  for (int j = 0; j < TW; ++j) {
+    acc[j][0] *= f0;
+    acc[j][2] *= f0;
+    acc[j][1] *= f1;
+    acc[j][3] *= f1;
+    float sa = (g0 ? acc[j][0] : 0.f) + (g1 ? acc[j][1] : 0.f);
+    float sb = (g0 ? acc[j][2] : 0.f) + (g1 ? acc[j][3] : 0.f);
+    sa += __shfl_xor_sync(0xffffffffu, sa, 1);
+    sb += __shfl_xor_sync(0xffffffffu, sb, 1);
+    sa += __shfl_xor_sync(0xffffffffu, sa, 2);
+    sb += __shfl_xor_sync(0xffffffffu, sb, 2);
+    const int tt = w + j * U;
+    if ((lane & 3) == 0 && tt < T) {
+#pragma unroll
+      for (int hsel = 0; hsel < 2; ++hsel) {
+        const int r = tt * 16 + r0 + 8 * hsel;
+        if (r < n) {
+          const float s = (r < m ? SC[r] : 0.f) + (hsel ? sb : sa) * p.inv_g;
+          if (r < m) gsc[r] = s;
+          else new_score = s;
+          const int pr = r < m ? PS[r] : t;
+          if (pr <= wlo) {
+            const unsigned long long key =
+                ((unsigned long long)__float_as_uint(s) << 32) |
+                (unsigned long long)(0xFFFFFFFFu - (unsigned)pr);
+            if (key < best) {
+              best = key;
+              bi = r;
+            }
+          }
+        }
+      }
+    }
+  }
+  // The lane that scored the new row passes its score to the whole warp.
+  new_score = __shfl_sync(0xffffffffu, new_score, ((m & 15) & 7) * 4);
+#pragma unroll
+  for (int o2 = 16; o2 > 0; o2 >>= 1) {
+    const unsigned long long ob = __shfl_xor_sync(0xffffffffu, best, o2);
+    const int oi = __shfl_xor_sync(0xffffffffu, bi, o2);
+    if (ob < best) {
+      best = ob;
+      bi = oi;
+    }
+  }
+
+  // 6. P as the PV B operand, split into two bf16 terms (hi + lo carries
+  //    ~16 mantissa bits; a single bf16 P would cost up to 2^-9 relative
+  //    per probability), each 8x8 block transposed in registers.
+  uint32_t bp[TW][2], bl[TW][2];
+#pragma unroll
+  for (int j = 0; j < TW; ++j) {
+    const uint32_t h0 = pack_bf16(acc[j][0], acc[j][1]);
+    const uint32_t h1 = pack_bf16(acc[j][2], acc[j][3]);
+    const __nv_bfloat162 hb0 = *reinterpret_cast<const __nv_bfloat162 *>(&h0);
+    const __nv_bfloat162 hb1 = *reinterpret_cast<const __nv_bfloat162 *>(&h1);
+    const uint32_t l0 = pack_bf16(acc[j][0] - __low2float(hb0),
+                                  acc[j][1] - __high2float(hb0));
+    const uint32_t l1 = pack_bf16(acc[j][2] - __low2float(hb1),
+                                  acc[j][3] - __high2float(hb1));
+    bp[j][0] = movm_t(h0);
+    bp[j][1] = movm_t(h1);
+    bl[j][0] = movm_t(l0);
+    bl[j][1] = movm_t(l1);
+  }
+
+  // 7. Partial out^T = V^T P^T over the owned tiles: M = head dim (8 tiles
+  //    of 16), K = rows, N = query heads.
+  float o[8][4];
+#pragma unroll
+  for (int mt = 0; mt < 8; ++mt) o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.f;
+#pragma unroll
+  for (int j = 0; j < TW; ++j) {
+    const int tt = w + j * U;
+    if (tt < T) {
+      const int row = tt * 16 + (lane & 7) + ((lane >> 4) << 3);
+      const uint32_t b0 = smem_u32(V0) + row * 128, b1 = smem_u32(V1) + row * 128;
+#pragma unroll
+      for (int mt = 0; mt < 8; ++mt) {
+        const int c16 = 2 * mt + ((lane >> 3) & 1);
+        const uint32_t addr = (c16 >> 3 ? b1 : b0) + (((c16 & 7) ^ (row & 7)) << 4);
+        uint32_t a0, a1, a2, a3;
+        ldsm_x4_t(addr, a0, a1, a2, a3);
+        mma_bf16(o[mt], a0, a1, a2, a3, bp[j][0], bp[j][1]);
+        mma_bf16(o[mt], a0, a1, a2, a3, bl[j][0], bl[j][1]);
+      }
+    }
+  }
+
+  // 8. Sum the partials across the group (in the K area: every warp has
+  //    passed the softmax exchange, so no one reads K any more) and agree on
+  //    the evicted row; each output tile is then finished by one warp and
+  //    stored straight from its fragments.
+  if (U > 1) {
+    float4 *XO = reinterpret_cast<float4 *>(K0);
+#pragma unroll
+    for (int mt = 0; mt < 8; ++mt)
+      XO[(w * 8 + mt) * 32 + lane] = make_float4(o[mt][0], o[mt][1], o[mt][2], o[mt][3]);
+    uint32_t *XW = reinterpret_cast<uint32_t *>(XS);
+    if (lane == 0) {
+      XW[w * kXsWords + 16] = (uint32_t)best;
+      XW[w * kXsWords + 17] = (uint32_t)(best >> 32);
+      XW[w * kXsWords + 18] = (uint32_t)bi;
+    }
+    group_bar(bar_id, GT);
+#pragma unroll
+    for (int mt = 0; mt < 8; ++mt) {
+      if (mt % U == w) {
+        float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int v = 0; v < U; ++v) {
+          const float4 a = XO[(v * 8 + mt) * 32 + lane];
+          sum.x += a.x;
+          sum.y += a.y;
+          sum.z += a.z;
+          sum.w += a.w;
+        }
+        o[mt][0] = sum.x;
+        o[mt][1] = sum.y;
+        o[mt][2] = sum.z;
+        o[mt][3] = sum.w;
+      }
+    }
+#pragma unroll
+    for (int v = 0; v < U; ++v) {
+      const unsigned long long kb =
+          ((unsigned long long)XW[v * kXsWords + 17] << 32) | XW[v * kXsWords + 16];
+      if (kb < best) {
+        best = kb;
+        bi = (int)XW[v * kXsWords + 18];
+      }
+    }
+  }
+  {
+    constexpr int osz = kOutBf16 ? 2 : 4;
+    unsigned char *gout = reinterpret_cast<unsigned char *>(p.out) +
+                          x.krow * G * 128 * osz;
+#pragma unroll
+    for (int mt = 0; mt < 8; ++mt) {
+      if (mt % U != w) continue;
+      if (kOutBf16) {
+        // (head dim, head) 8x8 blocks -> (head, head dim) pairs per lane.
+        const uint32_t lo = movm_t(pack_bf16(o[mt][0], o[mt][1]));
+        const uint32_t hi = movm_t(pack_bf16(o[mt][2], o[mt][3]));
+        const int g = lane >> 2, dd = 16 * mt + 2 * (lane & 3);
+        if (g < G) {
+          *reinterpret_cast<uint32_t *>(gout + ((size_t)g * 128 + dd) * 2) = lo;
+          *reinterpret_cast<uint32_t *>(gout + ((size_t)g * 128 + dd + 8) * 2) = hi;
+        }
+      } else {
+        float *of = reinterpret_cast<float *>(gout);
+        const int d0 = 16 * mt + r0;
+        if (g0) {
+          of[c2 * 128 + d0] = o[mt][0];
+          of[c2 * 128 + d0 + 8] = o[mt][2];
+        }
+        if (g1) {
+          of[(c2 + 1) * 128 + d0] = o[mt][1];
+          of[(c2 + 1) * 128 + d0 + 8] = o[mt][3];
+        }
+      }
+    }
+  }
+
+  // 9. The warp owning the new row writes it into the freed slot (or the
+  //    first free slot when nothing is evicted), with its position, score,
+  //    the live length and the next position.
+  if (own_new) {
+    const int victim = (p.evict && n > p.budget + p.window) ? bi : -1;
+    const int slot = victim < 0 ? m : (victim < m ? victim : -1);
+    if (slot >= 0) {
+      const int chunk = lane & 15;
+      __nv_bfloat16 *dst =
+          reinterpret_cast<__nv_bfloat16 *>(lane < 16 ? p.c.K : p.c.V) +
+          (x.ug * (size_t)p.c.cap + slot) * 128;
+      const unsigned char *src = lane < 16 ? KN : VN;
+      reinterpret_cast<int4 *>(dst)[chunk] =
+          *reinterpret_cast<const int4 *>(src + chunk * 16);
+      if (lane == 0) {
+        p.c.pos[x.ug * p.c.sstride + slot] = t;
+        gsc[slot] = new_score;
+      }
+    }
+    if (lane == 0) {
+      p.c.state[4 * x.ug] = victim < 0 ? m + 1 : m;
+      p.c.state[4 * x.ug + 1] = t + 1;
+    }
+  }
+}
