@@ -55,6 +55,12 @@ def parse():
                    help="shortest prior context (profiling uses a small case)")
     p.add_argument("--prior-max", type=int, default=inputs.PRIOR_LEN_RANGE[1])
     p.add_argument("--e2e-steps", type=int, default=1000)
+    p.add_argument("--fused-groups", type=int, default=0,
+                   help="units computed at once per SM by the fused kernel "
+                        "(0: the library's choice)")
+    p.add_argument("--fused-group-warps", type=int, default=0,
+                   help="warps sharing one unit in the fused kernel "
+                        "(0: the library's choice)")
     return p.parse_args()
 
 
@@ -206,6 +212,9 @@ def run_kvr(args, rank, world, local_rank):
     cap = int(lens.max()) + 1
     cache = kvr.Cache(S, L, H, G, d, cap, kv_dtype="bf16", out_dtype="bf16",
                       device=dev)
+    if args.fused_groups or args.fused_group_warps:
+        kvr.kvr_cache_set_fused_tuning(cache.handle, args.fused_groups,
+                                       args.fused_group_warps)
     gen = torch.Generator(device=dev)
     gen.manual_seed(1_000_003 * (args.seed + 1) + rank)
     for s in range(S):

@@ -9,13 +9,13 @@
  *      (grouped-query attention; softmax scale 1/sqrt(d) by default),
  *   3. adds to every live row's importance score s_i ("accumulated attention",
  *      Sec. 2.1) the mean over the G query heads of that row's probability,
- *   4. once the live length exceeds B' = B + W (App. C: eviction "fires every
- *      step once l > B'"), keeps the W most recent rows (the protected window
- *      of Sec. 4.1 / App. Impl.) plus the B best-scored others (TopB of Eq. 1;
+ *   4. once the live length exceeds B' = B + W (App. C: eviction then runs on
+ *      every step), keeps the W most recent rows (the protected window of
+ *      Sec. 4.1 / App. Impl.) plus the B best-scored others (TopB of Eq. 1;
  *      equal scores keep the lower position) and compacts K/V in place.
- * Candidates (Sec. 2.2 Eq. 2, App. Impl. "Best-of-(N+N)") fork from one cache
- * state, share its rows as a read-only prefix, decode a step each, and one of
- * them is committed back (Algorithm 1, "retain the selected base fork").
+ * Candidates (Sec. 2.2, Eq. 2; App. Impl., best-of-(N+N)) fork from one cache
+ * state, decode a step each, and the chosen one becomes the persistent state
+ * (Algorithm 1).
  *
  * Conventions for every call below:
  *  - A "unit" is one (sequence, layer, KV head).  Query head j of a layer
@@ -133,6 +133,14 @@ kvr_status kvr_decode_step(kvr_cache *cache, int layer_begin, int layer_end,
  * generic kernels for every shape.  Both compute the same step; this exists
  * for testing and measurement.  enable: 0 or 1. */
 kvr_status kvr_cache_set_fused(kvr_cache *cache, int enable);
+
+/* Tuning of the fused kernel.  groups: how many units each SM computes at
+ * once (1..4; 0 = the library's choice, the most the shared-memory ring and
+ * thread budget allow).  group_warps: warps sharing one unit, either one
+ * 16-row tile per warp or two (other values, and 0, select the library's
+ * choice).  Results do not depend on either. */
+kvr_status kvr_cache_set_fused_tuning(kvr_cache *cache, int groups,
+                                      int group_warps);
 
 /* ---- the same step for callers that cannot allocate -------------------- */
 

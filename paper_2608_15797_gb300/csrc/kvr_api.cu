@@ -97,6 +97,8 @@ struct kvr_cache {
   size_t bytes;
   uint64_t launches = 0;          // kernels launched through this handle
   bool fused = true;              // use the fused kernel where it applies
+  int fused_groups = 0;           // units computed at once per SM (0: auto)
+  int fused_group_warps = 0;      // warps per unit (0: auto)
   int sm_count = 0;               // of the device, queried on first use
   int smem_optin = 0;
   std::map<int, std::pair<CUtensorMap, CUtensorMap>> tmaps;  // by box rows
@@ -249,13 +251,15 @@ bool try_fused(kvr_cache *c, const StepArgs &a, bool evict, int budget,
   }
   const int R = kvr::round_up16(a.max_rows);
   const int Rb = std::max(8, (a.max_rows - 1 + 7) / 8 * 8);
-  const int U = kvr::fused_group_warps(R);
+  const int U = kvr::fused_group_warps(R, c->fused_group_warps);
   const int stage = kvr::fused_stage_bytes(R);
   const int avail = c->smem_optin - 1024 /*alignment*/ - 512 /*static*/;
   const int n_stages = std::min(8, avail / stage);
   if (U < 1 || n_stages < 2) return false;
-  const int n_groups = std::min(
-      {4, n_stages - 1, (kvr::fused_max_threads() / 32 - 1) / U});
+  // Keep two stages loading while the others are computed (measured best).
+  int n_groups = std::min({4, std::max(1, n_stages - 2),
+                           (kvr::fused_max_threads() / 32 - 1) / U});
+  if (c->fused_groups > 0) n_groups = std::min(n_groups, c->fused_groups);
   if (n_groups < 1) return false;
   auto it = c->tmaps.find(Rb);
   if (it == c->tmaps.end()) {
@@ -277,6 +281,7 @@ bool try_fused(kvr_cache *c, const StepArgs &a, bool evict, int budget,
   p.Rb = Rb;
   p.n_stages = n_stages;
   p.n_groups = n_groups;
+  p.group_warps = U;
   p.budget = budget;
   p.window = window;
   p.evict = evict ? 1 : 0;
@@ -392,6 +397,17 @@ kvr_status kvr_decode_attend_score(kvr_cache *c, int lb, int le, const void *q,
 kvr_status kvr_cache_set_fused(kvr_cache *c, int enable) {
   if (!c) return fail(KVR_EINVAL, "null cache");
   c->fused = enable != 0;
+  return KVR_OK;
+}
+
+kvr_status kvr_cache_set_fused_tuning(kvr_cache *c, int groups,
+                                      int group_warps) {
+  if (!c) return fail(KVR_EINVAL, "null cache");
+  if (groups < 0 || groups > 4 || group_warps < 0 || group_warps > 8)
+    return fail(KVR_EINVAL, "tuning (%d, %d) outside [0, 4] x [0, 8]", groups,
+                group_warps);
+  c->fused_groups = groups;
+  c->fused_group_warps = group_warps;
   return KVR_OK;
 }
 

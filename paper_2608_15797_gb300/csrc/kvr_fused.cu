@@ -148,7 +148,7 @@ __device__ __forceinline__ void group_bar(int id, int threads) {
 
 // Byte offsets inside one stage of R staged rows.
 struct StageLayout {
-  uint32_t k0, k1, v0, v1, q, kn, vn, sc, ps, st, xs, bytes;
+  uint32_t k0, k1, v0, v1, q, kn, vn, sc, ps, st, xs, info, bytes;
   __host__ __device__ explicit StageLayout(int R) {
     k0 = 0;
     k1 = k0 + R * 128;
@@ -161,7 +161,8 @@ struct StageLayout {
     ps = sc + 4 * R;
     st = ps + 4 * R;
     xs = st + 16;  // group exchange: kXsWords words per warp
-    bytes = ((xs + 4 * kXsWords * kMaxGroupWarps) + 1023) / 1024 * 1024;
+    info = xs + 4 * kXsWords * kMaxGroupWarps;  // cache unit, input row
+    bytes = ((info + 16) + 1023) / 1024 * 1024;
   }
 };
 
@@ -192,6 +193,10 @@ __device__ void issue_unit(const FusedParams &p, const CUtensorMap *tmK,
   const uint32_t s0 = smem_u32(stage);
   const uint32_t tx = 4u * p.Rb * 128u + (uint32_t)G * 256u + 512u +
                       8u * p.Rb + 16u;
+  // The unit's indices for the consumers (released by the arrive below).
+  uint32_t *info = reinterpret_cast<uint32_t *>(stage + L.info);
+  info[0] = (uint32_t)x.ug;
+  info[1] = (uint32_t)x.krow;
   mbar_expect_tx(bar, tx);
   const int row0 = (int)(x.ug * (size_t)p.c.cap);
   tma_load_2d(s0 + L.k0, tmK, 0, row0, bar);
@@ -287,9 +292,7 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
       group_bar(bar_id, 32 * U);
       if (!s_ok[grp]) break;
       mbar_try_wait(smem_u32(&full_bar[s]), ph);  // acquire for this thread
-      process_unit<T, U, kOutBf16>(p, smem + s * L.bytes,
-                                   (int)blockIdx.x + k * (int)gridDim.x, w,
-                                   lane, bar_id);
+      process_unit<T, U, kOutBf16>(p, smem + s * L.bytes, w, lane, bar_id);
       // Each warp releases the stage once its own reads and writes of it
       // are done (the async-proxy fence orders them before the refill).
       fence_proxy_async();
@@ -330,16 +333,19 @@ template <bool kOutBf16>
 cudaError_t launch_t(const CUtensorMap &tmK, const CUtensorMap &tmV,
                      const FusedParams &p, int grid, int smem_bytes,
                      cudaStream_t st) {
-  switch (p.R / 16) {
-    case 1: return launch_tu<1, 1, kOutBf16>(tmK, tmV, p, grid, smem_bytes, st);
-    case 2: return launch_tu<2, 2, kOutBf16>(tmK, tmV, p, grid, smem_bytes, st);
-    case 3: return launch_tu<3, 3, kOutBf16>(tmK, tmV, p, grid, smem_bytes, st);
-    case 4: return launch_tu<4, 4, kOutBf16>(tmK, tmV, p, grid, smem_bytes, st);
-    case 5: return launch_tu<5, 5, kOutBf16>(tmK, tmV, p, grid, smem_bytes, st);
-    case 6: return launch_tu<6, 3, kOutBf16>(tmK, tmV, p, grid, smem_bytes, st);
-    case 7: return launch_tu<7, 4, kOutBf16>(tmK, tmV, p, grid, smem_bytes, st);
-    case 8: return launch_tu<8, 4, kOutBf16>(tmK, tmV, p, grid, smem_bytes, st);
-  }
+  // (tiles, warps per unit): one tile per warp, or two.
+#define KVR_TU(T_, U_)                                                   \
+  if (p.R == 16 * T_ && p.group_warps == U_)                             \
+    return launch_tu<T_, U_, kOutBf16>(tmK, tmV, p, grid, smem_bytes, st);
+  KVR_TU(1, 1)
+  KVR_TU(2, 1) KVR_TU(2, 2)
+  KVR_TU(3, 2) KVR_TU(3, 3)
+  KVR_TU(4, 2) KVR_TU(4, 4)
+  KVR_TU(5, 3) KVR_TU(5, 5)
+  KVR_TU(6, 3) KVR_TU(6, 6)
+  KVR_TU(7, 4) KVR_TU(7, 7)
+  KVR_TU(8, 4) KVR_TU(8, 8)
+#undef KVR_TU
   return cudaErrorInvalidValue;
 }
 
@@ -347,9 +353,11 @@ cudaError_t launch_t(const CUtensorMap &tmK, const CUtensorMap &tmV,
 
 int fused_stage_bytes(int R) { return (int)StageLayout(R).bytes; }
 
-int fused_group_warps(int R) {
-  static const int u[9] = {0, 1, 2, 3, 4, 5, 3, 4, 4};
-  return (R % 16 == 0 && R >= 16 && R <= 128) ? u[R / 16] : 0;
+int fused_group_warps(int R, int requested) {
+  if (R % 16 != 0 || R < 16 || R > 128) return 0;
+  const int T = R / 16, one = T, two = (T + 1) / 2;
+  if (requested == one || requested == two) return requested;
+  return T <= 3 ? one : two;  // measured: two tiles per warp from T = 4 on
 }
 
 int fused_max_threads() { return kMaxThreads; }
@@ -357,9 +365,9 @@ int fused_max_threads() { return kMaxThreads; }
 cudaError_t launch_fused_step(const CUtensorMap &tmK, const CUtensorMap &tmV,
                               const FusedParams &p, int grid, int smem_bytes,
                               cudaStream_t st) {
-  if (fused_group_warps(p.R) == 0 || p.n_groups < 1 ||
-      p.n_groups > kMaxGroups || p.n_stages > kMaxStages ||
-      32 * (p.n_groups * fused_group_warps(p.R) + 1) > kMaxThreads)
+  if (fused_group_warps(p.R, p.group_warps) != p.group_warps ||
+      p.n_groups < 1 || p.n_groups > kMaxGroups || p.n_stages > kMaxStages ||
+      32 * (p.n_groups * p.group_warps + 1) > kMaxThreads)
     return cudaErrorInvalidValue;
   return p.c.out_bf16 ? launch_t<true>(tmK, tmV, p, grid, smem_bytes, st)
                       : launch_t<false>(tmK, tmV, p, grid, smem_bytes, st);

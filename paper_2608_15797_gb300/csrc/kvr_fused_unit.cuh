@@ -5,21 +5,32 @@
 // a shared-memory stage.  The unit has T = R / 16 row tiles; warp w of the
 // group owns tiles w, w + U, ... and everything about their rows: inserting
 // the new row if it falls in an owned tile, the logits, probabilities,
-// accumulated-attention scores, eviction candidates and the PV partial sums.
-// The group meets at two named barriers per unit: one to merge the softmax
-// statistics and one to sum the PV partials and agree on the evicted row.
+// accumulated-attention scores and eviction candidates.  The group meets at
+// two named barriers per unit: one to merge the softmax statistics, one to
+// share the probability tiles and agree on the evicted row.  PV is then
+// split by output columns (head-dim tiles), so no partial sums cross warps.
 //
-// Exchange words per warp (XS): [0,8) column max, [8,16) column sum under
-// that max, [16,18) argmin key, 18 argmin row.
+// Exchange record per warp (XS, five 16-byte slots): slot cp = 0..3 holds
+// (max, max, sum, sum) of columns 2cp and 2cp + 1; slot 4 holds the warp's
+// argmin (key low, key high, row, 0).
+
+struct UnitRows {
+  size_t ug;    // cache unit
+  size_t krow;  // row of this unit in the call's [S][nl][H] inputs
+};
 
 template <int T, int U, bool kOutBf16>
 __device__ void process_unit(const FusedParams &p, unsigned char *stage,
-                             int idx, int w, int lane, int bar_id) {
+                             int w, int lane, int bar_id) {
   constexpr int TW = (T + U - 1) / U;  // tiles per warp (at most)
   constexpr int R = 16 * T;
-  constexpr int GT = 32 * U;           // threads of the group
   const StageLayout L(R);
-  const UnitIdx x = unit_idx(p, idx);
+  UnitRows x;
+  {
+    const uint32_t *info = reinterpret_cast<const uint32_t *>(stage + L.info);
+    x.ug = info[0];
+    x.krow = info[1];
+  }
   const int G = p.c.G;
   unsigned char *K0 = stage + L.k0, *K1 = stage + L.k1;
   unsigned char *V0 = stage + L.v0, *V1 = stage + L.v1;
@@ -135,28 +146,24 @@ __device__ void process_unit(const FusedParams &p, unsigned char *stage,
     z1 += __shfl_xor_sync(0xffffffffu, z1, o);
   }
   float f0 = 1.f / z0, f1 = 1.f / z1;  // this warp's rescale factors
+  float4 *XS4 = reinterpret_cast<float4 *>(XS);
   if (U > 1) {
-    if (lane < 4) {
-      XS[w * kXsWords + c2] = ref0;
-      XS[w * kXsWords + c2 + 1] = ref1;
-      XS[w * kXsWords + 8 + c2] = z0;
-      XS[w * kXsWords + 8 + c2 + 1] = z1;
-    }
-    group_bar(bar_id, GT);
-    // Warps with no live row (z = 0) take no part in the merge.
+    if (lane < 4) XS4[w * 5 + (lane & 3)] = make_float4(ref0, ref1, z0, z1);
+    group_bar(bar_id, 32 * U);
+    // Warps with no live row (sum 0) take no part in the merge.
+    float4 r[U];
     float M0 = -INFINITY, M1 = -INFINITY;
 #pragma unroll
     for (int v = 0; v < U; ++v) {
-      if (XS[v * kXsWords + 8 + c2] > 0.f) M0 = fmaxf(M0, XS[v * kXsWords + c2]);
-      if (XS[v * kXsWords + 8 + c2 + 1] > 0.f)
-        M1 = fmaxf(M1, XS[v * kXsWords + c2 + 1]);
+      r[v] = XS4[v * 5 + (lane & 3)];
+      if (r[v].z > 0.f) M0 = fmaxf(M0, r[v].x);
+      if (r[v].w > 0.f) M1 = fmaxf(M1, r[v].y);
     }
     float Z0 = 0.f, Z1 = 0.f;
 #pragma unroll
     for (int v = 0; v < U; ++v) {
-      const float za = XS[v * kXsWords + 8 + c2], zb = XS[v * kXsWords + 8 + c2 + 1];
-      if (za > 0.f) Z0 += za * exp2f(XS[v * kXsWords + c2] - M0);
-      if (zb > 0.f) Z1 += zb * exp2f(XS[v * kXsWords + c2 + 1] - M1);
+      if (r[v].z > 0.f) Z0 += r[v].z * exp2f(r[v].x - M0);
+      if (r[v].w > 0.f) Z1 += r[v].w * exp2f(r[v].y - M1);
     }
     f0 = z0 > 0.f ? exp2f(ref0 - M0) / Z0 : 0.f;
     f1 = z1 > 0.f ? exp2f(ref1 - M1) / Z1 : 0.f;
@@ -212,22 +219,34 @@ __device__ void process_unit(const FusedParams &p, unsigned char *stage,
   }
   // The lane that scored the new row passes its score to the whole warp.
   new_score = __shfl_sync(0xffffffffu, new_score, ((m & 15) & 7) * 4);
-#pragma unroll
-  for (int o2 = 16; o2 > 0; o2 >>= 1) {
-    const unsigned long long ob = __shfl_xor_sync(0xffffffffu, best, o2);
-    const int oi = __shfl_xor_sync(0xffffffffu, bi, o2);
-    if (ob < best) {
-      best = ob;
-      bi = oi;
+  {
+    // Warp argmin of the key: lowest score bits, then highest position
+    // (keys are distinct because positions are).
+    const uint32_t sb = bi < 0 ? 0xFFFFFFFFu : (uint32_t)(best >> 32);
+    const int pb = bi < 0 ? -1 : (int)(0xFFFFFFFFu - (uint32_t)best);
+    const uint32_t smin = __reduce_min_sync(0xffffffffu, sb);
+    const int pmax = __reduce_max_sync(0xffffffffu, sb == smin ? pb : -1);
+    const uint32_t who = __ballot_sync(0xffffffffu, bi >= 0 && sb == smin && pb == pmax);
+    if (who) {
+      bi = __shfl_sync(0xffffffffu, bi, __ffs(who) - 1);
+      best = ((unsigned long long)smin << 32) |
+             (unsigned long long)(0xFFFFFFFFu - (uint32_t)pmax);
+    } else {
+      bi = -1;
+      best = ~0ull;
     }
   }
 
   // 6. P as the PV B operand, split into two bf16 terms (hi + lo carries
   //    ~16 mantissa bits; a single bf16 P would cost up to 2^-9 relative
-  //    per probability), each 8x8 block transposed in registers.
-  uint32_t bp[TW][2], bl[TW][2];
+  //    per probability), each 8x8 block transposed in registers, and
+  //    published to the group in the K area (no warp reads K any more once
+  //    everyone has passed the softmax exchange), together with the warp's
+  //    eviction candidate.
+  uint4 *PX = reinterpret_cast<uint4 *>(K0);  // [tile][lane]
 #pragma unroll
   for (int j = 0; j < TW; ++j) {
+    const int tt = w + j * U;
     const uint32_t h0 = pack_bf16(acc[j][0], acc[j][1]);
     const uint32_t h1 = pack_bf16(acc[j][2], acc[j][3]);
     const __nv_bfloat162 hb0 = *reinterpret_cast<const __nv_bfloat162 *>(&h0);
@@ -236,90 +255,67 @@ __device__ void process_unit(const FusedParams &p, unsigned char *stage,
                                   acc[j][1] - __high2float(hb0));
     const uint32_t l1 = pack_bf16(acc[j][2] - __low2float(hb1),
                                   acc[j][3] - __high2float(hb1));
-    bp[j][0] = movm_t(h0);
-    bp[j][1] = movm_t(h1);
-    bl[j][0] = movm_t(l0);
-    bl[j][1] = movm_t(l1);
+    const uint4 frag = make_uint4(movm_t(h0), movm_t(h1), movm_t(l0), movm_t(l1));
+    if (tt < T) PX[tt * 32 + lane] = frag;
+  }
+  if (U > 1) {
+    uint4 *XW = reinterpret_cast<uint4 *>(XS);
+    if (lane == 0)
+      XW[w * 5 + 4] = make_uint4((uint32_t)best, (uint32_t)(best >> 32),
+                                 (uint32_t)bi, 0u);
+    group_bar(bar_id, 32 * U);
+#pragma unroll
+    for (int v = 0; v < U; ++v) {
+      const uint4 a = XW[v * 5 + 4];
+      const unsigned long long kb = ((unsigned long long)a.y << 32) | a.x;
+      if (kb < best) {
+        best = kb;
+        bi = (int)a.z;
+      }
+    }
+  } else {
+    __syncwarp();
   }
 
-  // 7. Partial out^T = V^T P^T over the owned tiles: M = head dim (8 tiles
-  //    of 16), K = rows, N = query heads.
-  float o[8][4];
+  // 7. out^T = V^T P^T for the output tiles this warp owns (head-dim tiles
+  //    mt = w, w + U, ...) over every row tile: M = head dim, K = rows,
+  //    N = query heads.  No partial sums cross warps.
+  constexpr int MW = (8 + U - 1) / U;  // output tiles per warp (at most)
+  float o[MW][4];
 #pragma unroll
-  for (int mt = 0; mt < 8; ++mt) o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.f;
+  for (int i = 0; i < MW; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
 #pragma unroll
-  for (int j = 0; j < TW; ++j) {
-    const int tt = w + j * U;
-    if (tt < T) {
-      const int row = tt * 16 + (lane & 7) + ((lane >> 4) << 3);
-      const uint32_t b0 = smem_u32(V0) + row * 128, b1 = smem_u32(V1) + row * 128;
+  for (int tt = 0; tt < T; ++tt) {
+    const uint4 pf = PX[tt * 32 + lane];
+    const int row = tt * 16 + (lane & 7) + ((lane >> 4) << 3);
+    const uint32_t b0 = smem_u32(V0) + row * 128, b1 = smem_u32(V1) + row * 128;
 #pragma unroll
-      for (int mt = 0; mt < 8; ++mt) {
+    for (int i = 0; i < MW; ++i) {
+      const int mt = w + i * U;
+      if (mt < 8) {
         const int c16 = 2 * mt + ((lane >> 3) & 1);
         const uint32_t addr = (c16 >> 3 ? b1 : b0) + (((c16 & 7) ^ (row & 7)) << 4);
         uint32_t a0, a1, a2, a3;
         ldsm_x4_t(addr, a0, a1, a2, a3);
-        mma_bf16(o[mt], a0, a1, a2, a3, bp[j][0], bp[j][1]);
-        mma_bf16(o[mt], a0, a1, a2, a3, bl[j][0], bl[j][1]);
+        mma_bf16(o[i], a0, a1, a2, a3, pf.x, pf.y);
+        mma_bf16(o[i], a0, a1, a2, a3, pf.z, pf.w);
       }
     }
   }
 
-  // 8. Sum the partials across the group (in the K area: every warp has
-  //    passed the softmax exchange, so no one reads K any more) and agree on
-  //    the evicted row; each output tile is then finished by one warp and
-  //    stored straight from its fragments.
-  if (U > 1) {
-    float4 *XO = reinterpret_cast<float4 *>(K0);
-#pragma unroll
-    for (int mt = 0; mt < 8; ++mt)
-      XO[(w * 8 + mt) * 32 + lane] = make_float4(o[mt][0], o[mt][1], o[mt][2], o[mt][3]);
-    uint32_t *XW = reinterpret_cast<uint32_t *>(XS);
-    if (lane == 0) {
-      XW[w * kXsWords + 16] = (uint32_t)best;
-      XW[w * kXsWords + 17] = (uint32_t)(best >> 32);
-      XW[w * kXsWords + 18] = (uint32_t)bi;
-    }
-    group_bar(bar_id, GT);
-#pragma unroll
-    for (int mt = 0; mt < 8; ++mt) {
-      if (mt % U == w) {
-        float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-        for (int v = 0; v < U; ++v) {
-          const float4 a = XO[(v * 8 + mt) * 32 + lane];
-          sum.x += a.x;
-          sum.y += a.y;
-          sum.z += a.z;
-          sum.w += a.w;
-        }
-        o[mt][0] = sum.x;
-        o[mt][1] = sum.y;
-        o[mt][2] = sum.z;
-        o[mt][3] = sum.w;
-      }
-    }
-#pragma unroll
-    for (int v = 0; v < U; ++v) {
-      const unsigned long long kb =
-          ((unsigned long long)XW[v * kXsWords + 17] << 32) | XW[v * kXsWords + 16];
-      if (kb < best) {
-        best = kb;
-        bi = (int)XW[v * kXsWords + 18];
-      }
-    }
-  }
+  // 8. Store the owned output tiles straight from their fragments.
   {
     constexpr int osz = kOutBf16 ? 2 : 4;
     unsigned char *gout = reinterpret_cast<unsigned char *>(p.out) +
                           x.krow * G * 128 * osz;
 #pragma unroll
-    for (int mt = 0; mt < 8; ++mt) {
-      if (mt % U != w) continue;
+    for (int i = 0; i < MW; ++i) {
+      const int mt = w + i * U;
+      if (mt >= 8) continue;
       if (kOutBf16) {
         // (head dim, head) 8x8 blocks -> (head, head dim) pairs per lane.
-        const uint32_t lo = movm_t(pack_bf16(o[mt][0], o[mt][1]));
-        const uint32_t hi = movm_t(pack_bf16(o[mt][2], o[mt][3]));
+        const uint32_t lo = movm_t(pack_bf16(o[i][0], o[i][1]));
+        const uint32_t hi = movm_t(pack_bf16(o[i][2], o[i][3]));
         const int g = lane >> 2, dd = 16 * mt + 2 * (lane & 3);
         if (g < G) {
           *reinterpret_cast<uint32_t *>(gout + ((size_t)g * 128 + dd) * 2) = lo;
@@ -329,12 +325,12 @@ __device__ void process_unit(const FusedParams &p, unsigned char *stage,
         float *of = reinterpret_cast<float *>(gout);
         const int d0 = 16 * mt + r0;
         if (g0) {
-          of[c2 * 128 + d0] = o[mt][0];
-          of[c2 * 128 + d0 + 8] = o[mt][2];
+          of[c2 * 128 + d0] = o[i][0];
+          of[c2 * 128 + d0 + 8] = o[i][2];
         }
         if (g1) {
-          of[(c2 + 1) * 128 + d0] = o[mt][1];
-          of[(c2 + 1) * 128 + d0 + 8] = o[mt][3];
+          of[(c2 + 1) * 128 + d0] = o[i][1];
+          of[(c2 + 1) * 128 + d0 + 8] = o[i][3];
         }
       }
     }

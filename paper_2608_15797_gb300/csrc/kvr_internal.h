@@ -76,11 +76,14 @@ struct FusedParams {
   int R;                       // staged rows per unit (multiple of 16, <= 128)
   int Rb;                      // rows copied from a slab (multiple of 8, <= R)
   int n_stages, n_groups;      // ring depth; units computed at once
+  int group_warps;             // warps sharing one unit
   int budget, window, evict;
   float scale_log2e, inv_g;
 };
 int fused_stage_bytes(int R);
-int fused_group_warps(int R);  // warps that share one unit of R staged rows
+// Warps that share one unit of R staged rows: `requested` if it is one of
+// the supported choices (one or two row tiles per warp), else the default.
+int fused_group_warps(int R, int requested);
 int fused_max_threads();
 cudaError_t launch_fused_step(const CUtensorMap &tmK, const CUtensorMap &tmV,
                               const FusedParams &p, int grid, int smem_bytes,

@@ -66,6 +66,7 @@ _SIGS = {
     "kvr_cache_lengths": (_S, [_P, _P]),
     "kvr_cache_launch_count": (_S, [_P, _P]),
     "kvr_cache_set_fused": (_S, [_P, _I]),
+    "kvr_cache_set_fused_tuning": (_S, [_P, _I, _I]),
     "kvr_sync_status": (_S, [_P, _P]),
     "kvr_last_error": (ctypes.c_char_p, []),
 }
@@ -184,6 +185,11 @@ def kvr_cache_launch_count(h) -> int:
 
 def kvr_cache_set_fused(h, enable: bool):
     _check(lib.kvr_cache_set_fused(h, 1 if enable else 0), "kvr_cache_set_fused")
+
+
+def kvr_cache_set_fused_tuning(h, groups: int, group_warps: int = 0):
+    _check(lib.kvr_cache_set_fused_tuning(h, groups, group_warps),
+           "kvr_cache_set_fused_tuning")
 
 
 def kvr_sync_status(h, stream=None):
