@@ -281,9 +281,11 @@ __device__ void process_unit(const FusedParams &p, unsigned char *stage,
   //    mt = w, w + U, ...) over every row tile: M = head dim, K = rows,
   //    N = query heads.  No partial sums cross warps.
   constexpr int MW = (8 + U - 1) / U;  // output tiles per warp (at most)
-  float o[MW][4];
+  float o[MW][4], ol[MW][4];  // hi and lo terms on separate chains
 #pragma unroll
-  for (int i = 0; i < MW; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
+  for (int i = 0; i < MW; ++i)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) o[i][e] = ol[i][e] = 0.f;
 #pragma unroll
   for (int tt = 0; tt < T; ++tt) {
     const uint4 pf = PX[tt * 32 + lane];
@@ -298,10 +300,14 @@ __device__ void process_unit(const FusedParams &p, unsigned char *stage,
         uint32_t a0, a1, a2, a3;
         ldsm_x4_t(addr, a0, a1, a2, a3);
         mma_bf16(o[i], a0, a1, a2, a3, pf.x, pf.y);
-        mma_bf16(o[i], a0, a1, a2, a3, pf.z, pf.w);
+        mma_bf16(ol[i], a0, a1, a2, a3, pf.z, pf.w);
       }
     }
   }
+#pragma unroll
+  for (int i = 0; i < MW; ++i)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) o[i][e] += ol[i][e];
 
   // 8. Store the owned output tiles straight from their fragments.
   {
