@@ -127,6 +127,71 @@ kvr_status kvr_decode_step(kvr_cache *cache, int layer_begin, int layer_end,
                            const void *q, const void *k_new, const void *v_new,
                            void *out, int budget, int window, void *stream);
 
+/* ---- candidates: stepwise best-of-N over one shared cache state -------- */
+
+/* Sec. 2.2 (Eq. 2) and App. Impl. (best-of-(N+N)): each reasoning step draws
+ * N candidates from the same committed (evicted) cache state; the selected
+ * one becomes the persistent state (Algorithm 1).  The paper forks by
+ * copying the live rows; here the candidates share the parent's live rows
+ * read-only as a common prefix (the batched kernel reads every prefix row
+ * once for all N x G query rows) and keep only what differs: a private copy
+ * of the prefix scores and a private tail of appended rows.  Eviction is
+ * deferred to the end of the step (kvr_fork_commit), which cuts the chosen
+ * candidate to B + W exactly as kvr_evict_compact would cut a private copy
+ * that had decoded the same rows without eviction. */
+
+/* Device bytes a fork of `parent` into n_cand candidates with tail_cap rows
+ * per unit needs (0 for invalid arguments): per candidate, the prefix score
+ * copy [S][L][H][capacity], the tail K and V [S][L][H][tail_cap][d], tail
+ * scores, positions and lengths. */
+size_t kvr_fork_required_bytes(const kvr_cache *parent, int n_cand,
+                               int tail_cap);
+
+/* Fork the parent (all sequences) into n_cand >= 1 candidates over dev_buf
+ * (caller-owned, >= kvr_fork_required_bytes, 256-byte aligned).  The parent
+ * must not be modified by any other call while the fork is alive; its rows
+ * are the candidates' shared prefix.  Copies the parent's scores into every
+ * candidate (enqueued on stream). */
+kvr_status kvr_fork_candidates(kvr_cache *parent, int n_cand, int tail_cap,
+                               void *dev_buf, size_t bytes, void *stream,
+                               kvr_fork **out);
+
+/* One decode step of every candidate over layers [layer_begin, layer_end):
+ * candidate c appends its row to its tail, attends over prefix + its tail,
+ * and adds the mean over the G heads of each row's probability to its own
+ * scores.  No eviction.
+ *   q     dev [N][S][nl][H*G][d],  k_new, v_new dev [N][S][nl][H][d]
+ *   out   dev [N][S][nl][H*G][d] (the parent's out_dtype)
+ * KVR_ECAPACITY when a tail is full. */
+kvr_status kvr_fork_decode_attend_score(kvr_fork *fork, int layer_begin,
+                                        int layer_end, const void *q,
+                                        const void *k_new, const void *v_new,
+                                        void *out, void *stream);
+
+/* Commit: for every sequence s, candidate chosen[s] (host array [S]) is cut
+ * to budget + window rows (window = the W newest positions; TopB of the rest
+ * on the candidate's scores, ties to the lower position) and becomes the
+ * parent's state: kept prefix rows stay, freed parent slots receive the kept
+ * tail rows, and the parent's scores become the candidate's.  Every layer's
+ * tails must have the same length.  The fork is spent afterwards (further
+ * calls return KVR_ESTATE). */
+kvr_status kvr_fork_commit(kvr_fork *fork, const int32_t *chosen, int budget,
+                           int window, void *stream);
+
+/* Synchronising: candidate cand's view of sequence seq.  host_prefix_score
+ * [L][H][capacity] fp32 (slot order of the parent); host_tail_k/v
+ * [L][H][tail_cap][d] (kv_dtype); host_tail_score [L][H][tail_cap] fp32;
+ * host_tail_pos [L][H][tail_cap] int32; host_tail_len [L][H] int32.  Any
+ * pointer may be NULL. */
+kvr_status kvr_fork_export(const kvr_fork *fork, int cand, int seq,
+                           float *host_prefix_score, void *host_tail_k,
+                           void *host_tail_v, float *host_tail_score,
+                           int32_t *host_tail_pos, int32_t *host_tail_len,
+                           void *stream);
+
+/* Free the fork's host metadata (not its buffer). NULL is a no-op. */
+void kvr_fork_destroy(kvr_fork *fork);
+
 /* Choose whether kvr_decode_attend_score / kvr_decode_step may use the
  * fused single-pass kernel (bf16, head_dim 128, G <= 8, at most 128 live rows
  * per unit, at most one eviction per unit; the default) or must use the

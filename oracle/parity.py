@@ -141,23 +141,3 @@ def check_and_adopt(o: orc.OracleCache, exports, B, W, evict=True,
                 keep_sets[s][l][h] = got
     o.keep_positions(keep_sets)
     return st
-
-
-def oracle_from_export(exports, G, d, cap, kv=True):
-    """Build an OracleCache holding exactly the CUDA state (for single-step
-    sampled checks at sizes where a full lock-step run is too slow)."""
-    S = len(exports)
-    L, H = exports[0]["len"].shape
-    o = orc.OracleCache(S, L, H, G, d, cap)
-    for s, ex in enumerate(exports):
-        o.len[s] = ex["len"]
-        for l in range(L):
-            for h in range(H):
-                n = ex["len"][l, h]
-                o.pos[s, l, h, :n] = ex["pos"][l, h, :n]
-                o.score[s, l, h, :n] = ex["score"][l, h, :n]
-                if kv:
-                    o.K[s, l, h, :n] = ex["K"][l, h, :n]
-                    o.V[s, l, h, :n] = ex["V"][l, h, :n]
-                o.next_pos[s, l, h] = ex["next_pos"][l, h]
-    return o

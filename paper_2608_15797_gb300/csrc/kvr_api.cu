@@ -99,6 +99,7 @@ struct kvr_cache {
   bool fused = true;              // use the fused kernel where it applies
   int fused_groups = 0;           // units computed at once per SM (0: auto)
   int fused_group_warps = 0;      // warps per unit (0: auto)
+  int forks = 0;                  // live forks: the cache is read-only meanwhile
   int sm_count = 0;               // of the device, queried on first use
   int smem_optin = 0;
   std::map<int, std::pair<CUtensorMap, CUtensorMap>> tmaps;  // by box rows
@@ -163,6 +164,7 @@ int max_len(const kvr_cache *c, int lb, int le) {
 kvr_status check_step(kvr_cache *c, int lb, int le, const void *q,
                       const void *k_new, const void *v_new, void *out) {
   if (!c) return fail(KVR_EINVAL, "null cache");
+  if (c->forks) return fail(KVR_ESTATE, "the cache has a live fork");
   kvr_status st = check_layers(c, lb, le);
   if (st != KVR_OK) return st;
   if (!q || !k_new || !v_new || !out)
@@ -356,6 +358,7 @@ void kvr_cache_destroy(kvr_cache *cache) { delete cache; }
 kvr_status kvr_cache_load(kvr_cache *c, int seq, const void *k, const void *v,
                           int n_rows, int first_pos, void *stream) {
   if (!c) return fail(KVR_EINVAL, "null cache");
+  if (c->forks) return fail(KVR_ESTATE, "the cache has a live fork");
   if (seq < 0 || seq >= c->desc.n_seq)
     return fail(KVR_EINVAL, "sequence %d outside [0, %d)", seq, c->desc.n_seq);
   if (n_rows < 0 || first_pos < 0 ||
@@ -449,6 +452,7 @@ extern "C" {
 kvr_status kvr_evict_compact(kvr_cache *c, int lb, int le, int budget,
                              int window, void *stream) {
   if (!c) return fail(KVR_EINVAL, "null cache");
+  if (c->forks) return fail(KVR_ESTATE, "the cache has a live fork");
   kvr_status st = check_layers(c, lb, le);
   if (st != KVR_OK) return st;
   st = check_evict(budget, window);
@@ -563,5 +567,258 @@ kvr_status kvr_sync_status(kvr_cache *c, void *stream) {
 }
 
 const char *kvr_last_error(void) { return g_err.c_str(); }
+
+}  // extern "C"
+
+// ---- candidates ------------------------------------------------------------
+
+struct kvr_fork {
+  kvr_cache *parent;
+  kvr::ForkView view;
+  std::vector<int32_t> tlen;  // host mirror [S][L] (same for all candidates)
+  int32_t *chosen_dev;        // [S]
+  bool spent = false;
+};
+
+namespace {
+
+struct ForkLayout {
+  size_t pscore, tk, tv, tscore, tpos, tlen, chosen, total;
+};
+
+ForkLayout fork_layout(const kvr_cache *p, int n_cand, int tail_cap) {
+  const kvr_cache_desc &d = p->desc;
+  const size_t units = (size_t)d.n_seq * d.n_layers * d.n_kv_heads;
+  const size_t cu = units * (size_t)n_cand;
+  const size_t tstride = kvr::round_up16(tail_cap);
+  ForkLayout l{};
+  size_t off = 0;
+  l.pscore = off;
+  off = align_up(off + cu * kvr::round_up16(d.capacity) * sizeof(float));
+  l.tk = off;
+  off = align_up(off + cu * tail_cap * d.head_dim * esize(d.kv_dtype));
+  l.tv = off;
+  off = align_up(off + cu * tail_cap * d.head_dim * esize(d.kv_dtype));
+  l.tscore = off;
+  off = align_up(off + cu * tstride * sizeof(float));
+  l.tpos = off;
+  off = align_up(off + cu * tstride * sizeof(int32_t));
+  l.tlen = off;
+  off = align_up(off + cu * sizeof(int32_t));
+  l.chosen = off;
+  off = align_up(off + (size_t)d.n_seq * sizeof(int32_t));
+  l.total = off;
+  return l;
+}
+
+bool fork_args_ok(const kvr_cache *p, int n_cand, int tail_cap) {
+  return p && n_cand >= 1 && n_cand <= 64 && tail_cap >= 1 &&
+         tail_cap <= (1 << 20);
+}
+
+kvr_status check_fork(const kvr_fork *f) {
+  if (!f) return fail(KVR_EINVAL, "null fork");
+  if (f->spent) return fail(KVR_ESTATE, "the fork has been committed");
+  return KVR_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t kvr_fork_required_bytes(const kvr_cache *parent, int n_cand,
+                               int tail_cap) {
+  if (!fork_args_ok(parent, n_cand, tail_cap)) return 0;
+  return fork_layout(parent, n_cand, tail_cap).total;
+}
+
+kvr_status kvr_fork_candidates(kvr_cache *p, int n_cand, int tail_cap,
+                               void *dev_buf, size_t bytes, void *stream,
+                               kvr_fork **out) {
+  if (!out) return fail(KVR_EINVAL, "null output handle");
+  *out = nullptr;
+  if (!fork_args_ok(p, n_cand, tail_cap))
+    return fail(KVR_EINVAL, "bad fork arguments (%d candidates, tail %d)",
+                n_cand, tail_cap);
+  if (p->forks) return fail(KVR_ESTATE, "the cache already has a live fork");
+  if (!dev_buf || reinterpret_cast<uintptr_t>(dev_buf) % kAlign)
+    return fail(KVR_EINVAL, "null or unaligned fork buffer");
+  const ForkLayout lay = fork_layout(p, n_cand, tail_cap);
+  if (bytes < lay.total)
+    return fail(KVR_ENOMEM, "fork buffer of %zu bytes < required %zu", bytes,
+                lay.total);
+  kvr_fork *f = new (std::nothrow) kvr_fork();
+  if (!f) return fail(KVR_ENOMEM, "host allocation failed");
+  char *b = static_cast<char *>(dev_buf);
+  kvr::ForkView &v = f->view;
+  v.p = p->view;
+  v.N = n_cand;
+  v.tcap = tail_cap;
+  v.tstride = kvr::round_up16(tail_cap);
+  v.pscore = reinterpret_cast<float *>(b + lay.pscore);
+  v.TK = b + lay.tk;
+  v.TV = b + lay.tv;
+  v.tscore = reinterpret_cast<float *>(b + lay.tscore);
+  v.tpos = reinterpret_cast<int32_t *>(b + lay.tpos);
+  v.tlen = reinterpret_cast<int32_t *>(b + lay.tlen);
+  f->chosen_dev = reinterpret_cast<int32_t *>(b + lay.chosen);
+  f->parent = p;
+  f->tlen.assign(p->len.size(), 0);
+  const size_t units =
+      (size_t)p->desc.n_seq * p->desc.n_layers * p->desc.n_kv_heads;
+  const size_t sbytes = units * p->view.sstride * sizeof(float);
+  cudaStream_t st = as_stream(stream);
+  cudaError_t e = cudaSuccess;
+  for (int c = 0; c < n_cand && e == cudaSuccess; ++c)
+    e = cudaMemcpyAsync(v.pscore + c * units * p->view.sstride, p->view.score,
+                        sbytes, cudaMemcpyDeviceToDevice, st);
+  if (e == cudaSuccess)
+    e = cudaMemsetAsync(v.tlen, 0, units * n_cand * sizeof(int32_t), st);
+  if (e != cudaSuccess) {
+    delete f;
+    return cuda_fail("kvr_fork_candidates", e);
+  }
+  p->forks += 1;
+  *out = f;
+  return KVR_OK;
+}
+
+kvr_status kvr_fork_decode_attend_score(kvr_fork *f, int lb, int le,
+                                        const void *q, const void *k_new,
+                                        const void *v_new, void *out,
+                                        void *stream) {
+  kvr_status st = check_fork(f);
+  if (st != KVR_OK) return st;
+  kvr_cache *p = f->parent;
+  st = check_layers(p, lb, le);
+  if (st != KVR_OK) return st;
+  if (!q || !k_new || !v_new || !out)
+    return fail(KVR_EINVAL, "null q, k_new, v_new or out");
+  int max_prefix = 0, n_max = 0;
+  for (int s = 0; s < p->desc.n_seq; ++s)
+    for (int l = lb; l < le; ++l) {
+      const size_t i = (size_t)s * p->desc.n_layers + l;
+      if (f->tlen[i] + 1 > f->view.tcap)
+        return fail(KVR_ECAPACITY, "a candidate tail holds %d rows; capacity %d"
+                    " is full", f->tlen[i], f->view.tcap);
+      max_prefix = std::max(max_prefix, p->len[i]);
+      n_max = std::max(n_max, p->len[i] + f->tlen[i] + 1);
+    }
+  int dev = 0, optin = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  if (kvr::fork_attend_smem_bytes(p->view, n_max, max_prefix) > (size_t)optin)
+    return fail(KVR_EINVAL, "prefix of %d rows is too long for the candidate "
+                "kernel's shared memory", max_prefix);
+  StepArgs a{};
+  a.lb = lb;
+  a.nl = le - lb;
+  a.q = q;
+  a.k_new = k_new;
+  a.v_new = v_new;
+  a.out = out;
+  a.max_rows = n_max;
+  cudaError_t e =
+      kvr::launch_fork_attend(f->view, a, n_max, max_prefix, as_stream(stream));
+  if (e != cudaSuccess) return cuda_fail("kvr_fork_decode_attend_score", e);
+  p->launches += 1;
+  for (int s = 0; s < p->desc.n_seq; ++s)
+    for (int l = lb; l < le; ++l) f->tlen[(size_t)s * p->desc.n_layers + l] += 1;
+  return KVR_OK;
+}
+
+kvr_status kvr_fork_commit(kvr_fork *f, const int32_t *chosen, int budget,
+                           int window, void *stream) {
+  kvr_status st = check_fork(f);
+  if (st != KVR_OK) return st;
+  if (!chosen) return fail(KVR_EINVAL, "null chosen");
+  st = check_evict(budget, window);
+  if (st != KVR_OK) return st;
+  kvr_cache *p = f->parent;
+  for (int s = 0; s < p->desc.n_seq; ++s)
+    if (chosen[s] < 0 || chosen[s] >= f->view.N)
+      return fail(KVR_EINVAL, "chosen[%d] = %d outside [0, %d)", s, chosen[s],
+                  f->view.N);
+  int max_rows = 1;
+  for (size_t i = 0; i < p->len.size(); ++i)
+    max_rows = std::max(max_rows, p->len[i] + f->tlen[i]);
+  cudaStream_t strm = as_stream(stream);
+  cudaError_t e = cudaMemcpyAsync(f->chosen_dev, chosen,
+                                  p->desc.n_seq * sizeof(int32_t),
+                                  cudaMemcpyHostToDevice, strm);
+  if (e == cudaSuccess)
+    e = kvr::launch_fork_commit(f->view, f->chosen_dev, max_rows, budget,
+                                window, strm);
+  if (e != cudaSuccess) return cuda_fail("kvr_fork_commit", e);
+  p->launches += 1;
+  for (size_t i = 0; i < p->len.size(); ++i) {
+    p->len[i] = (int32_t)std::min<long long>((long long)p->len[i] + f->tlen[i],
+                                             (long long)budget + window);
+    p->next_pos[i] += f->tlen[i];
+  }
+  f->spent = true;
+  p->forks -= 1;
+  return KVR_OK;
+}
+
+kvr_status kvr_fork_export(const kvr_fork *f, int cand, int seq,
+                           float *host_prefix_score, void *host_tail_k,
+                           void *host_tail_v, float *host_tail_score,
+                           int32_t *host_tail_pos, int32_t *host_tail_len,
+                           void *stream) {
+  if (!f) return fail(KVR_EINVAL, "null fork");
+  const kvr_cache *p = f->parent;
+  const kvr::ForkView &v = f->view;
+  if (cand < 0 || cand >= v.N || seq < 0 || seq >= p->desc.n_seq)
+    return fail(KVR_EINVAL, "candidate %d / sequence %d out of range", cand,
+                seq);
+  cudaError_t e = cudaStreamSynchronize(as_stream(stream));
+  if (e != cudaSuccess) return cuda_fail("kvr_fork_export: sync", e);
+  const size_t units =
+      (size_t)p->desc.n_seq * p->desc.n_layers * p->desc.n_kv_heads;
+  const size_t per_seq = (size_t)p->desc.n_layers * p->desc.n_kv_heads;
+  const size_t cu0 = (size_t)cand * units + (size_t)seq * per_seq;
+  const size_t ebytes = (size_t)p->desc.head_dim * esize(p->desc.kv_dtype);
+  if (host_prefix_score &&
+      (e = cudaMemcpy2D(host_prefix_score, (size_t)p->view.cap * 4,
+                        v.pscore + cu0 * p->view.sstride,
+                        (size_t)p->view.sstride * 4, (size_t)p->view.cap * 4,
+                        per_seq, cudaMemcpyDeviceToHost)) != cudaSuccess)
+    return cuda_fail("kvr_fork_export", e);
+  const size_t tbytes = per_seq * v.tcap * ebytes;
+  if (host_tail_k &&
+      (e = cudaMemcpy(host_tail_k,
+                      static_cast<char *>(v.TK) + cu0 * v.tcap * ebytes, tbytes,
+                      cudaMemcpyDeviceToHost)) != cudaSuccess)
+    return cuda_fail("kvr_fork_export", e);
+  if (host_tail_v &&
+      (e = cudaMemcpy(host_tail_v,
+                      static_cast<char *>(v.TV) + cu0 * v.tcap * ebytes, tbytes,
+                      cudaMemcpyDeviceToHost)) != cudaSuccess)
+    return cuda_fail("kvr_fork_export", e);
+  if (host_tail_score &&
+      (e = cudaMemcpy2D(host_tail_score, (size_t)v.tcap * 4,
+                        v.tscore + cu0 * v.tstride, (size_t)v.tstride * 4,
+                        (size_t)v.tcap * 4, per_seq,
+                        cudaMemcpyDeviceToHost)) != cudaSuccess)
+    return cuda_fail("kvr_fork_export", e);
+  if (host_tail_pos &&
+      (e = cudaMemcpy2D(host_tail_pos, (size_t)v.tcap * 4,
+                        v.tpos + cu0 * v.tstride, (size_t)v.tstride * 4,
+                        (size_t)v.tcap * 4, per_seq,
+                        cudaMemcpyDeviceToHost)) != cudaSuccess)
+    return cuda_fail("kvr_fork_export", e);
+  if (host_tail_len &&
+      (e = cudaMemcpy(host_tail_len, v.tlen + cu0, per_seq * sizeof(int32_t),
+                      cudaMemcpyDeviceToHost)) != cudaSuccess)
+    return cuda_fail("kvr_fork_export", e);
+  return KVR_OK;
+}
+
+void kvr_fork_destroy(kvr_fork *f) {
+  if (!f) return;
+  if (!f->spent) f->parent->forks -= 1;
+  delete f;
+}
 
 }  // extern "C"

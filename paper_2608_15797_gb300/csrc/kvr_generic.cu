@@ -15,43 +15,13 @@
 #include <cuda_bf16.h>
 #include <math.h>
 
+#include "kvr_device.cuh"
 #include "kvr_internal.h"
 
 namespace kvr {
 namespace {
 
-constexpr int kThreads = 256;
-constexpr int kWarps = kThreads / 32;
-constexpr int kMaxG = 8;
-
-__device__ __forceinline__ float to_f(float x) { return x; }
-__device__ __forceinline__ float to_f(__nv_bfloat16 x) {
-  return __bfloat162float(x);
-}
-
-__device__ __forceinline__ float2 ld2(const float *p) {
-  return *reinterpret_cast<const float2 *>(p);
-}
-__device__ __forceinline__ float2 ld2(const __nv_bfloat16 *p) {
-  return __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(p));
-}
-
-__device__ __forceinline__ void st1(float *p, float x) { *p = x; }
-__device__ __forceinline__ void st1(__nv_bfloat16 *p, float x) {
-  *p = __float2bfloat16_rn(x);
-}
-
-__device__ __forceinline__ float warp_sum(float x) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
-  return x;
-}
-__device__ __forceinline__ float warp_max(float x) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1)
-    x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, o));
-  return x;
-}
+using namespace dev;
 
 struct Unit {
   int s, lr, l, h;
@@ -219,43 +189,6 @@ __global__ void __launch_bounds__(kThreads)
   }
 }
 
-// Collect, in slot order, the indices i in [lo, hi) with pred(i) into list.
-// Every thread of the block must call it; returns the count.
-template <typename Pred>
-__device__ int block_collect(int lo, int hi, Pred pred, int *list,
-                             int *s_wsum, int *s_base) {
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  if (tid == 0) *s_base = 0;
-  __syncthreads();
-  for (int base = lo; base < hi; base += kThreads) {
-    const int i = base + tid;
-    const bool f = i < hi && pred(i);
-    const unsigned bal = __ballot_sync(0xffffffffu, f);
-    if (lane == 0) s_wsum[warp] = __popc(bal);
-    __syncthreads();
-    int off = *s_base;
-    for (int w = 0; w < warp; ++w) off += s_wsum[w];
-    if (f) list[off + __popc(bal & ((1u << lane) - 1u))] = i;
-    __syncthreads();
-    if (tid == 0) {
-      int tot = 0;
-      for (int w = 0; w < kWarps; ++w) tot += s_wsum[w];
-      *s_base += tot;
-    }
-    __syncthreads();
-  }
-  const int total = *s_base;
-  __syncthreads();  // every thread has read the count before it is reused
-  return total;
-}
-
-// TopB key: higher score first, then lower position (scores are >= 0, so
-// their IEEE bit patterns order like the values).
-__device__ __forceinline__ unsigned long long rank_key(float s, int32_t p) {
-  return ((unsigned long long)__float_as_uint(s) << 32) |
-         (unsigned long long)(0xFFFFFFFFu - (unsigned)p);
-}
-
 template <typename T, int D>
 __global__ void __launch_bounds__(kThreads)
     evict_kernel(CacheView c, int lb, int nl, int B, int W) {
@@ -277,38 +210,13 @@ __global__ void __launch_bounds__(kThreads)
   // position is at most newest - W.
   const int wlo = c.state[4 * x.u + 1] - 1 - W;
 
-  // Radix select (8 passes of 8 bits) of the B-th largest candidate key.
+  // Radix select of the B-th largest candidate key.
   unsigned long long thr = ~0ull;
-  if (B > 0) {
-    unsigned long long prefix = 0, mask = 0;
-    int need = B;
-    for (int shift = 56; shift >= 0; shift -= 8) {
-      for (int i = tid; i < 256; i += kThreads) hist[i] = 0;
-      __syncthreads();
-      for (int i = tid; i < n; i += kThreads) {
-        if (pu[i] <= wlo) {
-          const unsigned long long k = rank_key(su[i], pu[i]);
-          if ((k & mask) == prefix) atomicAdd(&hist[(k >> shift) & 255], 1u);
-        }
-      }
-      __syncthreads();
-      if (tid == 0) {
-        int cnt = 0, dg = 255;
-        for (; dg > 0; --dg) {
-          if (cnt + (int)hist[dg] >= need) break;
-          cnt += (int)hist[dg];
-        }
-        s_prefix = prefix | ((unsigned long long)dg << shift);
-        s_need = need - cnt;
-      }
-      __syncthreads();
-      prefix = s_prefix;
-      need = s_need;
-      mask |= 0xFFull << shift;
-      __syncthreads();
-    }
-    thr = prefix;
-  }
+  if (B > 0)
+    thr = block_select(
+        n, B, [&](int i) { return pu[i] <= wlo; },
+        [&](int i) { return rank_key(su[i], pu[i]); }, hist, &s_prefix,
+        &s_need);
   auto keep = [&](int i) {
     const int32_t p = pu[i];
     return p > wlo || (B > 0 && rank_key(su[i], p) >= thr);

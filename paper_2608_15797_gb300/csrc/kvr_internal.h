@@ -89,6 +89,25 @@ cudaError_t launch_fused_step(const CUtensorMap &tmK, const CUtensorMap &tmV,
                               const FusedParams &p, int grid, int smem_bytes,
                               cudaStream_t st);
 
+// Candidates of one cache (kvr_fork.cu).  A candidate unit cu = c * units + u.
+struct ForkView {
+  CacheView p;       // the parent: its live rows are every candidate's prefix
+  int N;             // candidates
+  int tcap;          // tail rows per candidate unit
+  int tstride;       // tcap rounded up to 16
+  float *pscore;     // [N][units][p.sstride] candidate copies of the scores
+  void *TK, *TV;     // [N][units][tcap][d]
+  float *tscore;     // [N][units][tstride]
+  int32_t *tpos;     // [N][units][tstride]
+  int32_t *tlen;     // [N][units]
+};
+size_t fork_attend_smem_bytes(const CacheView &c, int n_max, int max_prefix);
+cudaError_t launch_fork_attend(const ForkView &f, const StepArgs &a, int n_max,
+                               int max_prefix, cudaStream_t st);
+cudaError_t launch_fork_commit(const ForkView &f, const int32_t *chosen,
+                               int max_rows, int budget, int window,
+                               cudaStream_t st);
+
 }  // namespace kvr
 
 struct kvr_cache;

@@ -290,3 +290,108 @@ class Cache:
 
     def sync_status(self, stream=None):
         kvr_sync_status(self.handle, stream)
+
+
+# ---- candidates -------------------------------------------------------------
+
+for _name, (_res, _args) in {
+    "kvr_fork_required_bytes": (ctypes.c_size_t, [_P, _I, _I]),
+    "kvr_fork_candidates": (_S, [_P, _I, _I, _P, ctypes.c_size_t, _P,
+                                 ctypes.POINTER(_P)]),
+    "kvr_fork_decode_attend_score": (_S, [_P, _I, _I, _P, _P, _P, _P, _P]),
+    "kvr_fork_commit": (_S, [_P, _P, _I, _I, _P]),
+    "kvr_fork_export": (_S, [_P, _I, _I, _P, _P, _P, _P, _P, _P, _P]),
+    "kvr_fork_destroy": (None, [_P]),
+}.items():
+    _f = getattr(lib, _name)
+    _f.restype = _res
+    _f.argtypes = _args
+
+
+def kvr_fork_required_bytes(parent, n_cand, tail_cap) -> int:
+    return int(lib.kvr_fork_required_bytes(parent, n_cand, tail_cap))
+
+
+def kvr_fork_candidates(parent, n_cand, tail_cap, dev_buf, nbytes, stream=None):
+    h = ctypes.c_void_p()
+    _check(lib.kvr_fork_candidates(parent, n_cand, tail_cap, _ptr(dev_buf),
+                                   nbytes, _stream(stream), ctypes.byref(h)),
+           "kvr_fork_candidates")
+    return h
+
+
+def kvr_fork_decode_attend_score(fork, layer_begin, layer_end, q, k_new, v_new,
+                                 out, stream=None):
+    _check(lib.kvr_fork_decode_attend_score(fork, layer_begin, layer_end,
+                                            _ptr(q), _ptr(k_new), _ptr(v_new),
+                                            _ptr(out), _stream(stream)),
+           "kvr_fork_decode_attend_score")
+
+
+def kvr_fork_commit(fork, chosen, budget, window, stream=None):
+    chosen = np.ascontiguousarray(chosen, dtype=np.int32)
+    _check(lib.kvr_fork_commit(fork, _ptr(chosen), budget, window,
+                               _stream(stream)), "kvr_fork_commit")
+
+
+def kvr_fork_export(fork, cand, seq, prefix_score, tail_k, tail_v, tail_score,
+                    tail_pos, tail_len, stream=None):
+    _check(lib.kvr_fork_export(fork, cand, seq, _ptr(prefix_score), _ptr(tail_k),
+                               _ptr(tail_v), _ptr(tail_score), _ptr(tail_pos),
+                               _ptr(tail_len), _stream(stream)),
+           "kvr_fork_export")
+
+
+def kvr_fork_destroy(fork):
+    lib.kvr_fork_destroy(fork)
+
+
+class Fork:
+    """N candidates of a Cache sharing its live rows (owner of the buffer)."""
+
+    def __init__(self, cache: Cache, n_cand: int, tail_cap: int, stream=None):
+        self.cache, self.N, self.tcap = cache, n_cand, tail_cap
+        self.nbytes = kvr_fork_required_bytes(cache.handle, n_cand, tail_cap)
+        if self.nbytes == 0:
+            raise KvrError(KVR_EINVAL, "Fork", "invalid fork arguments")
+        self.buf = torch.empty(self.nbytes, dtype=torch.uint8,
+                               device=cache.buf.device)
+        self.handle = kvr_fork_candidates(cache.handle, n_cand, tail_cap,
+                                          self.buf, self.nbytes, stream)
+
+    def __del__(self):
+        h = getattr(self, "handle", None)
+        if h:
+            kvr_fork_destroy(h)
+            self.handle = None
+
+    def attend_score(self, q, k_new, v_new, out=None, layers=None, stream=None):
+        c = self.cache
+        lb, le = (0, c.L) if layers is None else layers
+        if out is None:
+            out = torch.empty(self.N, c.S, le - lb, c.H * c.G, c.d,
+                              dtype=c.out_torch_dtype, device=c.buf.device)
+        kvr_fork_decode_attend_score(self.handle, lb, le, q, k_new, v_new, out,
+                                     stream)
+        return out
+
+    def commit(self, chosen, budget, window, stream=None):
+        kvr_fork_commit(self.handle, chosen, budget, window, stream)
+
+    def export(self, cand, seq, kv=False, stream=None):
+        c = self.cache
+        ps = np.zeros((c.L, c.H, c.cap), np.float32)
+        ts = np.zeros((c.L, c.H, self.tcap), np.float32)
+        tp = np.zeros((c.L, c.H, self.tcap), np.int32)
+        tl = np.zeros((c.L, c.H), np.int32)
+        tk = tv = None
+        if kv:
+            tk = torch.empty(c.L, c.H, self.tcap, c.d, dtype=c.kv_torch_dtype)
+            tv = torch.empty_like(tk)
+        kvr_fork_export(self.handle, cand, seq, ps, tk, tv, ts, tp, tl, stream)
+        res = {"prefix_score": ps, "tail_score": ts, "tail_pos": tp,
+               "tail_len": tl}
+        if kv:
+            res["tail_K"] = tk.float().numpy()
+            res["tail_V"] = tv.float().numpy()
+        return res

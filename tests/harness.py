@@ -66,3 +66,69 @@ def lockstep(c: kvr.Cache, o: orc.OracleCache, w: inputs.Workload, seed: int,
         stats.steps = t - step0 + 1
     c.sync_status()
     return stats
+
+
+def _unit_map(pos, score):
+    return dict(zip(np.asarray(pos).tolist(), np.asarray(score, np.float64).tolist()))
+
+
+def fork_lockstep(c: kvr.Cache, o: orc.OracleCache, w: inputs.Workload,
+                  seed: int, n_cand: int, steps: int, budget: int, window: int,
+                  pick_step: int = 0, tail_cap=None):
+    """Fork both sides into n_cand candidates, decode `steps` tokens per
+    candidate checking every candidate after every token (outputs; scores of
+    every prefix and tail row, by position), then commit a seeded pick (the
+    stand-in for the PRM argmax of Eq. 2) on both sides and check the parent.
+    Returns (oracle after commit, chosen, stats)."""
+    S = c.S
+    parent_pos = [c.export(s, kv=False) for s in range(S)]
+    f = kvr.Fork(c, n_cand, tail_cap or steps)
+    cands = o.fork(n_cand)
+    stats = parity.Stats()
+    for t in range(steps):
+        per = [inputs.step_inputs(w, seed, 10_000 + t, S, cand=k + 1)
+               for k in range(n_cand)]
+        Q, K, V = (np.stack([p[i] for p in per]) for i in range(3))
+        out = f.attend_score(dev(Q, w.dtype), dev(K, w.dtype), dev(V, w.dtype))
+        torch.cuda.synchronize()
+        out = out.float().cpu().numpy()
+        for k in range(n_cand):
+            ref = cands[k].step(*per[k], evict=False)
+            stats.max_out_excess = max(stats.max_out_excess, parity.check_out(
+                out[k], ref, what=f"candidate {k} out at token {t}"))
+            for s in range(S):
+                ex = f.export(k, s)
+                for l in range(c.L):
+                    for h in range(c.H):
+                        n_p = parent_pos[s]["len"][l, h]
+                        n_t = ex["tail_len"][l, h]
+                        got = _unit_map(parent_pos[s]["pos"][l, h, :n_p],
+                                        ex["prefix_score"][l, h, :n_p])
+                        got.update(_unit_map(ex["tail_pos"][l, h, :n_t],
+                                             ex["tail_score"][l, h, :n_t]))
+                        p_ref, s_ref, _, _ = cands[k].unit_rows(s, l, h)
+                        want = _unit_map(p_ref, s_ref)
+                        if got.keys() != want.keys():
+                            raise parity.ParityError(
+                                f"candidate {k} seq {s} layer {l} head {h}: "
+                                f"rows differ at token {t}")
+                        a = np.array([got[p] for p in want])
+                        b = np.array([want[p] for p in want])
+                        rel = np.abs(a - b) / np.maximum(np.abs(b), parity.SCORE_FLOOR)
+                        if rel.max() > parity.SCORE_RTOL:
+                            raise parity.ParityError(
+                                f"candidate {k} seq {s} layer {l} head {h}: score"
+                                f" rel {rel.max():.3g} at token {t}")
+                        stats.max_score_rel = max(stats.max_score_rel, float(rel.max()))
+        stats.steps += 1
+    chosen = inputs.candidate_pick(seed, pick_step, S, n_cand)
+    f.commit(chosen, budget, window)
+    committed = o.copy()
+    for s in range(S):
+        src = cands[int(chosen[s])]
+        for name in ("K", "V", "score", "pos", "len", "next_pos"):
+            getattr(committed, name)[s] = getattr(src, name)[s]
+    exports = [c.export(s, kv=False) for s in range(S)]
+    stats.merge(parity.check_and_adopt(committed, exports, budget, window))
+    c.sync_status()
+    return committed, chosen, stats

@@ -1,0 +1,123 @@
+"""Candidates (Sec. 2.2 Eq. 2, App. Impl. best-of-(N+N)) against the oracle.
+
+The oracle forks by physical copy (what the paper's engine does): each
+candidate is a full copy of the parent that decodes its tokens without
+eviction and is cut to B + W at commit.  The CUDA path shares the parent's
+rows as a read-only prefix; both must agree on every candidate's outputs and
+scores after every token, and on the committed parent.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import parity
+from paper_2608_15797_gb300 import inputs, kvr
+from tests import harness
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(autouse=True)
+def _cuda():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA device")
+    torch.cuda.set_device(0)
+
+
+def _evicted_pair(w, seed, S, cap, prompt_lens, warm_steps):
+    """Load prompts and run evicting steps so the parent sits at B + W rows."""
+    c, o = harness.make_pair(w, seed, S, cap=cap, prompt_lens=prompt_lens)
+    harness.lockstep(c, o, w, seed, warm_steps, w.budget, w.window)
+    return c, o
+
+
+@pytest.mark.parametrize("n_cand", [1, 3])
+def test_small_fork_commit_then_continue(n_cand):
+    w = inputs.Workload("f", 2, 2, 3, 128, "bf16", 12, 4, 30, 0, sigma=1.0)
+    c, o = _evicted_pair(w, 21, 2, cap=40, prompt_lens=[30, 9], warm_steps=3)
+    o2, chosen, st = harness.fork_lockstep(c, o, w, 21, n_cand, 7, w.budget,
+                                           w.window)
+    assert (c.lengths() == np.minimum(o2.len.max(axis=2), 16)).all()
+    # the committed parent keeps decoding in lock-step
+    harness.lockstep(c, o2, w, 21, 4, w.budget, w.window, step0=100)
+
+
+def test_fork_parent_is_read_only_while_alive():
+    w = inputs.Workload("f", 1, 1, 2, 64, "f32", 4, 2, 8, 0, sigma=1.0)
+    c, _ = harness.make_pair(w, 22, 1, cap=16)
+    f = kvr.Fork(c, 2, 4)
+    q, kn, vn = (harness.dev(a, "f32") for a in inputs.step_inputs(w, 22, 0, 1))
+    with pytest.raises(kvr.KvrError) as e:
+        c.step(q, kn, vn, 4, 2)
+    assert e.value.status == kvr.KVR_ESTATE
+    with pytest.raises(kvr.KvrError) as e:
+        f.commit(np.array([2], np.int32), 4, 2)
+    assert e.value.status == kvr.KVR_EINVAL
+    f.commit(np.array([1], np.int32), 4, 2)
+    with pytest.raises(kvr.KvrError) as e:
+        f.commit(np.array([1], np.int32), 4, 2)
+    assert e.value.status == kvr.KVR_ESTATE
+    c.step(q, kn, vn, 4, 2)  # the parent is writable again
+
+
+def test_fork_tail_capacity():
+    w = inputs.Workload("f", 1, 1, 2, 128, "bf16", 4, 2, 8, 0, sigma=1.0)
+    c, _ = harness.make_pair(w, 23, 1, cap=16)
+    f = kvr.Fork(c, 2, 2)
+    per = [inputs.step_inputs(w, 23, 0, 1, cand=k + 1) for k in range(2)]
+    Q, K, V = (harness.dev(np.stack([p[i] for p in per]), "bf16") for i in range(3))
+    f.attend_score(Q, K, V)
+    f.attend_score(Q, K, V)
+    with pytest.raises(kvr.KvrError) as e:
+        f.attend_score(Q, K, V)
+    assert e.value.status == kvr.KVR_ECAPACITY
+
+
+def test_single_candidate_equals_plain_deferred_eviction():
+    """With N = 1, fork + T tokens + commit equals the plain cache driven
+    through the same T tokens with eviction held back, then one eviction."""
+    w = inputs.Workload("f", 2, 2, 4, 128, "bf16", 10, 3, 40, 0, sigma=1.0)
+    c1, o1 = _evicted_pair(w, 24, 2, cap=41, prompt_lens=[40, 22], warm_steps=2)
+    c2, _ = _evicted_pair(w, 24, 2, cap=41, prompt_lens=[40, 22], warm_steps=2)
+    T = 6
+    f = kvr.Fork(c1, 1, T)
+    for t in range(T):
+        q, kn, vn = inputs.step_inputs(w, 24, 10_000 + t, 2, cand=1)
+        f.attend_score(*(harness.dev(a[None], "bf16") for a in (q, kn, vn)))
+        c2.attend_score(*(harness.dev(a, "bf16") for a in (q, kn, vn)))
+    f.commit(np.zeros(2, np.int32), w.budget, w.window)
+    c2.evict(w.budget, w.window)
+    for s in range(2):
+        a, b = c1.export(s, kv=False), c2.export(s, kv=False)
+        assert (a["len"] == b["len"]).all()
+        for l in range(2):
+            for h in range(2):
+                n = a["len"][l, h]
+                ma = dict(zip(a["pos"][l, h, :n].tolist(), a["score"][l, h, :n].tolist()))
+                mb = dict(zip(b["pos"][l, h, :n].tolist(), b["score"][l, h, :n].tolist()))
+                assert ma.keys() == mb.keys()
+                for p in ma:
+                    assert abs(ma[p] - mb[p]) <= 1e-4 * max(abs(mb[p]), 1e-6)
+
+
+def test_7b_best_of_4():
+    """7B geometry stepwise best-of-4: an evicted cache (prompt 512, B=128,
+    W=8; heavy keys), forked to 4 candidates that decode a 16-token step
+    sharing the prefix, then re-evicted and committed."""
+    w = inputs.WORKLOADS["7b_bon4"]
+    c, o = _evicted_pair(w, 25, 1, cap=w.prompt + 1, prompt_lens=[w.prompt],
+                         warm_steps=2)
+    o2, chosen, st = harness.fork_lockstep(c, o, w, 25, w.n_cand, 16, w.budget,
+                                           w.window)
+    assert (c.lengths() == w.budget + w.window).all()
+
+
+def test_72b_best_of_8():
+    """72B geometry (80 layers, 8 KV heads, G=8), B=64, N=8 candidates, an
+    8-token step (reduced from 64 to keep the oracle fast)."""
+    w = inputs.Workload("72b_small", 80, 8, 8, 128, "bf16", 64, 8, 200, 0,
+                        sigma=1.0 / np.sqrt(128.0))
+    c, o = _evicted_pair(w, 26, 1, cap=w.prompt + 1, prompt_lens=[w.prompt],
+                         warm_steps=1)
+    harness.fork_lockstep(c, o, w, 26, 8, 8, w.budget, w.window)
+    assert (c.lengths() == w.budget + w.window).all()
