@@ -127,6 +127,28 @@ kvr_status kvr_decode_step(kvr_cache *cache, int layer_begin, int layer_end,
                            const void *q, const void *k_new, const void *v_new,
                            void *out, int budget, int window, void *stream);
 
+/* ---- full-context decode (the helper's cache: no scores, no eviction) -- */
+
+/* The full-context helper of KV-Rescue keeps its whole cache (Sec. 3.1;
+ * App. C, Eq. 11): its decode step is Attn(q_t, C_t) of Eq. 1 over every
+ * cached row, with no importance scores and no eviction.  This call appends
+ * the new row (position = next position, score 0) and attends over all
+ * rows, splitting each unit's rows over n_splits CTAs whose partial softmax
+ * states are merged afterwards (two kernels).  The other units' scores are
+ * not touched.  bf16 caches with head_dim 128 and G <= 8 only (KVR_EINVAL
+ * otherwise).  Shapes as kvr_decode_attend_score.  n_splits = 0 lets the
+ * library choose; workspace (device, caller-owned, 16-byte aligned) must
+ * hold kvr_decode_attend_workspace_bytes(cache, layer_begin, layer_end,
+ * n_splits) bytes (KVR_ENOMEM otherwise). */
+size_t kvr_decode_attend_workspace_bytes(const kvr_cache *cache,
+                                         int layer_begin, int layer_end,
+                                         int n_splits);
+kvr_status kvr_decode_attend(kvr_cache *cache, int layer_begin, int layer_end,
+                             const void *q, const void *k_new,
+                             const void *v_new, void *out, int n_splits,
+                             void *workspace, size_t workspace_bytes,
+                             void *stream);
+
 /* ---- candidates: stepwise best-of-N over one shared cache state -------- */
 
 /* Sec. 2.2 (Eq. 2) and App. Impl. (best-of-(N+N)): each reasoning step draws

@@ -227,6 +227,39 @@ bool aligned16(const void *p) {
 
 // Launch the fused kernel if this call qualifies; returns false (and does
 // nothing) if it does not, true with *err set otherwise.
+// Device facts the dispatch needs, queried once per handle.
+bool device_facts(kvr_cache *c) {
+  if (c->sm_count) return true;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&c->sm_count, cudaDevAttrMultiProcessorCount,
+                             dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&c->smem_optin,
+                             cudaDevAttrMaxSharedMemoryPerBlockOptin,
+                             dev) != cudaSuccess) {
+    c->sm_count = 0;
+    return false;
+  }
+  return true;
+}
+
+// The K and V tensor maps with boxes of `box_rows` rows (created on first
+// use and kept in the handle); NULL if they cannot be encoded.
+const std::pair<CUtensorMap, CUtensorMap> *slab_maps(kvr_cache *c,
+                                                      int box_rows) {
+  auto it = c->tmaps.find(box_rows);
+  if (it == c->tmaps.end()) {
+    const CacheView &v = c->view;
+    const size_t rows = (size_t)v.S * v.L * v.H * v.cap;
+    std::pair<CUtensorMap, CUtensorMap> maps;
+    if (!encode_slab(&maps.first, v.K, rows, box_rows) ||
+        !encode_slab(&maps.second, v.V, rows, box_rows))
+      return nullptr;
+    it = c->tmaps.emplace(box_rows, maps).first;
+  }
+  return &it->second;
+}
+
 bool try_fused(kvr_cache *c, const StepArgs &a, bool evict, int budget,
                int window, cudaStream_t stream, cudaError_t *err) {
   const CacheView &v = c->view;
@@ -239,18 +272,7 @@ bool try_fused(kvr_cache *c, const StepArgs &a, bool evict, int budget,
   if (!aligned16(a.q) || !aligned16(a.k_new) || !aligned16(a.v_new) ||
       !aligned16(a.out))
     return false;
-  if (!c->sm_count) {
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&c->sm_count, cudaDevAttrMultiProcessorCount,
-                               dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&c->smem_optin,
-                               cudaDevAttrMaxSharedMemoryPerBlockOptin,
-                               dev) != cudaSuccess) {
-      c->sm_count = 0;
-      return false;
-    }
-  }
+  if (!device_facts(c)) return false;
   const int R = kvr::round_up16(a.max_rows);
   const int Rb = std::max(8, (a.max_rows - 1 + 7) / 8 * 8);
   const int U = kvr::fused_group_warps(R, c->fused_group_warps);
@@ -263,14 +285,8 @@ bool try_fused(kvr_cache *c, const StepArgs &a, bool evict, int budget,
                            (kvr::fused_max_threads() / 32 - 1) / U});
   if (c->fused_groups > 0) n_groups = std::min(n_groups, c->fused_groups);
   if (n_groups < 1) return false;
-  auto it = c->tmaps.find(Rb);
-  if (it == c->tmaps.end()) {
-    std::pair<CUtensorMap, CUtensorMap> maps;
-    if (!encode_slab(&maps.first, v.K, rows, Rb) ||
-        !encode_slab(&maps.second, v.V, rows, Rb))
-      return false;
-    it = c->tmaps.emplace(Rb, maps).first;
-  }
+  const std::pair<CUtensorMap, CUtensorMap> *maps = slab_maps(c, Rb);
+  if (!maps) return false;
   kvr::FusedParams p{};
   p.c = v;
   p.q = static_cast<const __nv_bfloat16 *>(a.q);
@@ -291,14 +307,81 @@ bool try_fused(kvr_cache *c, const StepArgs &a, bool evict, int budget,
   p.inv_g = 1.f / (float)v.G;
   const int units = v.S * a.nl * v.H;
   const int grid = std::min(c->sm_count, units);
-  *err = kvr::launch_fused_step(it->second.first, it->second.second, p, grid,
+  *err = kvr::launch_fused_step(maps->first, maps->second, p, grid,
                                 n_stages * stage + 1024, stream);
   return true;
+}
+
+// Splits for kvr_decode_attend: about two waves of the partial kernel (three
+// CTAs per SM), never less than 256 rows per split.
+int auto_splits(const kvr_cache *c, int lb, int le) {
+  const int units = c->desc.n_seq * (le - lb) * c->desc.n_kv_heads;
+  const int rows = max_len(c, lb, le) + 1;
+  const int sms = c->sm_count > 0 ? c->sm_count : 148;
+  const int want = (2 * 3 * sms + units - 1) / units;
+  return std::max(1, std::min(want, (rows + 255) / 256));
 }
 
 }  // namespace
 
 extern "C" {
+
+size_t kvr_decode_attend_workspace_bytes(const kvr_cache *c, int lb, int le,
+                                         int n_splits) {
+  if (!c || lb < 0 || le > c->desc.n_layers || lb >= le || n_splits < 0)
+    return 0;
+  if (n_splits == 0) {
+    device_facts(const_cast<kvr_cache *>(c));
+    n_splits = auto_splits(c, lb, le);
+  }
+  return kvr::split_workspace_bytes(c->view, le - lb, n_splits);
+}
+
+kvr_status kvr_decode_attend(kvr_cache *c, int lb, int le, const void *q,
+                             const void *k_new, const void *v_new, void *out,
+                             int n_splits, void *workspace,
+                             size_t workspace_bytes, void *stream) {
+  kvr_status st = check_step(c, lb, le, q, k_new, v_new, out);
+  if (st != KVR_OK) return st;
+  const CacheView &v = c->view;
+  if (!v.kv_bf16 || v.d != 128 || v.G > 8)
+    return fail(KVR_EINVAL, "kvr_decode_attend needs bf16, head_dim 128, G<=8");
+  if (n_splits < 0 || n_splits > 4096)
+    return fail(KVR_EINVAL, "bad n_splits %d", n_splits);
+  if (!aligned16(q) || !aligned16(k_new) || !aligned16(v_new) ||
+      !aligned16(out) || !aligned16(workspace))
+    return fail(KVR_EINVAL, "q, k_new, v_new, out and workspace must be "
+                "16-byte aligned");
+  const size_t rows = (size_t)v.S * v.L * v.H * v.cap;
+  if (rows >= (size_t)INT32_MAX)
+    return fail(KVR_EINVAL, "slab of %zu rows is beyond the TMA coordinate "
+                "range", rows);
+  if (!device_facts(c)) return fail(KVR_ECUDA, "cannot query the device");
+  if (n_splits == 0) n_splits = auto_splits(c, lb, le);
+  const size_t need = kvr::split_workspace_bytes(v, le - lb, n_splits);
+  if (!workspace || workspace_bytes < need)
+    return fail(KVR_ENOMEM, "workspace of %zu bytes < required %zu",
+                workspace_bytes, need);
+  const int box = kvr::split_rows_per_stage();
+  const std::pair<CUtensorMap, CUtensorMap> *maps = slab_maps(c, box);
+  if (!maps) return fail(KVR_ECUDA, "cannot encode the TMA descriptors");
+  kvr::SplitParams p{};
+  p.c = v;
+  p.q = static_cast<const __nv_bfloat16 *>(q);
+  p.k_new = static_cast<const __nv_bfloat16 *>(k_new);
+  p.v_new = static_cast<const __nv_bfloat16 *>(v_new);
+  p.lb = lb;
+  p.nl = le - lb;
+  p.n_splits = n_splits;
+  p.ws = static_cast<float *>(workspace);
+  p.scale_log2e = v.scale * 1.4426950408889634f;
+  cudaError_t e = kvr::launch_split_attend(maps->first, maps->second, p, out,
+                                           as_stream(stream));
+  if (e != cudaSuccess) return cuda_fail("kvr_decode_attend", e);
+  c->launches += 2;
+  mirror_append(c, lb, le);
+  return KVR_OK;
+}
 
 size_t kvr_cache_required_bytes(const kvr_cache_desc *desc) {
   if (!desc_ok(desc)) return 0;

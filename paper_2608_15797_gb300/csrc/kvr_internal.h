@@ -89,6 +89,21 @@ cudaError_t launch_fused_step(const CUtensorMap &tmK, const CUtensorMap &tmV,
                               const FusedParams &p, int grid, int smem_bytes,
                               cudaStream_t st);
 
+// Full-context decode split over the rows (kvr_split.cu): bf16, d = 128,
+// G <= 8.  ws holds [units of the call][n_splits][G][130] floats.
+struct SplitParams {
+  CacheView c;
+  const __nv_bfloat16 *q, *k_new, *v_new;
+  int lb, nl, n_splits;
+  float *ws;
+  float scale_log2e;
+};
+size_t split_workspace_bytes(const CacheView &c, int nl, int n_splits);
+int split_rows_per_stage();
+cudaError_t launch_split_attend(const CUtensorMap &tmK, const CUtensorMap &tmV,
+                                const SplitParams &p, void *out,
+                                cudaStream_t st);
+
 // Candidates of one cache (kvr_fork.cu).  A candidate unit cu = c * units + u.
 struct ForkView {
   CacheView p;       // the parent: its live rows are every candidate's prefix

@@ -395,3 +395,42 @@ class Fork:
             res["tail_K"] = tk.float().numpy()
             res["tail_V"] = tv.float().numpy()
         return res
+
+
+# ---- full-context decode ----------------------------------------------------
+
+for _name, (_res, _args) in {
+    "kvr_decode_attend_workspace_bytes": (ctypes.c_size_t, [_P, _I, _I, _I]),
+    "kvr_decode_attend": (_S, [_P, _I, _I, _P, _P, _P, _P, _I, _P,
+                               ctypes.c_size_t, _P]),
+}.items():
+    _f = getattr(lib, _name)
+    _f.restype = _res
+    _f.argtypes = _args
+
+
+def kvr_decode_attend_workspace_bytes(h, layer_begin, layer_end, n_splits=0):
+    return int(lib.kvr_decode_attend_workspace_bytes(h, layer_begin, layer_end,
+                                                     n_splits))
+
+
+def kvr_decode_attend(h, layer_begin, layer_end, q, k_new, v_new, out,
+                      n_splits, workspace, workspace_bytes, stream=None):
+    _check(lib.kvr_decode_attend(h, layer_begin, layer_end, _ptr(q),
+                                 _ptr(k_new), _ptr(v_new), _ptr(out), n_splits,
+                                 _ptr(workspace), workspace_bytes,
+                                 _stream(stream)), "kvr_decode_attend")
+
+
+def attend_full(cache: Cache, q, k_new, v_new, out=None, layers=None,
+                n_splits=0, workspace=None, stream=None):
+    """Full-context decode step on `cache` (no scores, no eviction)."""
+    lb, le = (0, cache.L) if layers is None else layers
+    out = cache.new_out(le - lb) if out is None else out
+    need = kvr_decode_attend_workspace_bytes(cache.handle, lb, le, n_splits)
+    if workspace is None:
+        workspace = torch.empty(max(need, 16), dtype=torch.uint8,
+                                device=cache.buf.device)
+    kvr_decode_attend(cache.handle, lb, le, q, k_new, v_new, out, n_splits,
+                      workspace, workspace.numel(), stream)
+    return out
