@@ -58,6 +58,12 @@ def parse():
     p.add_argument("--fused-groups", type=int, default=0,
                    help="units computed at once per SM by the fused kernel "
                         "(0: the library's choice)")
+    p.add_argument("--mode", default="step", choices=["step", "helper", "fork"],
+                   help="step: the evicted decode step (the headline); "
+                        "helper: full-context decode of the 1.5B helper at "
+                        "16k context; fork: 72B best-of-8 candidate step")
+    p.add_argument("--seqs", type=int, default=0,
+                   help="sequences for --mode helper/fork (0: 16 / 4)")
     p.add_argument("--fused-group-warps", type=int, default=0,
                    help="warps sharing one unit in the fused kernel "
                         "(0: the library's choice)")
@@ -313,6 +319,160 @@ def run_kvr(args, rank, world, local_rank):
                 launches=launches)
 
 
+# --------------------------------------------------------------------------
+# other rows of the path: full-context helper decode, candidate steps
+# --------------------------------------------------------------------------
+
+def _timed(fn, K, stream):
+    import torch
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
+    torch.cuda.synchronize()
+    for i in range(K):
+        starts[i].record(stream)
+        fn(i)
+        ends[i].record(stream)
+    torch.cuda.synchronize()
+    total = starts[0].elapsed_time(ends[-1])
+    per = sum(a.elapsed_time(b) for a, b in zip(starts, ends)) / K
+    return total, per
+
+
+def run_helper(args):
+    """1.5B helper geometry (28 layers, 12 q / 2 kv heads, d 128) at context
+    16384: append + attention over every row, no scores, no eviction."""
+    import torch
+    from paper_2608_15797_gb300 import kvr
+    w = inputs.WORKLOADS["1p5b_full16k"]
+    S = args.seqs or 16
+    L, H, G, d, ctx = w.n_layers, w.n_kv_heads, w.group, w.head_dim, w.prompt
+    K, Wm = args.steps, args.warmup
+    dev = torch.device("cuda", 0)
+    cache = kvr.Cache(S, L, H, G, d, ctx + K + Wm + 1, "bf16", "bf16", device=dev)
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(args.seed + 17)
+    for s in range(S):
+        k = (torch.randn(L, H, ctx, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+        v = (torch.randn(L, H, ctx, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+        cache.load(s, k, v)
+        del k, v
+    q = (torch.randn(S, L, H * G, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+    kn = (torch.randn(S, L, H, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+    vn = (torch.randn(S, L, H, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+    out = cache.new_out(L)
+    need = kvr.kvr_decode_attend_workspace_bytes(cache.handle, 0, L, 0)
+    ws = torch.empty(need, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step(i):
+        kvr.kvr_decode_attend(cache.handle, 0, L, q, kn, vn, out, 0, ws,
+                              ws.numel(), stream)
+
+    for i in range(Wm):
+        step(i)
+    n0 = cache.launch_count()
+    total, per = _timed(step, K, stream)
+    launches = cache.launch_count() - n0
+    cache.sync_status()
+    m_mean = ctx + Wm + (K - 1) / 2.0  # rows before the append, mean over steps
+    per_unit = cost_model.attend_full_unit_bytes(m_mean, d, G, 2, 2)
+    launch_bytes = per_unit * S * L * H
+    return dict(metric=f"full-context helper decode steps/s (1.5B geometry, "
+                       f"context {ctx}, {S} sequences x {L} layers per step)",
+                total_ms=total, per_ms=per, K=K, launches=launches,
+                launch_bytes=launch_bytes,
+                config={"workload": "1p5b_full16k", "n_seq": S, "layers": L,
+                        "kv_heads": H, "group": G, "head_dim": d,
+                        "context": ctx, "splits": "auto"},
+                kernel="kvr_decode_attend (split partials + combine)")
+
+
+def run_fork(args):
+    """72B geometry (80 layers, 64 q / 8 kv heads, d 128), B=64, W=8: an
+    evicted parent (B+W rows) forked to 8 candidates; one timed step is one
+    candidate token for all 8 candidates, all layers, all sequences; the 64
+    tokens of a reasoning step are followed by a commit (timed apart)."""
+    import torch
+    from paper_2608_15797_gb300 import kvr
+    w = inputs.WORKLOADS["72b_bon8"]
+    S = args.seqs or 4
+    L, H, G, d, N = w.n_layers, w.n_kv_heads, w.group, w.head_dim, w.n_cand
+    B, Wn, T = w.budget, w.window, w.cand_step
+    dev = torch.device("cuda", 0)
+    cache = kvr.Cache(S, L, H, G, d, B + Wn + T + 1, "bf16", "bf16", device=dev)
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(args.seed + 29)
+    for s in range(S):
+        k = (torch.randn(L, H, B + Wn, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+        v = (torch.randn(L, H, B + Wn, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+        cache.load(s, k, v)
+    q = (torch.randn(N, S, L, H * G, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+    kn = (torch.randn(N, S, L, H, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+    vn = (torch.randn(N, S, L, H, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+    out = torch.empty(N, S, L, H * G, d, dtype=torch.bfloat16, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    chosen = np.zeros(S, np.int32)
+    K = max(1, min(args.steps, 64 * 50))
+    tok_ms, commit_ms, bytes_tok, launches = [], [], 0.0, 0
+    n0 = cache.launch_count()
+    done = 0
+    warm = True
+    while done < K:
+        f = kvr.Fork(cache, N, T)
+        steps_here = T
+        def step(i):
+            kvr.kvr_fork_decode_attend_score(f.handle, 0, L, q, kn, vn, out, stream)
+        tot, per = _timed(step, steps_here, stream)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        f.commit(chosen, B, Wn)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        if warm:
+            warm = False
+            n0 = cache.launch_count()
+            continue
+        tok_ms.append(per)
+        commit_ms.append(e0.elapsed_time(e1))
+        done += steps_here
+    cache.sync_status()
+    launches = cache.launch_count() - n0
+    # algorithmic bytes of one candidate token (mean tail length T/2)
+    np_rows, nt = B + Wn, (T - 1) / 2.0
+    per_unit = (2 * np_rows * d * 2 + N * (2 * nt * d * 2 + 4 * d * 2 + 2 * G * d * 2
+                                          + 8 * np_rows + 8 * (nt + 1) + 4))
+    return dict(metric=f"72B best-of-{N} candidate tokens/s (B={B}, W={Wn}, "
+                       f"{S} sequences x {L} layers x {N} candidates per token)",
+                total_ms=float(np.mean(tok_ms)) * done, per_ms=float(np.mean(tok_ms)),
+                K=done, launches=launches, launch_bytes=per_unit * S * L * H,
+                commit_ms=float(np.mean(commit_ms)),
+                config={"workload": "72b_bon8", "n_seq": S, "layers": L,
+                        "kv_heads": H, "group": G, "head_dim": d, "n_cand": N,
+                        "budget": B, "window": Wn, "cand_step": T},
+                kernel="kvr_fork_decode_attend_score")
+
+
+def print_row_line(args, r):
+    peaks, peak_kind = measured_peaks()
+    peak = float(peaks["hbm_gbs"])
+    achieved = r["launch_bytes"] / (r["per_ms"] / 1e3) / 1e9
+    line = {"metric": r["metric"], "value": r["K"] / (r["total_ms"] / 1e3),
+            "unit": "steps/s", "n_gpus": 1, "steps": r["K"],
+            "warmup": args.warmup, "ms_per_step": r["total_ms"] / r["K"],
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16", "data": "synthetic", "config": r["config"],
+            "hbm_gbs": achieved,
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak,
+                         "unit": "GB/s", "frac": achieved / peak,
+                         "peak_kind": peak_kind, "traffic": None,
+                         "algorithmic_bytes_per_launch": r["launch_bytes"],
+                         "launch_ms": r["per_ms"], "kernel": r["kernel"]},
+            "gpu_launches": r["launches"]}
+    if "commit_ms" in r:
+        line["commit_ms"] = r["commit_ms"]
+    print(json.dumps(line))
+
+
 def main():
     args = parse()
     w = inputs.WORKLOADS[args.workload]
@@ -348,6 +508,11 @@ def main():
         return 0
 
     import torch
+    if args.mode != "step":
+        if rank == 0:
+            r = run_helper(args) if args.mode == "helper" else run_fork(args)
+            print_row_line(args, r)
+        return 0
     if world > 1:
         torch.distributed.init_process_group("nccl")
     r = run_kvr(args, rank, world, local_rank)
