@@ -312,6 +312,42 @@ bool try_fused(kvr_cache *c, const StepArgs &a, bool evict, int budget,
   return true;
 }
 
+// Launch the streaming fused step (longer units) if this call qualifies.
+bool try_stream(kvr_cache *c, const StepArgs &a, bool evict, int budget,
+                int window, cudaStream_t stream, cudaError_t *err) {
+  const CacheView &v = c->view;
+  if (!c->fused || !v.kv_bf16 || v.d != 128 || v.G > 8) return false;
+  if (a.max_rows > kvr::stream_max_rows()) return false;
+  if (evict && (long long)a.max_rows > (long long)budget + window + 1)
+    return false;
+  const size_t rows = (size_t)v.S * v.L * v.H * v.cap;
+  if (rows >= (size_t)INT32_MAX) return false;
+  if (!aligned16(a.q) || !aligned16(a.k_new) || !aligned16(a.v_new) ||
+      !aligned16(a.out))
+    return false;
+  if (!device_facts(c)) return false;
+  if (kvr::stream_smem_bytes(a.max_rows) + 512 > (size_t)c->smem_optin)
+    return false;
+  const std::pair<CUtensorMap, CUtensorMap> *maps =
+      slab_maps(c, kvr::stream_box_rows());
+  if (!maps) return false;
+  kvr::StreamParams p{};
+  p.c = v;
+  p.q = static_cast<const __nv_bfloat16 *>(a.q);
+  p.k_new = static_cast<const __nv_bfloat16 *>(a.k_new);
+  p.v_new = static_cast<const __nv_bfloat16 *>(a.v_new);
+  p.out = a.out;
+  p.lb = a.lb;
+  p.nl = a.nl;
+  p.n_max = a.max_rows;
+  p.budget = budget;
+  p.window = window;
+  p.evict = evict ? 1 : 0;
+  p.scale_log2e = v.scale * 1.4426950408889634f;
+  *err = kvr::launch_stream_step(maps->first, maps->second, p, stream);
+  return true;
+}
+
 // Splits for kvr_decode_attend: about two waves of the partial kernel (three
 // CTAs per SM), never less than 256 rows per split.
 int auto_splits(const kvr_cache *c, int lb, int le) {
@@ -472,7 +508,8 @@ kvr_status kvr_decode_attend_score(kvr_cache *c, int lb, int le, const void *q,
   if (st != KVR_OK) return st;
   StepArgs a = step_args(c, lb, le, q, k_new, v_new, out);
   cudaError_t e = cudaSuccess;
-  if (!try_fused(c, a, false, 0, 0, as_stream(stream), &e))
+  if (!try_fused(c, a, false, 0, 0, as_stream(stream), &e) &&
+      !try_stream(c, a, false, 0, 0, as_stream(stream), &e))
     e = kvr::launch_attend_score_generic(c->view, a, as_stream(stream));
   if (e != cudaSuccess) return cuda_fail("kvr_decode_attend_score", e);
   c->launches += 1;
@@ -559,7 +596,8 @@ kvr_status kvr_decode_step(kvr_cache *c, int lb, int le, const void *q,
   if (st != KVR_OK) return st;
   StepArgs a = step_args(c, lb, le, q, k_new, v_new, out);
   cudaError_t e = cudaSuccess;
-  if (try_fused(c, a, true, budget, window, as_stream(stream), &e)) {
+  if (try_fused(c, a, true, budget, window, as_stream(stream), &e) ||
+      try_stream(c, a, true, budget, window, as_stream(stream), &e)) {
     if (e != cudaSuccess) return cuda_fail("kvr_decode_step", e);
     c->launches += 1;
     mirror_append(c, lb, le);

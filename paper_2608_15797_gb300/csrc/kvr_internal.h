@@ -89,6 +89,23 @@ cudaError_t launch_fused_step(const CUtensorMap &tmK, const CUtensorMap &tmV,
                               const FusedParams &p, int grid, int smem_bytes,
                               cudaStream_t st);
 
+// Fused step for longer units (kvr_stream.cu): bf16, d = 128, G <= 8, at
+// most stream_max_rows() rows after the append, at most one eviction.
+struct StreamParams {
+  CacheView c;
+  const __nv_bfloat16 *q, *k_new, *v_new;
+  void *out;
+  int lb, nl;
+  int n_max;                   // largest live length after the append
+  int budget, window, evict;
+  float scale_log2e;
+};
+int stream_box_rows();
+int stream_max_rows();
+size_t stream_smem_bytes(int n_max);
+cudaError_t launch_stream_step(const CUtensorMap &tmK, const CUtensorMap &tmV,
+                               const StreamParams &p, cudaStream_t st);
+
 // Full-context decode split over the rows (kvr_split.cu): bf16, d = 128,
 // G <= 8.  ws holds [units of the call][n_splits][G][130] floats.
 struct SplitParams {

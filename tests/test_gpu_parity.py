@@ -178,3 +178,26 @@ def test_capacity_and_argument_errors():
     c.evict(2, 1)
     assert c.lengths().tolist() == [[3]]
     c.sync_status()
+
+
+@pytest.mark.parametrize("B,G,out", [(128, 7, "bf16"), (256, 7, "f32"),
+                                     (512, 8, "bf16"), (150, 1, "f32")])
+def test_long_unit_fused_step(B, G, out):
+    """Budgets above the staged kernel's 128 rows (the throughput sweep's
+    B = 128 / 256 / 512, W = 8): the streaming fused kernel, one launch per
+    step, in lock-step with the oracle from B + W rows on."""
+    W = 8
+    w = inputs.Workload("long_b", 2, 2, G, 128, "bf16", B, W, B + W, 5, sigma=1.0)
+    c, o = harness.make_pair(w, 13, 2, cap=B + W + 1,
+                             prompt_lens=[B + W, B + W - 37], out_dtype=out)
+    n0 = c.launch_count()
+    harness.lockstep(c, o, w, 13, 5, B, W)
+    assert c.launch_count() - n0 == 5
+
+
+def test_long_unit_growth_without_eviction():
+    """Units growing from 100 to 300 rows with no eviction: the staged kernel
+    while they fit, then the streaming kernel."""
+    w = inputs.Workload("grow", 1, 2, 4, 128, "bf16", 1 << 20, 0, 0, 40, sigma=1.0)
+    c, o = harness.make_pair(w, 14, 2, cap=400, prompt_lens=[100, 290])
+    harness.lockstep(c, o, w, 14, 40, w.budget, w.window)
