@@ -699,6 +699,8 @@ struct kvr_fork {
   std::vector<int32_t> tlen;  // host mirror [S][L] (same for all candidates)
   int32_t *chosen_dev;        // [S]
   bool spent = false;
+  bool tail_maps = false;     // TK / TV tensor maps encoded (tensor-core path)
+  CUtensorMap tmTK, tmTV;
 };
 
 namespace {
@@ -799,6 +801,13 @@ kvr_status kvr_fork_candidates(kvr_cache *p, int n_cand, int tail_cap,
     delete f;
     return cuda_fail("kvr_fork_candidates", e);
   }
+  if (p->view.kv_bf16 && p->view.d == 128 &&
+      (size_t)n_cand * units * tail_cap < (size_t)INT32_MAX) {
+    const size_t trows = (size_t)n_cand * units * tail_cap;
+    f->tail_maps =
+        encode_slab(&f->tmTK, v.TK, trows, kvr::fork_mma_box_rows()) &&
+        encode_slab(&f->tmTV, v.TV, trows, kvr::fork_mma_box_rows());
+  }
   p->forks += 1;
   *out = f;
   return KVR_OK;
@@ -839,8 +848,39 @@ kvr_status kvr_fork_decode_attend_score(kvr_fork *f, int lb, int le,
   a.v_new = v_new;
   a.out = out;
   a.max_rows = n_max;
-  cudaError_t e =
-      kvr::launch_fork_attend(f->view, a, n_max, max_prefix, as_stream(stream));
+  cudaError_t e = cudaSuccess;
+  int nt_max = 0;
+  for (int s = 0; s < p->desc.n_seq; ++s)
+    for (int l = lb; l < le; ++l)
+      nt_max = std::max(nt_max, f->tlen[(size_t)s * p->desc.n_layers + l]);
+  const CacheView &pv = p->view;
+  const std::pair<CUtensorMap, CUtensorMap> *maps = nullptr;
+  const bool mma_ok =
+      p->fused && f->tail_maps && pv.G <= 8 &&
+      f->view.N <= kvr::fork_mma_max_cand() && device_facts(p) &&
+      kvr::fork_mma_smem_bytes(max_prefix, nt_max, f->view.N) + 512 <=
+          (size_t)p->smem_optin &&
+      (size_t)pv.S * pv.L * pv.H * pv.cap < (size_t)INT32_MAX &&
+      aligned16(q) && aligned16(k_new) && aligned16(v_new) && aligned16(out) &&
+      (maps = slab_maps(p, kvr::fork_mma_box_rows())) != nullptr;
+  if (mma_ok) {
+    kvr::ForkMmaParams mp{};
+    mp.f = f->view;
+    mp.q = static_cast<const __nv_bfloat16 *>(q);
+    mp.k_new = static_cast<const __nv_bfloat16 *>(k_new);
+    mp.v_new = static_cast<const __nv_bfloat16 *>(v_new);
+    mp.out = out;
+    mp.lb = lb;
+    mp.nl = le - lb;
+    mp.np_max = max_prefix;
+    mp.nt_max = nt_max;
+    mp.scale_log2e = pv.scale * 1.4426950408889634f;
+    e = kvr::launch_fork_mma(maps->first, maps->second, f->tmTK, f->tmTV, mp,
+                             as_stream(stream));
+  } else {
+    e = kvr::launch_fork_attend(f->view, a, n_max, max_prefix,
+                                as_stream(stream));
+  }
   if (e != cudaSuccess) return cuda_fail("kvr_fork_decode_attend_score", e);
   p->launches += 1;
   for (int s = 0; s < p->desc.n_seq; ++s)

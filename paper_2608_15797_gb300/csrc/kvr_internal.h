@@ -134,6 +134,24 @@ struct ForkView {
   int32_t *tlen;     // [N][units]
 };
 size_t fork_attend_smem_bytes(const CacheView &c, int n_max, int max_prefix);
+
+// Candidate step on tensor cores (kvr_fork_mma.cu): bf16, d = 128, G <= 8,
+// N <= fork_mma_max_cand(); one CTA per unit, one warp per candidate.
+struct ForkMmaParams {
+  ForkView f;
+  const __nv_bfloat16 *q, *k_new, *v_new;  // [N][S][nl][...][128]
+  void *out;
+  int lb, nl;
+  int np_max;   // longest prefix over the call's units
+  int nt_max;   // longest tail (before the append) over the call's units
+  float scale_log2e;
+};
+size_t fork_mma_smem_bytes(int np_max, int nt_max, int n_cand);
+int fork_mma_box_rows();
+int fork_mma_max_cand();
+cudaError_t launch_fork_mma(const CUtensorMap &tmK, const CUtensorMap &tmV,
+                            const CUtensorMap &tmTK, const CUtensorMap &tmTV,
+                            const ForkMmaParams &p, cudaStream_t st);
 cudaError_t launch_fork_attend(const ForkView &f, const StepArgs &a, int n_max,
                                int max_prefix, cudaStream_t st);
 cudaError_t launch_fork_commit(const ForkView &f, const int32_t *chosen,

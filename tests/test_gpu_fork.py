@@ -24,18 +24,25 @@ def _cuda():
     torch.cuda.set_device(0)
 
 
-def _evicted_pair(w, seed, S, cap, prompt_lens, warm_steps):
-    """Load prompts and run evicting steps so the parent sits at B + W rows."""
-    c, o = harness.make_pair(w, seed, S, cap=cap, prompt_lens=prompt_lens)
+def _evicted_pair(w, seed, S, cap, prompt_lens, warm_steps, fused=True):
+    """Load prompts and run evicting steps so the parent sits at B + W rows.
+    fused=False keeps the parent (and its forks) on the generic kernels."""
+    c, o = harness.make_pair(w, seed, S, cap=cap, prompt_lens=prompt_lens,
+                             fused=fused)
     harness.lockstep(c, o, w, seed, warm_steps, w.budget, w.window)
     return c, o
 
 
-@pytest.mark.parametrize("n_cand", [1, 3])
-def test_small_fork_commit_then_continue(n_cand):
+@pytest.mark.parametrize("fused", [True, False])
+@pytest.mark.parametrize("n_cand", [1, 3, 8])
+def test_small_fork_commit_then_continue(n_cand, fused):
+    """Tail lengths cross the 16-row tile boundary (7 tokens from a ragged
+    parent, 19 for N = 8)."""
     w = inputs.Workload("f", 2, 2, 3, 128, "bf16", 12, 4, 30, 0, sigma=1.0)
-    c, o = _evicted_pair(w, 21, 2, cap=40, prompt_lens=[30, 9], warm_steps=3)
-    o2, chosen, st = harness.fork_lockstep(c, o, w, 21, n_cand, 7, w.budget,
+    c, o = _evicted_pair(w, 21, 2, cap=40, prompt_lens=[30, 9], warm_steps=3,
+                         fused=fused)
+    o2, chosen, st = harness.fork_lockstep(c, o, w, 21, n_cand,
+                                           19 if n_cand == 8 else 7, w.budget,
                                            w.window)
     assert (c.lengths() == np.minimum(o2.len.max(axis=2), 16)).all()
     # the committed parent keeps decoding in lock-step
