@@ -282,7 +282,8 @@ bool try_fused(kvr_cache *c, const StepArgs &a, bool evict, int budget,
   if (U < 1 || n_stages < 2) return false;
   // Keep two stages loading while the others are computed (measured best).
   int n_groups = std::min({4, std::max(1, n_stages - 2),
-                           (kvr::fused_max_threads() / 32 - 1) / U});
+                           (kvr::fused_max_threads() / 32 -
+                            kvr::fused_producer_warps()) / U});
   if (c->fused_groups > 0) n_groups = std::min(n_groups, c->fused_groups);
   if (n_groups < 1) return false;
   const std::pair<CUtensorMap, CUtensorMap> *maps = slab_maps(c, Rb);

@@ -40,7 +40,8 @@ using namespace ptx;
 constexpr int kMaxStages = 8;
 constexpr int kMaxGroups = 4;      // units in flight on the consumer side
 constexpr int kMaxGroupWarps = 8;  // warps sharing one unit
-constexpr int kMaxThreads = 544;   // 16 consumer warps + the producer
+constexpr int kProducers = 2;      // TMA-issuing warps
+constexpr int kMaxThreads = 576;   // 16 consumer warps + the producers
 constexpr int kXsWords = 20;       // exchange words per warp of a group
 constexpr int kQPitch = 272;  // bytes per staged query row (256 + 16 padding)
 
@@ -159,10 +160,16 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
   fence_proxy_async();
   __syncthreads();
 
-  if (warp == consumers) {
+  if (warp >= consumers) {
+    // Producers: warp `consumers + j` owns the stages s with s % kProducers
+    // == j, so every stage is refilled by one thread, round after round (two
+    // threads on one stage could run a full ring ahead and alias the
+    // mbarrier parity).
+    const int j = warp - consumers;
     if (lane == 0) {
       for (int k = 0; k < mine; ++k) {
         const int s = k % p.n_stages;
+        if (s % kProducers != j) continue;
         const uint32_t ph = (uint32_t)(k / p.n_stages) & 1u;
         if (!mbar_wait(smem_u32(&empty_bar[s]), ph ^ 1u, &s_abort)) {
           atomicOr(p.c.err, ERR_TIMEOUT);
@@ -226,7 +233,7 @@ cudaError_t launch_tu(const CUtensorMap &tmK, const CUtensorMap &tmV,
   cudaError_t e = cudaFuncSetAttribute(
       kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
   if (e != cudaSuccess) return e;
-  const int threads = 32 * (p.n_groups * U + 1);
+  const int threads = 32 * (p.n_groups * U + kProducers);
   kern<<<grid, threads, smem_bytes, st>>>(tmK, tmV, p);
   return cudaGetLastError();
 }
@@ -263,13 +270,14 @@ int fused_group_warps(int R, int requested) {
 }
 
 int fused_max_threads() { return kMaxThreads; }
+int fused_producer_warps() { return kProducers; }
 
 cudaError_t launch_fused_step(const CUtensorMap &tmK, const CUtensorMap &tmV,
                               const FusedParams &p, int grid, int smem_bytes,
                               cudaStream_t st) {
   if (fused_group_warps(p.R, p.group_warps) != p.group_warps ||
       p.n_groups < 1 || p.n_groups > kMaxGroups || p.n_stages > kMaxStages ||
-      32 * (p.n_groups * p.group_warps + 1) > kMaxThreads)
+      32 * (p.n_groups * p.group_warps + kProducers) > kMaxThreads)
     return cudaErrorInvalidValue;
   return p.c.out_bf16 ? launch_t<true>(tmK, tmV, p, grid, smem_bytes, st)
                       : launch_t<false>(tmK, tmV, p, grid, smem_bytes, st);

@@ -85,6 +85,7 @@ int fused_stage_bytes(int R);
 // the supported choices (one or two row tiles per warp), else the default.
 int fused_group_warps(int R, int requested);
 int fused_max_threads();
+int fused_producer_warps();
 cudaError_t launch_fused_step(const CUtensorMap &tmK, const CUtensorMap &tmV,
                               const FusedParams &p, int grid, int smem_bytes,
                               cudaStream_t st);
