@@ -23,6 +23,13 @@
 //    evicted (warp argmin of the (score, -position) key over non-window
 //    rows) and the new row is written straight into the freed slot: the
 //    compaction moves no other row.
+//  - Units go to the groups round-robin, so when the ring depth is not a
+//    multiple of the group count, one stage's consecutive units belong to
+//    different groups and a group can reach a stage's next unit before the
+//    previous one has landed.  A parity wait cannot tell those two phases
+//    apart, so a group first waits until the producer has recorded the unit
+//    as issued (which implies the earlier phase completed) and only then on
+//    the stage's full barrier.
 //  - Every wait on an mbarrier is bounded (about 2 s); on timeout the kernel
 //    sets ERR_TIMEOUT in the device error word and drains its own copies.
 #include <cuda.h>
@@ -118,6 +125,17 @@ __device__ void issue_unit(const FusedParams &p, const CUtensorMap *tmK,
 
 #include "kvr_fused_unit.cuh"
 
+// Bounded wait until the producer has recorded unit k (or a later one) as
+// issued into this stage; false on timeout or abort.
+__device__ bool wait_issued(volatile int *issued, int k, volatile int *abort) {
+  if (*issued >= k) return true;
+  const uint64_t t0 = global_ns();
+  while (*issued < k) {
+    if (*abort || global_ns() - t0 > kWaitNs) return false;
+  }
+  return true;
+}
+
 template <int T, int U, bool kOutBf16>
 __global__ void __launch_bounds__(kMaxThreads, 1)
     fused_step_kernel(const __grid_constant__ CUtensorMap tmK,
@@ -126,7 +144,7 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
   extern __shared__ unsigned char smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[kMaxStages];
   __shared__ __align__(8) uint64_t empty_bar[kMaxStages];
-  __shared__ int issued_k[kMaxStages];
+  __shared__ volatile int issued_k[kMaxStages];
   __shared__ int consumed_k[kMaxStages];
   __shared__ volatile int s_abort;
   __shared__ volatile int s_ok[kMaxGroups];
@@ -189,7 +207,8 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
       // One warp waits (bounded) and tells the group, so that every warp
       // of the group takes the same branch before the next named barrier.
       if (w == 0) {
-        const bool ok = mbar_wait(smem_u32(&full_bar[s]), ph, &s_abort);
+        const bool ok = wait_issued(&issued_k[s], k, &s_abort) &&
+                        mbar_wait(smem_u32(&full_bar[s]), ph, &s_abort);
         if (lane == 0) {
           s_ok[grp] = ok ? 1 : 0;
           if (!ok) {
