@@ -276,16 +276,24 @@ bool try_fused(kvr_cache *c, const StepArgs &a, bool evict, int budget,
   const int R = kvr::round_up16(a.max_rows);
   const int Rb = std::max(8, (a.max_rows - 1 + 7) / 8 * 8);
   const int U = kvr::fused_group_warps(R, c->fused_group_warps);
+  if (U < 1) return false;
   const int stage = kvr::fused_stage_bytes(R);
+  const int gbytes = kvr::fused_group_bytes(U);
   const int avail = c->smem_optin - 1024 /*alignment*/ - 512 /*static*/;
-  const int n_stages = std::min(8, avail / stage);
-  if (U < 1 || n_stages < 2) return false;
-  // Keep two stages loading while the others are computed (measured best).
-  int n_groups = std::min({4, std::max(1, n_stages - 2),
-                           (kvr::fused_max_threads() / 32 -
-                            kvr::fused_producer_warps()) / U});
-  if (c->fused_groups > 0) n_groups = std::min(n_groups, c->fused_groups);
-  if (n_groups < 1) return false;
+  // Consumer groups hold a stage only while reading it; the rest of shared
+  // memory is ring.  By default as many groups as there are stages (at most
+  // four; measured best), a tuned count as long as two stages remain.
+  const int max_groups = std::min(kvr::fused_max_groups(),
+                                  (kvr::fused_max_threads() / 32 -
+                                   kvr::fused_producer_warps()) / U);
+  const bool tuned = c->fused_groups > 0;
+  int n_groups = std::min(max_groups, tuned ? c->fused_groups : 4);
+  int n_stages = 0;
+  for (; n_groups >= 1; --n_groups) {
+    n_stages = std::min(8, (avail - n_groups * gbytes) / stage);
+    if (n_stages >= (tuned ? 2 : std::max(2, n_groups))) break;
+  }
+  if (n_groups < 1 || n_stages < 2) return false;
   const std::pair<CUtensorMap, CUtensorMap> *maps = slab_maps(c, Rb);
   if (!maps) return false;
   kvr::FusedParams p{};
@@ -309,7 +317,8 @@ bool try_fused(kvr_cache *c, const StepArgs &a, bool evict, int budget,
   const int units = v.S * a.nl * v.H;
   const int grid = std::min(c->sm_count, units);
   *err = kvr::launch_fused_step(maps->first, maps->second, p, grid,
-                                n_stages * stage + 1024, stream);
+                                n_stages * stage + n_groups * gbytes + 1024,
+                                stream);
   return true;
 }
 

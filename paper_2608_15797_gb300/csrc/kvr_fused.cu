@@ -6,12 +6,16 @@
 //
 // Design (GB300, sm_103a):
 //  - Persistent CTAs, one per SM.  Each CTA owns a ring of shared-memory
-//    stages; a producer warp fills a stage with one unit's K and V (two
+//    stages; two producer warps fill a stage with one unit's K and V (two
 //    128B-swizzled TMA boxes each: columns 0-63 and 64-127, all rows of the
-//    unit), its G query rows, the new k/v row, scores, positions and state,
-//    all completing on the stage's mbarrier.  Consumer groups of U warps
+//    unit), completing on the stage's mbarrier.  Consumer groups of U warps
 //    each take whole units; within a group every warp owns one or two
 //    16-row tiles of the unit (kvr_fused_unit.cuh).
+//  - The small per-unit inputs (the G query rows, the new k/v row, scores,
+//    positions and state) are fetched by the producer warp's 32 lanes with
+//    16-byte cp.async copies that arrive on the same mbarrier, so a stage
+//    costs the TMA unit only its four K/V boxes and the query rows land at
+//    a padded pitch that keeps the ldmatrix reads free of bank conflicts.
 //  - QK^T and PV run on warp-level bf16 tensor-core MMAs (m16n8k16, fp32
 //    accumulate): K rows are the M side, the <= 8 query heads of the group
 //    the N side.  The probability tile leaves the QK accumulators in
@@ -46,19 +50,18 @@ using namespace ptx;
 
 constexpr int kMaxStages = 8;
 constexpr int kMaxGroups = 4;      // units in flight on the consumer side
-constexpr int kMaxGroupWarps = 8;  // warps sharing one unit
 constexpr int kProducers = 2;      // TMA-issuing warps
-constexpr int kMaxThreads = 576;   // 16 consumer warps + the producers
-constexpr int kXsWords = 20;       // exchange words per warp of a group
+constexpr int kMaxThreads = 512;   // consumer warps + the producers
 constexpr int kQPitch = 272;  // bytes per staged query row (256 + 16 padding)
 
 __device__ __forceinline__ void group_bar(int id, int threads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
 }
 
-// Byte offsets inside one stage of R staged rows.
+// Byte offsets inside one stage of R staged rows (R a multiple of 16, so
+// every box starts on a 1024-byte boundary as the 128B swizzle needs).
 struct StageLayout {
-  uint32_t k0, k1, v0, v1, q, kn, vn, sc, ps, st, xs, info, bytes;
+  uint32_t k0, k1, v0, v1, q, kn, vn, sc, ps, st, bytes;
   __host__ __device__ explicit StageLayout(int R) {
     k0 = 0;
     k1 = k0 + R * 128;
@@ -70,57 +73,79 @@ struct StageLayout {
     sc = vn + 256;
     ps = sc + 4 * R;
     st = ps + 4 * R;
-    xs = st + 16;  // group exchange: kXsWords words per warp
-    info = xs + 4 * kXsWords * kMaxGroupWarps;  // cache unit, input row
-    bytes = ((info + 16) + 1023) / 1024 * 1024;
+    bytes = ((st + 16) + 1023) / 1024 * 1024;
   }
 };
 
+// Byte offsets inside one consumer group's private exchange area (after the
+// ring): five 16-byte slots per warp, then the warps' partial outputs
+// ([warp][8 head-dim tiles][32 lanes] float4).  A one-warp group needs none.
+struct GroupLayout {
+  uint32_t xs, ox, bytes;
+  __host__ __device__ explicit GroupLayout(int U) {
+    xs = 0;
+    ox = (U * 5 * 16 + 127) / 128 * 128;
+    bytes = U > 1 ? ox + U * 8 * 32 * 16 : 0;
+  }
+};
+
+// Cache unit and input row of the launch's unit idx (sequence-major, then
+// layer, then KV head).
 struct UnitIdx {
-  int h, lr, sq;
   size_t ug;    // cache unit
   size_t krow;  // row of this unit in the call's [S][nl][H] inputs
 };
 
 __device__ __forceinline__ UnitIdx unit_idx(const FusedParams &p, int idx) {
+  const int h = idx % p.c.H;
+  const int lr = (idx / p.c.H) % p.nl;
+  const int sq = idx / (p.c.H * p.nl);
   UnitIdx x;
-  x.h = idx % p.c.H;
-  x.lr = (idx / p.c.H) % p.nl;
-  x.sq = idx / (p.c.H * p.nl);
-  x.ug = ((size_t)x.sq * p.c.L + p.lb + x.lr) * p.c.H + x.h;
-  x.krow = ((size_t)x.sq * p.nl + x.lr) * p.c.H + x.h;
+  x.ug = ((size_t)sq * p.c.L + p.lb + lr) * p.c.H + h;
+  x.krow = ((size_t)sq * p.nl + lr) * p.c.H + h;
   return x;
 }
 
-// Producer: enqueue every copy of one unit into a stage.  K and V come as
-// two 128B-swizzled boxes of Rb rows each (columns 0-63, 64-127).
-__device__ void issue_unit(const FusedParams &p, const CUtensorMap *tmK,
-                           const CUtensorMap *tmV, unsigned char *stage,
-                           uint32_t bar, int idx) {
+// Producer warp: enqueue one unit into a stage.  Lane 0 issues K and V as
+// two 128B-swizzled TMA boxes of Rb rows each (columns 0-63, 64-127); all
+// 32 lanes copy the small inputs in 16-byte pieces and arrive when theirs
+// have landed (the full barrier expects 1 + 32 arrivals).
+__device__ __forceinline__ void issue_unit(const FusedParams &p,
+                                           const CUtensorMap *tmK,
+                                           const CUtensorMap *tmV,
+                                           unsigned char *stage, uint32_t bar,
+                                           int idx, int lane) {
   const StageLayout L(p.R);
   const UnitIdx x = unit_idx(p, idx);
-  const int G = p.c.G;
   const uint32_t s0 = smem_u32(stage);
-  const uint32_t tx = 4u * p.Rb * 128u + (uint32_t)G * 256u + 512u +
-                      8u * p.Rb + 16u;
-  // The unit's indices for the consumers (released by the arrive below).
-  uint32_t *info = reinterpret_cast<uint32_t *>(stage + L.info);
-  info[0] = (uint32_t)x.ug;
-  info[1] = (uint32_t)x.krow;
-  mbar_expect_tx(bar, tx);
-  const int row0 = (int)(x.ug * (size_t)p.c.cap);
-  tma_load_2d(s0 + L.k0, tmK, 0, row0, bar);
-  tma_load_2d(s0 + L.k1, tmK, 64, row0, bar);
-  tma_load_2d(s0 + L.v0, tmV, 0, row0, bar);
-  tma_load_2d(s0 + L.v1, tmV, 64, row0, bar);
-  const __nv_bfloat16 *q = p.q + x.krow * G * 128;
-  for (int g = 0; g < G; ++g)
-    bulk_load(s0 + L.q + g * kQPitch, q + g * 128, 256, bar);
-  bulk_load(s0 + L.kn, p.k_new + x.krow * 128, 256, bar);
-  bulk_load(s0 + L.vn, p.v_new + x.krow * 128, 256, bar);
-  bulk_load(s0 + L.sc, p.c.score + x.ug * p.c.sstride, 4u * p.Rb, bar);
-  bulk_load(s0 + L.ps, p.c.pos + x.ug * p.c.sstride, 4u * p.Rb, bar);
-  bulk_load(s0 + L.st, p.c.state + x.ug * 4, 16, bar);
+  if (lane == 0) {
+    mbar_expect_tx(bar, 4u * p.Rb * 128u);
+    const int row0 = (int)(x.ug * (size_t)p.c.cap);
+    tma_load_2d(s0 + L.k0, tmK, 0, row0, bar);
+    tma_load_2d(s0 + L.k1, tmK, 64, row0, bar);
+    tma_load_2d(s0 + L.v0, tmV, 0, row0, bar);
+    tma_load_2d(s0 + L.v1, tmV, 64, row0, bar);
+  }
+  const int G = p.c.G;
+  const unsigned char *q =
+      reinterpret_cast<const unsigned char *>(p.q + x.krow * G * 128);
+  for (int i = lane; i < G * 16; i += 32)  // query rows, 16 pieces each
+    cp_async16(s0 + L.q + (i >> 4) * kQPitch + (i & 15) * 16, q + i * 16);
+  cp_async16(s0 + (lane < 16 ? L.kn : L.vn) + (lane & 15) * 16,
+             reinterpret_cast<const unsigned char *>(
+                 (lane < 16 ? p.k_new : p.v_new) + x.krow * 128) +
+                 (lane & 15) * 16);
+  const int nsc = p.Rb / 4;  // 16-byte pieces of the scores (and positions)
+  const unsigned char *sc =
+      reinterpret_cast<const unsigned char *>(p.c.score + x.ug * p.c.sstride);
+  const unsigned char *ps =
+      reinterpret_cast<const unsigned char *>(p.c.pos + x.ug * p.c.sstride);
+  for (int i = lane; i < 2 * nsc; i += 32)
+    cp_async16(s0 + (i < nsc ? L.sc + i * 16 : L.ps + (i - nsc) * 16),
+               (i < nsc ? sc + i * 16 : ps + (i - nsc) * 16));
+  if (lane == 31)
+    cp_async16(s0 + L.st, p.c.state + x.ug * 4);
+  cp_async_arrive_noinc(bar);
 }
 
 #include "kvr_fused_unit.cuh"
@@ -160,7 +185,7 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < p.n_stages; ++s) {
-      mbar_init(smem_u32(&full_bar[s]), 1);
+      mbar_init(smem_u32(&full_bar[s]), 1 + 32);  // TMA + producer lanes
       mbar_init(smem_u32(&empty_bar[s]), U);  // one arrival per group warp
       issued_k[s] = -1;
       consumed_k[s] = -1;
@@ -184,23 +209,32 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
     // threads on one stage could run a full ring ahead and alias the
     // mbarrier parity).
     const int j = warp - consumers;
-    if (lane == 0) {
-      for (int k = 0; k < mine; ++k) {
-        const int s = k % p.n_stages;
-        if (s % kProducers != j) continue;
-        const uint32_t ph = (uint32_t)(k / p.n_stages) & 1u;
-        if (!mbar_wait(smem_u32(&empty_bar[s]), ph ^ 1u, &s_abort)) {
+    for (int k = 0; k < mine; ++k) {
+      const int s = k % p.n_stages;
+      if (s % kProducers != j) continue;
+      const uint32_t ph = (uint32_t)(k / p.n_stages) & 1u;
+      // Lane 0 waits (bounded) and tells the warp; __syncwarp orders the
+      // other lanes' copies after the consumers' release it observed.
+      int ok = 1;
+      if (lane == 0) ok = mbar_wait(smem_u32(&empty_bar[s]), ph ^ 1u, &s_abort);
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) {
+        if (lane == 0) {
           atomicOr(p.c.err, ERR_TIMEOUT);
           s_abort = 1;
-          break;
         }
-        issue_unit(p, &tmK, &tmV, smem + s * L.bytes, smem_u32(&full_bar[s]),
-                   (int)blockIdx.x + k * (int)gridDim.x);
-        issued_k[s] = k;
+        break;
       }
+      __syncwarp();
+      issue_unit(p, &tmK, &tmV, smem + s * L.bytes, smem_u32(&full_bar[s]),
+                 (int)blockIdx.x + k * (int)gridDim.x, lane);
+      __syncwarp();
+      if (lane == 0) issued_k[s] = k;
     }
   } else if (warp < consumers) {
     const int grp = warp / U, w = warp % U, bar_id = 1 + grp;
+    unsigned char *garea =
+        smem + p.n_stages * L.bytes + grp * GroupLayout(U).bytes;
     for (int k = grp; k < mine; k += p.n_groups) {
       const int s = k % p.n_stages;
       const uint32_t ph = (uint32_t)(k / p.n_stages) & 1u;
@@ -220,14 +254,22 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
       group_bar(bar_id, 32 * U);
       if (!s_ok[grp]) break;
       mbar_try_wait(smem_u32(&full_bar[s]), ph);  // acquire for this thread
-      process_unit<T, U, kOutBf16>(p, smem + s * L.bytes, w, lane, bar_id);
+      UnitFront<(T + U - 1) / U> f;
+      const bool ok = unit_front<T, U>(p, smem + s * L.bytes,
+                                       (int)blockIdx.x + k * (int)gridDim.x,
+                                       w, lane, f);
       // Each warp releases the stage once its own reads and writes of it
-      // are done (the async-proxy fence orders them before the refill).
+      // are done (the async-proxy fence orders them before the refill); the
+      // rest of the unit runs from registers and the group's own area.
       fence_proxy_async();
       __syncwarp();
       if (lane == 0) {
         if (w == 0) consumed_k[s] = k;
         mbar_arrive(smem_u32(&empty_bar[s]));
+      }
+      if (ok) {
+        unit_publish<T, U>(garea, f, w, lane);
+        unit_back<T, U, kOutBf16>(p, garea, f, w, lane, bar_id);
       }
     }
   }
@@ -288,6 +330,8 @@ int fused_group_warps(int R, int requested) {
   return T <= 3 ? one : two;  // measured: two tiles per warp from T = 4 on
 }
 
+int fused_group_bytes(int U) { return (int)GroupLayout(U).bytes; }
+int fused_max_groups() { return kMaxGroups; }
 int fused_max_threads() { return kMaxThreads; }
 int fused_producer_warps() { return kProducers; }
 

@@ -84,6 +84,9 @@ int fused_stage_bytes(int R);
 // Warps that share one unit of R staged rows: `requested` if it is one of
 // the supported choices (one or two row tiles per warp), else the default.
 int fused_group_warps(int R, int requested);
+// Bytes of one consumer group's exchange area (after the ring of stages).
+int fused_group_bytes(int U);
+int fused_max_groups();
 int fused_max_threads();
 int fused_producer_warps();
 cudaError_t launch_fused_step(const CUtensorMap &tmK, const CUtensorMap &tmV,
