@@ -34,6 +34,12 @@
 //    apart, so a group first waits until the producer has recorded the unit
 //    as issued (which implies the earlier phase completed) and only then on
 //    the stage's full barrier.
+//  - Launched with programmatic stream serialization: a launch may start
+//    while the previous kernel of the stream drains (its barrier setup
+//    overlaps that tail); griddepcontrol.wait then holds every thread until
+//    the previous grid has completed and its writes are visible, before the
+//    first access to global memory.  Each CTA allows the next launch to
+//    start once its own setup is done.
 //  - Every wait on an mbarrier is bounded (about 2 s); on timeout the kernel
 //    sets ERR_TIMEOUT in the device error word and drains its own copies.
 #include <cuda.h>
@@ -202,6 +208,8 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
   }
   fence_proxy_async();
   __syncthreads();
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
   if (warp >= consumers) {
     // Producers: warp `consumers + j` owns the stages s with s % kProducers
@@ -294,9 +302,17 @@ cudaError_t launch_tu(const CUtensorMap &tmK, const CUtensorMap &tmV,
   cudaError_t e = cudaFuncSetAttribute(
       kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
   if (e != cudaSuccess) return e;
-  const int threads = 32 * (p.n_groups * U + kProducers);
-  kern<<<grid, threads, smem_bytes, st>>>(tmK, tmV, p);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(32 * (p.n_groups * U + kProducers));
+  cfg.dynamicSmemBytes = smem_bytes;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, tmK, tmV, p);
 }
 
 template <bool kOutBf16>
