@@ -51,6 +51,7 @@ __host__ __device__ constexpr size_t fork_fixed_bytes(int D, int n_max) {
 template <typename T, typename O, int D>
 __global__ void __launch_bounds__(kThreads)
     fork_attend_kernel(ForkView f, StepArgs a, int n_max) {
+  pdl_begin();
   extern __shared__ __align__(16) unsigned char smem_raw[];
   constexpr int P = D / 2;         // dimension pairs
   constexpr int R = kThreads / P;  // row groups of the PV pass
@@ -215,6 +216,7 @@ __global__ void __launch_bounds__(kThreads)
 template <typename T, int D>
 __global__ void __launch_bounds__(kThreads)
     fork_commit_kernel(ForkView f, const int32_t *chosen, int B, int W) {
+  pdl_begin();
   __shared__ unsigned hist[256];
   __shared__ unsigned long long s_prefix;
   __shared__ int s_need, s_base, s_count;
@@ -317,8 +319,8 @@ cudaError_t fork_attend_dispatch(const ForkView &f, const StepArgs &a,
   cudaError_t e = cudaFuncSetAttribute(
       kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
   if (e != cudaSuccess) return e;
-  kern<<<f.p.S * a.nl * f.p.H, kThreads, bytes, st>>>(f, a, n_max);
-  return cudaGetLastError();
+  return launch_pdl(kern, dim3(f.p.S * a.nl * f.p.H), dim3(kThreads), bytes,
+                    st, f, a, n_max);
 }
 
 template <typename T, int D>
@@ -329,8 +331,8 @@ cudaError_t fork_commit_dispatch(const ForkView &f, const int32_t *chosen,
   cudaError_t e = cudaFuncSetAttribute(
       kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
   if (e != cudaSuccess) return e;
-  kern<<<f.p.S * f.p.L * f.p.H, kThreads, bytes, st>>>(f, chosen, B, W);
-  return cudaGetLastError();
+  return launch_pdl(kern, dim3(f.p.S * f.p.L * f.p.H), dim3(kThreads), bytes,
+                    st, f, chosen, B, W);
 }
 
 }  // namespace

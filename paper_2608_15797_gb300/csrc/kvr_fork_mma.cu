@@ -131,6 +131,7 @@ __global__ void __launch_bounds__(32 * kMaxCand)
                     const __grid_constant__ CUtensorMap tmTK,
                     const __grid_constant__ CUtensorMap tmTV,
                     const ForkMmaParams p) {
+  pdl_begin();
   extern __shared__ unsigned char smem_raw[];
   __shared__ __align__(8) uint64_t pre_bar;
   __shared__ __align__(8) uint64_t ring_bar[kMaxCand][2];
@@ -392,14 +393,15 @@ cudaError_t launch_fork_mma(const CUtensorMap &tmK, const CUtensorMap &tmV,
     e = cudaFuncSetAttribute(fork_mma_kernel<true>,
                              cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
-    fork_mma_kernel<true><<<units, threads, smem, st>>>(tmK, tmV, tmTK, tmTV, p);
+    return launch_pdl(fork_mma_kernel<true>, dim3(units), dim3(threads), smem,
+                      st, tmK, tmV, tmTK, tmTV, p);
   } else {
     e = cudaFuncSetAttribute(fork_mma_kernel<false>,
                              cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
-    fork_mma_kernel<false><<<units, threads, smem, st>>>(tmK, tmV, tmTK, tmTV, p);
+    return launch_pdl(fork_mma_kernel<false>, dim3(units), dim3(threads), smem,
+                      st, tmK, tmV, tmTK, tmTV, p);
   }
-  return cudaGetLastError();
 }
 
 }  // namespace kvr

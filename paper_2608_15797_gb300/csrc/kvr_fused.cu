@@ -190,6 +190,8 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
   const int consumers = p.n_groups * U;
 
   if (threadIdx.x == 0) {
+    prefetch_tmap(&tmK);
+    prefetch_tmap(&tmV);
     for (int s = 0; s < p.n_stages; ++s) {
       mbar_init(smem_u32(&full_bar[s]), 1 + 32);  // TMA + producer lanes
       mbar_init(smem_u32(&empty_bar[s]), U);  // one arrival per group warp
@@ -208,8 +210,7 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
   }
   fence_proxy_async();
   __syncthreads();
-  asm volatile("griddepcontrol.wait;" ::: "memory");
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  pdl_begin();
 
   if (warp >= consumers) {
     // Producers: warp `consumers + j` owns the stages s with s % kProducers
@@ -302,17 +303,8 @@ cudaError_t launch_tu(const CUtensorMap &tmK, const CUtensorMap &tmV,
   cudaError_t e = cudaFuncSetAttribute(
       kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
   if (e != cudaSuccess) return e;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(grid);
-  cfg.blockDim = dim3(32 * (p.n_groups * U + kProducers));
-  cfg.dynamicSmemBytes = smem_bytes;
-  cfg.stream = st;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, kern, tmK, tmV, p);
+  return launch_pdl(kern, dim3(grid), dim3(32 * (p.n_groups * U + kProducers)),
+                    smem_bytes, st, tmK, tmV, p);
 }
 
 template <bool kOutBf16>

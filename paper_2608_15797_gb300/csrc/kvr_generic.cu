@@ -52,6 +52,7 @@ template <typename T, typename O, int D, bool kExtScratch = false>
 __global__ void __launch_bounds__(kThreads)
     attend_score_kernel(CacheView c, StepArgs a, int logits_in_smem,
                         float *ext) {
+  pdl_begin();
   extern __shared__ float smem[];
   constexpr int P = D / 2;         // dimension pairs
   constexpr int R = kThreads / P;  // row groups of the PV pass
@@ -192,6 +193,7 @@ __global__ void __launch_bounds__(kThreads)
 template <typename T, int D>
 __global__ void __launch_bounds__(kThreads)
     evict_kernel(CacheView c, int lb, int nl, int B, int W) {
+  pdl_begin();
   __shared__ unsigned hist[256];
   __shared__ unsigned long long s_prefix;
   __shared__ int s_need, s_base, s_count;
@@ -309,8 +311,8 @@ cudaError_t attend_dispatch(const CacheView &c, const StepArgs &a,
       kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
   if (e != cudaSuccess) return e;
   const int grid = c.S * a.nl * c.H;
-  kern<<<grid, kThreads, bytes, st>>>(c, a, in_smem, nullptr);
-  return cudaGetLastError();
+  return launch_pdl(kern, dim3(grid), dim3(kThreads), bytes, st, c, a, in_smem,
+                    static_cast<float *>(nullptr));
 }
 
 template <typename T, typename O, int D>
@@ -321,8 +323,8 @@ cudaError_t attend_ext_dispatch(const CacheView &c, const StepArgs &a,
   cudaError_t e = cudaFuncSetAttribute(
       kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
   if (e != cudaSuccess) return e;
-  kern<<<c.S * a.nl * c.H, kThreads, bytes, st>>>(c, a, 0, ext);
-  return cudaGetLastError();
+  return launch_pdl(kern, dim3(c.S * a.nl * c.H), dim3(kThreads), bytes, st, c,
+                    a, 0, ext);
 }
 
 template <typename T, int D>
@@ -335,8 +337,8 @@ cudaError_t evict_dispatch(const CacheView &c, int lb, int nl, int max_rows,
   cudaError_t e = cudaFuncSetAttribute(
       kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
   if (e != cudaSuccess) return e;
-  kern<<<c.S * nl * c.H, kThreads, bytes, st>>>(c, lb, nl, B, W);
-  return cudaGetLastError();
+  return launch_pdl(kern, dim3(c.S * nl * c.H), dim3(kThreads), bytes, st, c,
+                    lb, nl, B, W);
 }
 
 }  // namespace

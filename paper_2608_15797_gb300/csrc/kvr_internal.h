@@ -19,6 +19,32 @@ enum : unsigned {
 
 __host__ __device__ inline int round_up16(int x) { return (x + 15) & ~15; }
 
+// Every kernel of libkvr is launched with programmatic stream serialization
+// (launch_pdl): it may start while the previous kernel of the stream drains,
+// so it runs pdl_begin() before its first global memory access.  The wait
+// returns once the previous grid has completed and its writes are visible;
+// the trigger then lets the next launch start early in turn.
+__device__ __forceinline__ void pdl_begin() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block,
+                       size_t smem, cudaStream_t st, Args &&...args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, static_cast<Args &&>(args)...);
+}
+
 // Device view of one cache: every pointer points into the caller's buffer.
 // A unit u = (s * L + l) * H + h.
 struct CacheView {

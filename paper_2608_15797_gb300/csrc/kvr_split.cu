@@ -45,6 +45,7 @@ __global__ void __launch_bounds__(32 * kWarps)
     split_partial_kernel(const __grid_constant__ CUtensorMap tmK,
                          const __grid_constant__ CUtensorMap tmV,
                          const SplitParams p) {
+  pdl_begin();
   extern __shared__ unsigned char smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[kStages];
   __shared__ volatile int s_abort;
@@ -293,6 +294,7 @@ __global__ void __launch_bounds__(32 * kWarps)
 template <typename O>
 __global__ void __launch_bounds__(128) split_combine_kernel(const SplitParams p,
                                                             void *out) {
+  pdl_begin();
   const CacheView &c = p.c;
   const int G = c.G, idx = blockIdx.x;
   const int h = idx % c.H, lr = (idx / c.H) % p.nl, sq = idx / (c.H * p.nl);
@@ -348,15 +350,14 @@ cudaError_t launch_split_attend(const CUtensorMap &tmK, const CUtensorMap &tmV,
       split_partial_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   const int units = p.c.S * p.nl * p.c.H;
-  split_partial_kernel<<<dim3(p.n_splits, units), 32 * kWarps, smem, st>>>(
-      tmK, tmV, p);
-  e = cudaGetLastError();
+  e = launch_pdl(split_partial_kernel, dim3(p.n_splits, units),
+                 dim3(32 * kWarps), smem, st, tmK, tmV, p);
   if (e != cudaSuccess) return e;
   if (p.c.out_bf16)
-    split_combine_kernel<__nv_bfloat16><<<units, 128, 0, st>>>(p, out);
-  else
-    split_combine_kernel<float><<<units, 128, 0, st>>>(p, out);
-  return cudaGetLastError();
+    return launch_pdl(split_combine_kernel<__nv_bfloat16>, dim3(units),
+                      dim3(128), 0, st, p, out);
+  return launch_pdl(split_combine_kernel<float>, dim3(units), dim3(128), 0, st,
+                    p, out);
 }
 
 }  // namespace kvr

@@ -54,6 +54,7 @@ __global__ void __launch_bounds__(32 * kWarps)
     stream_step_kernel(const __grid_constant__ CUtensorMap tmK,
                        const __grid_constant__ CUtensorMap tmV,
                        const StreamParams p) {
+  pdl_begin();
   extern __shared__ unsigned char smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[kStages];
   __shared__ volatile int s_abort;
@@ -403,14 +404,15 @@ cudaError_t launch_stream_step(const CUtensorMap &tmK, const CUtensorMap &tmV,
     e = cudaFuncSetAttribute(stream_step_kernel<true>,
                              cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
-    stream_step_kernel<true><<<units, 32 * kWarps, smem, st>>>(tmK, tmV, p);
+    return launch_pdl(stream_step_kernel<true>, dim3(units), dim3(32 * kWarps),
+                      smem, st, tmK, tmV, p);
   } else {
     e = cudaFuncSetAttribute(stream_step_kernel<false>,
                              cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
-    stream_step_kernel<false><<<units, 32 * kWarps, smem, st>>>(tmK, tmV, p);
+    return launch_pdl(stream_step_kernel<false>, dim3(units), dim3(32 * kWarps),
+                      smem, st, tmK, tmV, p);
   }
-  return cudaGetLastError();
 }
 
 }  // namespace kvr
