@@ -51,6 +51,12 @@ def parse():
     p.add_argument("--seed", type=int, default=0)
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=15.0)
+    p.add_argument("--cpu-all-seconds", type=float, default=8.0,
+                   help="oracle seconds per process for the all-cores rate")
+    p.add_argument("--per-layer-steps", type=int, default=500,
+                   help="steps timed as one launch per layer")
+    p.add_argument("--latency-steps", type=int, default=1000,
+                   help="steps of the single-sequence latency run")
     p.add_argument("--prior-min", type=int, default=inputs.PRIOR_LEN_RANGE[0],
                    help="shortest prior context (profiling uses a small case)")
     p.add_argument("--prior-max", type=int, default=inputs.PRIOR_LEN_RANGE[1])
@@ -106,6 +112,23 @@ def oracle_rate(w, seed, max_seconds, max_steps=None):
     per_seq_step = spent / n
     # one step of the workload = n_seq sequences
     return 1.0 / (per_seq_step * w.n_seq), n, spent
+
+
+def _oracle_worker(job):
+    workload, seed, seconds = job
+    w = inputs.WORKLOADS[workload]
+    rate, n, spent = oracle_rate(w, seed, seconds)
+    return rate, n, spent
+
+
+def oracle_rate_all_cores(workload, seed, seconds, procs):
+    """The same oracle sample on `procs` processes at once (one sequence
+    each, started with spawn); returns the summed rate in steps/s."""
+    import multiprocessing as mp
+    with mp.get_context("spawn").Pool(procs) as pool:
+        res = pool.map(_oracle_worker,
+                       [(workload, seed + 101 * i, seconds) for i in range(procs)])
+    return sum(r for r, _, _ in res), sum(n for _, n, _ in res)
 
 
 # --------------------------------------------------------------------------
@@ -288,6 +311,32 @@ def run_kvr(args, rank, world, local_rank):
     per_launch_ms = total_ms / max(1, launches)
     cache.sync_status()
 
+    # The same steady-state steps as one launch per layer (L calls a step),
+    # each layer's inputs and output contiguous.
+    Kl = max(1, min(K, args.per_layer_steps))
+    lpool = [[tuple(x[:, l:l + 1].contiguous() for x in pool[i])
+              for l in range(L)] for i in range(4)]
+    lout = [torch.empty(S, 1, H * G, d, dtype=torch.bfloat16, device=dev)
+            for _ in range(L)]
+
+    def layer_step(i):
+        for l in range(L):
+            q, kn, vn = lpool[i % 4][l]
+            kvr.kvr_decode_step(cache.handle, l, l + 1, q, kn, vn, lout[l], B,
+                                W, stream)
+
+    for i in range(3):
+        layer_step(i)
+    torch.cuda.synchronize()
+    t0.record(stream)
+    for i in range(Kl):
+        layer_step(i)
+    t1.record(stream)
+    torch.cuda.synchronize()
+    per_layer_ms = t0.elapsed_time(t1) / Kl
+    cache.sync_status()
+    del lpool, lout
+
     if world > 1:
         t = torch.tensor([total_ms], device=dev)
         torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
@@ -318,9 +367,49 @@ def run_kvr(args, rank, world, local_rank):
     unit_bytes = cost_model.step_unit_bytes(B + W, d, G, 2, 2, B, W)
     launch_bytes = unit_bytes * S * L * H
     return dict(total_ms=total_ms, per_launch_ms=per_launch_ms, K=K,
+                per_layer_ms=per_layer_ms, Kl=Kl,
                 first_ms=first_ms, clocks=clocks, e2e_ms=e2e_ms, Ke=Ke,
                 bi=bi, bo=bo, launch_bytes=launch_bytes, lens=lens,
                 launches=launches)
+
+
+def run_latency_s1(args, local_rank):
+    """Single-sequence 7B decode (prompt 512, B=64, W=8): steady-state
+    step latency over all 28 layers, one launch per step.  The working set
+    (4.8 MB) stays in L2, so this is a latency figure, not a bandwidth one."""
+    import torch
+    from paper_2608_15797_gb300 import kvr
+    dev = torch.device("cuda", local_rank)
+    w = inputs.WORKLOADS["7b_b64"]
+    S, L, H, G, d = 1, w.n_layers, w.n_kv_heads, w.group, w.head_dim
+    cache = kvr.Cache(S, L, H, G, d, w.prompt + 1, kv_dtype="bf16",
+                      out_dtype="bf16", device=dev)
+    k, v = inputs.prompt(w, args.seed, 0, w.prompt)
+    bf = torch.bfloat16
+    cache.load(0, torch.from_numpy(k).to(dev).to(bf),
+               torch.from_numpy(v).to(dev).to(bf))
+    pool = []
+    for i in range(8):
+        q, kn, vn = inputs.step_inputs(w, args.seed, i, 1)
+        pool.append(tuple(torch.from_numpy(x).to(dev).to(bf) for x in (q, kn, vn)))
+    out = torch.empty(S, L, H * G, d, dtype=torch.bfloat16, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    for i in range(30):
+        kvr.kvr_decode_step(cache.handle, 0, L, *pool[i % 8], out, w.budget,
+                            w.window, stream)
+    torch.cuda.synchronize()
+    K = max(1, args.latency_steps)
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for i in range(K):
+        kvr.kvr_decode_step(cache.handle, 0, L, *pool[i % 8], out, w.budget,
+                            w.window, stream)
+    t1.record(stream)
+    torch.cuda.synchronize()
+    cache.sync_status()
+    return {"workload": "7b_b64 (1 sequence, prompt 512, B=64, W=8)",
+            "us_per_step": t0.elapsed_time(t1) * 1e3 / K, "steps": K}
 
 
 # --------------------------------------------------------------------------
@@ -529,6 +618,7 @@ def main():
     peak = float(peaks["hbm_gbs"])
     steps_per_s = world * r["K"] / (r["total_ms"] / 1e3)
     achieved = r["launch_bytes"] / (r["per_launch_ms"] / 1e3) / 1e9
+    lat = run_latency_s1(args, local_rank) if world == 1 else None
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
         rate, n, spent = oracle_rate(w, args.seed, args.cpu_seconds)
@@ -536,6 +626,16 @@ def main():
                "sample": f"{n} steady-state steps of 1 of the {w.n_seq} "
                          f"sequences ({spent:.1f} s of fp64 oracle), scaled "
                          f"x{w.n_seq}"}
+        procs = os.cpu_count() or 1
+        if procs > 1 and args.cpu_all_seconds > 0:
+            rate_all, n_all = oracle_rate_all_cores(
+                args.workload, args.seed, args.cpu_all_seconds, procs)
+            cpu["all_cores"] = {
+                "value": rate_all, "cores": procs,
+                "sample": f"{procs} processes, one sequence each, "
+                          f"{args.cpu_all_seconds:.0f} s each ({n_all} "
+                          f"sequence-steps), summed and scaled to "
+                          f"{w.n_seq} sequences"}
     line = {
         "metric": metric_name(w), "value": steps_per_s, "unit": "steps/s",
         "n_gpus": world, "steps": r["K"], "warmup": args.warmup,
@@ -566,6 +666,11 @@ def main():
                 "unit": "steps/s", "h2d_bytes_per_step": r["bi"],
                 "d2h_bytes_per_step": r["bo"]},
         "gpu_launches": r["launches"],
+        "per_layer_launches": {
+            "launches_per_step": w.n_layers,
+            "ms_per_step": r["per_layer_ms"],
+            "steps_per_s": 1e3 / r["per_layer_ms"], "steps": r["Kl"]},
+        "latency_1seq": lat,
         "clocks": r["clocks"],
         "cpu_baseline": cpu,
     }
