@@ -70,6 +70,10 @@ def parse():
                         "16k context; fork: 72B best-of-8 candidate step")
     p.add_argument("--seqs", type=int, default=0,
                    help="sequences for --mode helper/fork (0: 16 / 4)")
+    p.add_argument("--chunk-groups", type=int, default=0,
+                   help="chunked kernel: consumer groups per SM (0 auto, -1 off)")
+    p.add_argument("--chunk-stages", type=int, default=0,
+                   help="chunked kernel: ring stages per group (0 auto)")
     p.add_argument("--fused-group-warps", type=int, default=0,
                    help="warps sharing one unit in the fused kernel "
                         "(0: the library's choice)")
@@ -244,6 +248,9 @@ def run_kvr(args, rank, world, local_rank):
     if args.fused_groups or args.fused_group_warps:
         kvr.kvr_cache_set_fused_tuning(cache.handle, args.fused_groups,
                                        args.fused_group_warps)
+    if args.chunk_groups or args.chunk_stages:
+        kvr.kvr_cache_set_chunk_tuning(cache.handle, args.chunk_groups,
+                                       args.chunk_stages)
     gen = torch.Generator(device=dev)
     gen.manual_seed(1_000_003 * (args.seed + 1) + rank)
     for s in range(S):
@@ -493,6 +500,9 @@ def run_fork(args):
     B, Wn, T = w.budget, w.window, w.cand_step
     dev = torch.device("cuda", 0)
     cache = kvr.Cache(S, L, H, G, d, B + Wn + T + 1, "bf16", "bf16", device=dev)
+    if args.chunk_groups or args.chunk_stages:
+        kvr.kvr_cache_set_chunk_tuning(cache.handle, args.chunk_groups,
+                                       args.chunk_stages)
     gen = torch.Generator(device=dev)
     gen.manual_seed(args.seed + 29)
     for s in range(S):

@@ -229,6 +229,17 @@ kvr_status kvr_cache_set_fused(kvr_cache *cache, int enable);
 kvr_status kvr_cache_set_fused_tuning(kvr_cache *cache, int groups,
                                       int group_warps);
 
+/* Tuning of the chunked kernel that runs units of 129..1024 live rows and
+ * the candidate step (bf16, head_dim 128, G <= 8): units stream in 32-row
+ * chunks through per-group shared-memory rings.  groups: consumer groups per
+ * SM (1..4; 0 = the library's choice; -1 = never use this kernel, so the
+ * older one-CTA-per-unit kernels run instead).  stages: ring stages per
+ * group (2..4; 0 = the library's choice).  A choice that does not fit in
+ * shared memory for a call falls back to the older kernels for that call.
+ * Results do not depend on either. */
+kvr_status kvr_cache_set_chunk_tuning(kvr_cache *cache, int groups,
+                                      int stages);
+
 /* ---- the same step for callers that cannot allocate -------------------- */
 
 /* The paper has no counterpart to this call: it is a deployment variant.

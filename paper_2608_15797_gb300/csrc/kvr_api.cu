@@ -99,6 +99,8 @@ struct kvr_cache {
   bool fused = true;              // use the fused kernel where it applies
   int fused_groups = 0;           // units computed at once per SM (0: auto)
   int fused_group_warps = 0;      // warps per unit (0: auto)
+  int chunk_groups = 0;           // chunked kernel: groups (0 auto, -1 off)
+  int chunk_stages = 0;           // chunked kernel: stages per group (0 auto)
   int forks = 0;                  // live forks: the cache is read-only meanwhile
   int sm_count = 0;               // of the device, queried on first use
   int smem_optin = 0;
@@ -358,6 +360,69 @@ bool try_stream(kvr_cache *c, const StepArgs &a, bool evict, int budget,
   return true;
 }
 
+// Consumer groups and ring stages per group of the chunked kernel for jobs
+// of up to n_max rows: the first of (4,2) (3,3) (3,2) (2,3) (2,2) (1,3)
+// (1,2) that fits in shared memory (more groups first: measured), or the
+// tuned choice.
+bool chunk_config(const kvr_cache *c, int n_max, int *groups, int *stages) {
+  static const int order[7][2] = {{4, 2}, {3, 3}, {3, 2}, {2, 3},
+                                  {2, 2}, {1, 3}, {1, 2}};
+  const size_t limit = (size_t)c->smem_optin - 512;
+  const int tg = c->chunk_groups, ts = c->chunk_stages;
+  for (const auto &o : order) {
+    const int g = tg > 0 ? tg : o[0], s = ts > 0 ? ts : o[1];
+    if (g > kvr::chunk_max_groups() || s > kvr::chunk_max_stages()) continue;
+    if (kvr::chunk_smem_bytes(n_max, g, s) <= limit) {
+      *groups = g;
+      *stages = s;
+      return true;
+    }
+  }
+  return false;
+}
+
+// Launch the chunked step for plain units if this call qualifies.
+bool try_chunked(kvr_cache *c, const StepArgs &a, bool evict, int budget,
+                 int window, cudaStream_t stream, cudaError_t *err) {
+  const CacheView &v = c->view;
+  if (!c->fused || c->chunk_groups < 0 || !v.kv_bf16 || v.d != 128 ||
+      v.G > 8)
+    return false;
+  if (a.max_rows > kvr::chunk_max_rows()) return false;
+  if (evict && (long long)a.max_rows > (long long)budget + window + 1)
+    return false;
+  const size_t rows = (size_t)v.S * v.L * v.H * v.cap;
+  if (rows >= (size_t)INT32_MAX) return false;
+  if (!aligned16(a.q) || !aligned16(a.k_new) || !aligned16(a.v_new) ||
+      !aligned16(a.out))
+    return false;
+  if (!device_facts(c)) return false;
+  kvr::ChunkParams p{};
+  if (!chunk_config(c, a.max_rows, &p.n_groups, &p.n_stages)) return false;
+  const std::pair<CUtensorMap, CUtensorMap> *maps =
+      slab_maps(c, kvr::chunk_box_rows());
+  if (!maps) return false;
+  p.c = v;
+  p.fork = 0;
+  p.q = static_cast<const __nv_bfloat16 *>(a.q);
+  p.k_new = static_cast<const __nv_bfloat16 *>(a.k_new);
+  p.v_new = static_cast<const __nv_bfloat16 *>(a.v_new);
+  p.out = a.out;
+  p.lb = a.lb;
+  p.nl = a.nl;
+  p.n_jobs = v.S * a.nl * v.H;
+  p.n_max = a.max_rows;
+  p.budget = budget;
+  p.window = window;
+  p.evict = evict ? 1 : 0;
+  p.scale_log2e = v.scale * 1.4426950408889634f;
+  p.inv_g = 1.f / (float)v.G;
+  const int grid = std::min(c->sm_count, p.n_jobs);
+  *err = kvr::launch_chunk_step(maps->first, maps->second, nullptr, nullptr, p,
+                                grid, stream);
+  return true;
+}
+
 // Splits for kvr_decode_attend: about two waves of the partial kernel (three
 // CTAs per SM), never less than 256 rows per split.
 int auto_splits(const kvr_cache *c, int lb, int le) {
@@ -519,6 +584,7 @@ kvr_status kvr_decode_attend_score(kvr_cache *c, int lb, int le, const void *q,
   StepArgs a = step_args(c, lb, le, q, k_new, v_new, out);
   cudaError_t e = cudaSuccess;
   if (!try_fused(c, a, false, 0, 0, as_stream(stream), &e) &&
+      !try_chunked(c, a, false, 0, 0, as_stream(stream), &e) &&
       !try_stream(c, a, false, 0, 0, as_stream(stream), &e))
     e = kvr::launch_attend_score_generic(c->view, a, as_stream(stream));
   if (e != cudaSuccess) return cuda_fail("kvr_decode_attend_score", e);
@@ -541,6 +607,16 @@ kvr_status kvr_cache_set_fused_tuning(kvr_cache *c, int groups,
                 group_warps);
   c->fused_groups = groups;
   c->fused_group_warps = group_warps;
+  return KVR_OK;
+}
+
+kvr_status kvr_cache_set_chunk_tuning(kvr_cache *c, int groups, int stages) {
+  if (!c) return fail(KVR_EINVAL, "null cache");
+  if (groups < -1 || groups > 4 || stages < 0 || stages > 4 || stages == 1)
+    return fail(KVR_EINVAL, "chunk tuning (%d, %d) outside [-1, 4] x "
+                "{0, 2, 3, 4}", groups, stages);
+  c->chunk_groups = groups;
+  c->chunk_stages = stages;
   return KVR_OK;
 }
 
@@ -607,6 +683,7 @@ kvr_status kvr_decode_step(kvr_cache *c, int lb, int le, const void *q,
   StepArgs a = step_args(c, lb, le, q, k_new, v_new, out);
   cudaError_t e = cudaSuccess;
   if (try_fused(c, a, true, budget, window, as_stream(stream), &e) ||
+      try_chunked(c, a, true, budget, window, as_stream(stream), &e) ||
       try_stream(c, a, true, budget, window, as_stream(stream), &e)) {
     if (e != cudaSuccess) return cuda_fail("kvr_decode_step", e);
     c->launches += 1;
@@ -865,7 +942,15 @@ kvr_status kvr_fork_decode_attend_score(kvr_fork *f, int lb, int le,
       nt_max = std::max(nt_max, f->tlen[(size_t)s * p->desc.n_layers + l]);
   const CacheView &pv = p->view;
   const std::pair<CUtensorMap, CUtensorMap> *maps = nullptr;
-  const bool mma_ok =
+  kvr::ChunkParams cp{};
+  const bool chunk_ok =
+      p->fused && p->chunk_groups >= 0 && f->tail_maps && pv.G <= 8 &&
+      n_max <= kvr::chunk_max_rows() && device_facts(p) &&
+      chunk_config(p, n_max, &cp.n_groups, &cp.n_stages) &&
+      (size_t)pv.S * pv.L * pv.H * pv.cap < (size_t)INT32_MAX &&
+      aligned16(q) && aligned16(k_new) && aligned16(v_new) && aligned16(out) &&
+      (maps = slab_maps(p, kvr::chunk_box_rows())) != nullptr;
+  const bool mma_ok = !chunk_ok &&
       p->fused && f->tail_maps && pv.G <= 8 &&
       f->view.N <= kvr::fork_mma_max_cand() && device_facts(p) &&
       kvr::fork_mma_smem_bytes(max_prefix, nt_max, f->view.N) + 512 <=
@@ -873,7 +958,24 @@ kvr_status kvr_fork_decode_attend_score(kvr_fork *f, int lb, int le,
       (size_t)pv.S * pv.L * pv.H * pv.cap < (size_t)INT32_MAX &&
       aligned16(q) && aligned16(k_new) && aligned16(v_new) && aligned16(out) &&
       (maps = slab_maps(p, kvr::fork_mma_box_rows())) != nullptr;
-  if (mma_ok) {
+  if (chunk_ok) {
+    cp.c = pv;
+    cp.f = f->view;
+    cp.fork = 1;
+    cp.q = static_cast<const __nv_bfloat16 *>(q);
+    cp.k_new = static_cast<const __nv_bfloat16 *>(k_new);
+    cp.v_new = static_cast<const __nv_bfloat16 *>(v_new);
+    cp.out = out;
+    cp.lb = lb;
+    cp.nl = le - lb;
+    cp.n_jobs = f->view.N * pv.S * (le - lb) * pv.H;
+    cp.n_max = n_max;
+    cp.scale_log2e = pv.scale * 1.4426950408889634f;
+    cp.inv_g = 1.f / (float)pv.G;
+    const int grid = std::min(p->sm_count, cp.n_jobs);
+    e = kvr::launch_chunk_step(maps->first, maps->second, &f->tmTK, &f->tmTV,
+                               cp, grid, as_stream(stream));
+  } else if (mma_ok) {
     kvr::ForkMmaParams mp{};
     mp.f = f->view;
     mp.q = static_cast<const __nv_bfloat16 *>(q);

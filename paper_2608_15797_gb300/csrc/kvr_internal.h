@@ -188,6 +188,33 @@ cudaError_t launch_fork_commit(const ForkView &f, const int32_t *chosen,
                                int max_rows, int budget, int window,
                                cudaStream_t st);
 
+// Persistent chunked step (kvr_chunked.cu): bf16, d = 128, G <= 8, at most
+// chunk_max_rows() rows per job with the new row.  A job is one unit of the
+// cache (fork == 0: its live rows, the new row, at most one eviction) or one
+// candidate of one unit (fork == 1: the parent's live rows as a read-only
+// prefix, the candidate's tail, the new row appended to the tail).
+struct ChunkParams {
+  CacheView c;
+  ForkView f;                  // fork == 1 only
+  int fork;
+  const __nv_bfloat16 *q, *k_new, *v_new;  // [jobs' rows][...][128]
+  void *out;
+  int lb, nl;
+  int n_jobs;                  // S * nl * H, times N for candidates
+  int n_max;                   // largest job (rows with the new row)
+  int n_groups, n_stages;      // consumer groups; ring stages per group
+  int budget, window, evict;
+  float scale_log2e, inv_g;
+};
+int chunk_box_rows();
+int chunk_max_rows();
+int chunk_max_groups();
+int chunk_max_stages();
+size_t chunk_smem_bytes(int n_max, int n_groups, int n_stages);
+cudaError_t launch_chunk_step(const CUtensorMap &tmK, const CUtensorMap &tmV,
+                              const CUtensorMap *tmTK, const CUtensorMap *tmTV,
+                              const ChunkParams &p, int grid, cudaStream_t st);
+
 }  // namespace kvr
 
 struct kvr_cache;

@@ -67,6 +67,7 @@ _SIGS = {
     "kvr_cache_launch_count": (_S, [_P, _P]),
     "kvr_cache_set_fused": (_S, [_P, _I]),
     "kvr_cache_set_fused_tuning": (_S, [_P, _I, _I]),
+    "kvr_cache_set_chunk_tuning": (_S, [_P, _I, _I]),
     "kvr_sync_status": (_S, [_P, _P]),
     "kvr_last_error": (ctypes.c_char_p, []),
 }
@@ -192,6 +193,11 @@ def kvr_cache_set_fused_tuning(h, groups: int, group_warps: int = 0):
            "kvr_cache_set_fused_tuning")
 
 
+def kvr_cache_set_chunk_tuning(h, groups: int, stages: int = 0):
+    _check(lib.kvr_cache_set_chunk_tuning(h, groups, stages),
+           "kvr_cache_set_chunk_tuning")
+
+
 def kvr_sync_status(h, stream=None):
     _check(lib.kvr_sync_status(h, _stream(stream)), "kvr_sync_status")
 
@@ -284,6 +290,10 @@ class Cache:
 
     def set_fused(self, enable: bool):
         kvr_cache_set_fused(self.handle, enable)
+
+    def set_chunk_tuning(self, groups: int, stages: int = 0):
+        """groups -1 keeps the chunked kernel off (older per-unit kernels)."""
+        kvr_cache_set_chunk_tuning(self.handle, groups, stages)
 
     def launch_count(self):
         return kvr_cache_launch_count(self.handle)

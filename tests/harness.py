@@ -22,12 +22,15 @@ def dev(x: np.ndarray, dtype: str) -> torch.Tensor:
 
 
 def make_pair(w: inputs.Workload, seed: int, S: int, cap: int,
-              prompt_lens=None, out_dtype="f32", first_pos=None, fused=True):
+              prompt_lens=None, out_dtype="f32", first_pos=None, fused=True,
+              chunk=(0, 0)):
     """A CUDA cache and an oracle cache loaded with the same prompts.
-    fused=False restricts the CUDA cache to the generic kernels."""
+    fused=False restricts the CUDA cache to the generic kernels; chunk is
+    the chunked kernel's (groups, stages) tuning, groups -1 turning it off."""
     c = kvr.Cache(S, w.n_layers, w.n_kv_heads, w.group, w.head_dim, cap,
                   kv_dtype=w.dtype, out_dtype=out_dtype)
     c.set_fused(fused)
+    c.set_chunk_tuning(*chunk)
     o = orc.OracleCache(S, w.n_layers, w.n_kv_heads, w.group, w.head_dim, cap)
     lens = [w.prompt] * S if prompt_lens is None else list(prompt_lens)
     for s in range(S):

@@ -24,25 +24,32 @@ def _cuda():
     torch.cuda.set_device(0)
 
 
-def _evicted_pair(w, seed, S, cap, prompt_lens, warm_steps, fused=True):
-    """Load prompts and run evicting steps so the parent sits at B + W rows.
-    fused=False keeps the parent (and its forks) on the generic kernels."""
+# The candidate kernels: the chunked persistent kernel (default), the
+# one-CTA-per-unit tensor-core kernel, and the generic kernels.
+PATHS = {"chunked": dict(fused=True, chunk=(0, 0)),
+         "mma": dict(fused=True, chunk=(-1, 0)),
+         "generic": dict(fused=False, chunk=(0, 0))}
+
+
+def _evicted_pair(w, seed, S, cap, prompt_lens, warm_steps, path="chunked"):
+    """Load prompts and run evicting steps so the parent sits at B + W rows;
+    the parent (and its forks) run on the kernels `path` names."""
     c, o = harness.make_pair(w, seed, S, cap=cap, prompt_lens=prompt_lens,
-                             fused=fused)
+                             **PATHS[path])
     harness.lockstep(c, o, w, seed, warm_steps, w.budget, w.window)
     return c, o
 
 
-@pytest.mark.parametrize("fused", [True, False])
+@pytest.mark.parametrize("path", list(PATHS))
 @pytest.mark.parametrize("n_cand", [1, 3, 8])
-def test_small_fork_commit_then_continue(n_cand, fused):
-    """Tail lengths cross the 16-row tile boundary (7 tokens from a ragged
-    parent, 19 for N = 8)."""
+def test_small_fork_commit_then_continue(n_cand, path):
+    """Tail lengths cross the 16-row tile and 32-row chunk boundaries (7
+    tokens from a ragged parent, 37 for N = 8)."""
     w = inputs.Workload("f", 2, 2, 3, 128, "bf16", 12, 4, 30, 0, sigma=1.0)
-    c, o = _evicted_pair(w, 21, 2, cap=40, prompt_lens=[30, 9], warm_steps=3,
-                         fused=fused)
+    c, o = _evicted_pair(w, 21, 2, cap=60, prompt_lens=[30, 9], warm_steps=3,
+                         path=path)
     o2, chosen, st = harness.fork_lockstep(c, o, w, 21, n_cand,
-                                           19 if n_cand == 8 else 7, w.budget,
+                                           37 if n_cand == 8 else 7, w.budget,
                                            w.window)
     assert (c.lengths() == np.minimum(o2.len.max(axis=2), 16)).all()
     # the committed parent keeps decoding in lock-step
@@ -107,13 +114,14 @@ def test_single_candidate_equals_plain_deferred_eviction():
                     assert abs(ma[p] - mb[p]) <= 1e-4 * max(abs(mb[p]), 1e-6)
 
 
-def test_7b_best_of_4():
+@pytest.mark.parametrize("path", ["chunked", "mma"])
+def test_7b_best_of_4(path):
     """7B geometry stepwise best-of-4: an evicted cache (prompt 512, B=128,
     W=8; heavy keys), forked to 4 candidates that decode a 16-token step
     sharing the prefix, then re-evicted and committed."""
     w = inputs.WORKLOADS["7b_bon4"]
     c, o = _evicted_pair(w, 25, 1, cap=w.prompt + 1, prompt_lens=[w.prompt],
-                         warm_steps=2)
+                         warm_steps=2, path=path)
     o2, chosen, st = harness.fork_lockstep(c, o, w, 25, w.n_cand, 16, w.budget,
                                            w.window)
     assert (c.lengths() == w.budget + w.window).all()
@@ -128,3 +136,12 @@ def test_72b_best_of_8():
                          warm_steps=1)
     harness.fork_lockstep(c, o, w, 26, 8, 8, w.budget, w.window)
     assert (c.lengths() == w.budget + w.window).all()
+
+
+def test_fork_empty_prefix_and_chunk_edges():
+    """A parent with no live rows (empty prompt: the prefix segment is empty)
+    and one whose prefix is an exact multiple of the 32-row chunk, forked and
+    decoded so the tails cross 32 rows, then committed."""
+    w = inputs.Workload("fe", 1, 2, 2, 128, "bf16", 24, 8, 0, 0, sigma=1.0)
+    c, o = harness.make_pair(w, 27, 2, cap=80, prompt_lens=[0, 32])
+    harness.fork_lockstep(c, o, w, 27, 2, 34, w.budget, w.window)

@@ -180,24 +180,63 @@ def test_capacity_and_argument_errors():
     c.sync_status()
 
 
+@pytest.mark.parametrize("chunk", [(0, 0), (-1, 0)], ids=["chunked", "stream"])
 @pytest.mark.parametrize("B,G,out", [(128, 7, "bf16"), (256, 7, "f32"),
                                      (512, 8, "bf16"), (150, 1, "f32")])
-def test_long_unit_fused_step(B, G, out):
+def test_long_unit_fused_step(B, G, out, chunk):
     """Budgets above the staged kernel's 128 rows (the throughput sweep's
-    B = 128 / 256 / 512, W = 8): the streaming fused kernel, one launch per
-    step, in lock-step with the oracle from B + W rows on."""
+    B = 128 / 256 / 512, W = 8): the chunked kernel (and the older
+    one-CTA-per-unit streaming kernel), one launch per step, in lock-step
+    with the oracle from B + W rows on."""
     W = 8
     w = inputs.Workload("long_b", 2, 2, G, 128, "bf16", B, W, B + W, 5, sigma=1.0)
     c, o = harness.make_pair(w, 13, 2, cap=B + W + 1,
-                             prompt_lens=[B + W, B + W - 37], out_dtype=out)
+                             prompt_lens=[B + W, B + W - 37], out_dtype=out,
+                             chunk=chunk)
     n0 = c.launch_count()
     harness.lockstep(c, o, w, 13, 5, B, W)
     assert c.launch_count() - n0 == 5
 
 
-def test_long_unit_growth_without_eviction():
+@pytest.mark.parametrize("chunk", [(0, 0), (-1, 0)], ids=["chunked", "stream"])
+def test_long_unit_growth_without_eviction(chunk):
     """Units growing from 100 to 300 rows with no eviction: the staged kernel
-    while they fit, then the streaming kernel."""
+    while they fit, then the chunked (or streaming) kernel."""
     w = inputs.Workload("grow", 1, 2, 4, 128, "bf16", 1 << 20, 0, 0, 40, sigma=1.0)
-    c, o = harness.make_pair(w, 14, 2, cap=400, prompt_lens=[100, 290])
+    c, o = harness.make_pair(w, 14, 2, cap=400, prompt_lens=[100, 290],
+                             chunk=chunk)
     harness.lockstep(c, o, w, 14, 40, w.budget, w.window)
+
+
+def test_chunked_ring_configurations_agree_bitwise():
+    """The chunked kernel's group count and ring depth change only the
+    schedule: every (groups, stages) gives bit-identical outputs, scores and
+    retained rows, on ragged units of 1..300 rows that cross chunk ends."""
+    W, B = 8, 200
+    w = inputs.Workload("cfg", 3, 2, 5, 128, "bf16", B, W, 0, 4, sigma=1.0)
+    lens = [0, 31, 32, 33, 129, 300]
+    res = []
+    # every configuration here fits shared memory at 301 rows (the first
+    # step's attend); one that did not would fall back to another kernel,
+    # with other rounding
+    for chunk in [(1, 2), (1, 3), (2, 2), (2, 3), (3, 2)]:
+        c, _ = harness.make_pair(w, 15, len(lens), cap=310, prompt_lens=lens,
+                                 chunk=chunk)
+        outs = []
+        for t in range(3):
+            q, kn, vn = (harness.dev(a, "bf16")
+                         for a in inputs.step_inputs(w, 15, t, len(lens)))
+            outs.append(c.step(q, kn, vn, B, W).float().cpu().numpy())
+        ex = [c.export(s, kv=True) for s in range(len(lens))]
+        res.append((outs, ex))
+        c.sync_status()
+    for outs, ex in res[1:]:
+        for a, b in zip(outs, res[0][0]):
+            assert np.array_equal(a, b)
+        for ea, eb in zip(ex, res[0][1]):
+            assert np.array_equal(ea["len"], eb["len"])
+            for l in range(w.n_layers):
+                for h in range(w.n_kv_heads):
+                    n = int(ea["len"][l, h])  # rows past len are unset memory
+                    for key in ("pos", "score", "K", "V"):
+                        assert np.array_equal(ea[key][l, h, :n], eb[key][l, h, :n])
