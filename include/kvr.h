@@ -214,6 +214,16 @@ kvr_status kvr_fork_export(const kvr_fork *fork, int cand, int seq,
 /* Free the fork's host metadata (not its buffer). NULL is a no-op. */
 void kvr_fork_destroy(kvr_fork *fork);
 
+/* Which kernel runs the fork's candidate steps (for testing and
+ * measurement; every choice computes the same step, Sec. 2.2 Eq. 2).
+ * kernel: 0 = the library's choice (the first of 1, 2, 3 that applies,
+ * else 4); 1 = candidate-batched (bf16, head_dim 128, G <= 8, N <= 8: a
+ * warp per candidate, each prefix row read once per unit for all
+ * candidates); 2 = chunked (one job per candidate and unit); 3 = one CTA per
+ * unit; 4 = generic.  A choice that does not apply to a call runs the
+ * generic kernel for that call.  Returns KVR_EINVAL outside [0, 4]. */
+kvr_status kvr_fork_set_kernel(kvr_fork *fork, int kernel);
+
 /* Choose whether kvr_decode_attend_score / kvr_decode_step may use the
  * fused single-pass kernel (bf16, head_dim 128, G <= 8, at most 128 live rows
  * per unit, at most one eviction per unit; the default) or must use the

@@ -141,6 +141,22 @@ bool encode_slab(CUtensorMap *m, void *base, size_t rows, int R) {
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// The N candidates' tails as one 3-D tensor {128 elements, units * tcap rows,
+// N candidates}: a box {64, T, N} fetches T rows of every candidate at once.
+bool encode_tails3(CUtensorMap *m, void *base, size_t rows_per_cand, int n_cand,
+                   int T) {
+  auto fn = encode_tiled();
+  if (!fn) return false;
+  cuuint64_t dims[3] = {128, (cuuint64_t)rows_per_cand, (cuuint64_t)n_cand};
+  cuuint64_t strides[2] = {256, (cuuint64_t)rows_per_cand * 256};
+  cuuint32_t box[3] = {64, (cuuint32_t)T, (cuuint32_t)n_cand};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, base, dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 }  // namespace
 
 namespace {
@@ -787,7 +803,10 @@ struct kvr_fork {
   int32_t *chosen_dev;        // [S]
   bool spent = false;
   bool tail_maps = false;     // TK / TV tensor maps encoded (tensor-core path)
-  CUtensorMap tmTK, tmTV;
+  CUtensorMap tmTK, tmTV;     // 16-row boxes
+  bool batch_maps = false;    // 3-D tail maps (candidate-batched kernel)
+  CUtensorMap tmTK3, tmTV3;
+  int kernel = 0;             // kvr_fork_set_kernel choice
 };
 
 namespace {
@@ -894,6 +913,11 @@ kvr_status kvr_fork_candidates(kvr_cache *p, int n_cand, int tail_cap,
     f->tail_maps =
         encode_slab(&f->tmTK, v.TK, trows, kvr::fork_mma_box_rows()) &&
         encode_slab(&f->tmTV, v.TV, trows, kvr::fork_mma_box_rows());
+    const int T = kvr::fork_batch_tail_rows(n_cand);
+    f->batch_maps =
+        T > 0 &&
+        encode_tails3(&f->tmTK3, v.TK, units * (size_t)tail_cap, n_cand, T) &&
+        encode_tails3(&f->tmTV3, v.TV, units * (size_t)tail_cap, n_cand, T);
   }
   p->forks += 1;
   *out = f;
@@ -941,16 +965,26 @@ kvr_status kvr_fork_decode_attend_score(kvr_fork *f, int lb, int le,
     for (int l = lb; l < le; ++l)
       nt_max = std::max(nt_max, f->tlen[(size_t)s * p->desc.n_layers + l]);
   const CacheView &pv = p->view;
-  const std::pair<CUtensorMap, CUtensorMap> *maps = nullptr;
+  const std::pair<CUtensorMap, CUtensorMap> *maps = nullptr, *maps128 = nullptr;
+  const int want = p->fused ? f->kernel : 4;  // 0 auto, 1..4 one kernel
+  const bool batch_ok =
+      (want == 0 || want == 1) && p->fused && f->batch_maps && pv.G <= 8 &&
+      f->view.N <= kvr::fork_batch_max_cand() && device_facts(p) &&
+      kvr::fork_batch_smem_bytes(n_max, f->view.N) + 512 <=
+          (size_t)p->smem_optin &&
+      (size_t)pv.S * pv.L * pv.H * pv.cap < (size_t)INT32_MAX &&
+      aligned16(q) && aligned16(k_new) && aligned16(v_new) && aligned16(out) &&
+      (maps = slab_maps(p, kvr::chunk_box_rows())) != nullptr &&
+      (maps128 = slab_maps(p, kvr::fork_batch_prefix_box_rows())) != nullptr;
   kvr::ChunkParams cp{};
-  const bool chunk_ok =
+  const bool chunk_ok = !batch_ok && (want == 0 || want == 2) &&
       p->fused && p->chunk_groups >= 0 && f->tail_maps && pv.G <= 8 &&
       n_max <= kvr::chunk_max_rows() && device_facts(p) &&
       chunk_config(p, n_max, &cp.n_groups, &cp.n_stages) &&
       (size_t)pv.S * pv.L * pv.H * pv.cap < (size_t)INT32_MAX &&
       aligned16(q) && aligned16(k_new) && aligned16(v_new) && aligned16(out) &&
       (maps = slab_maps(p, kvr::chunk_box_rows())) != nullptr;
-  const bool mma_ok = !chunk_ok &&
+  const bool mma_ok = !batch_ok && !chunk_ok && (want == 0 || want == 3) &&
       p->fused && f->tail_maps && pv.G <= 8 &&
       f->view.N <= kvr::fork_mma_max_cand() && device_facts(p) &&
       kvr::fork_mma_smem_bytes(max_prefix, nt_max, f->view.N) + 512 <=
@@ -958,7 +992,23 @@ kvr_status kvr_fork_decode_attend_score(kvr_fork *f, int lb, int le,
       (size_t)pv.S * pv.L * pv.H * pv.cap < (size_t)INT32_MAX &&
       aligned16(q) && aligned16(k_new) && aligned16(v_new) && aligned16(out) &&
       (maps = slab_maps(p, kvr::fork_mma_box_rows())) != nullptr;
-  if (chunk_ok) {
+  if (batch_ok) {
+    kvr::ForkBatchParams bp{};
+    bp.f = f->view;
+    bp.q = static_cast<const __nv_bfloat16 *>(q);
+    bp.k_new = static_cast<const __nv_bfloat16 *>(k_new);
+    bp.v_new = static_cast<const __nv_bfloat16 *>(v_new);
+    bp.out = out;
+    bp.lb = lb;
+    bp.nl = le - lb;
+    bp.n_max = n_max;
+    bp.scale_log2e = pv.scale * 1.4426950408889634f;
+    bp.inv_g = 1.f / (float)pv.G;
+    const int units = pv.S * (le - lb) * pv.H;
+    e = kvr::launch_fork_batch(maps->first, maps->second, maps128->first,
+                               maps128->second, f->tmTK3, f->tmTV3, bp,
+                               std::min(p->sm_count, units), as_stream(stream));
+  } else if (chunk_ok) {
     cp.c = pv;
     cp.f = f->view;
     cp.fork = 1;
@@ -1085,6 +1135,14 @@ kvr_status kvr_fork_export(const kvr_fork *f, int cand, int seq,
       (e = cudaMemcpy(host_tail_len, v.tlen + cu0, per_seq * sizeof(int32_t),
                       cudaMemcpyDeviceToHost)) != cudaSuccess)
     return cuda_fail("kvr_fork_export", e);
+  return KVR_OK;
+}
+
+kvr_status kvr_fork_set_kernel(kvr_fork *f, int kernel) {
+  if (!f) return fail(KVR_EINVAL, "null fork");
+  if (kernel < 0 || kernel > 4)
+    return fail(KVR_EINVAL, "fork kernel %d outside [0, 4]", kernel);
+  f->kernel = kernel;
   return KVR_OK;
 }
 

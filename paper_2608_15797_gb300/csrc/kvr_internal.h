@@ -188,6 +188,31 @@ cudaError_t launch_fork_commit(const ForkView &f, const int32_t *chosen,
                                int max_rows, int budget, int window,
                                cudaStream_t st);
 
+// Candidate-batched step (kvr_fork_batch.cu): bf16, d = 128, G <= 8,
+// N <= fork_batch_max_cand(); persistent CTAs, a warp per candidate, the
+// parent's rows streamed once per unit for all candidates.
+struct ForkBatchParams {
+  ForkView f;
+  const __nv_bfloat16 *q, *k_new, *v_new;  // [N][S][nl][...][128]
+  void *out;
+  int lb, nl;
+  int n_max;   // largest prefix + tail + 1 over the call's units
+  float scale_log2e, inv_g;
+};
+int fork_batch_max_cand();
+// Box heights of the maps it takes: the parent slab in 16-row boxes and in
+// fork_batch_prefix_box_rows()-row boxes (a full prefix block); the tails as
+// a 3-D map {128, units * tcap, N} with boxes {64, fork_batch_tail_rows(N), N}.
+int fork_batch_prefix_box_rows();
+int fork_batch_tail_rows(int n_cand);
+size_t fork_batch_smem_bytes(int n_max, int n_cand);
+cudaError_t launch_fork_batch(const CUtensorMap &tmK, const CUtensorMap &tmV,
+                              const CUtensorMap &tmK128,
+                              const CUtensorMap &tmV128,
+                              const CUtensorMap &tmTK, const CUtensorMap &tmTV,
+                              const ForkBatchParams &p, int grid,
+                              cudaStream_t st);
+
 // Persistent chunked step (kvr_chunked.cu): bf16, d = 128, G <= 8, at most
 // chunk_max_rows() rows per job with the new row.  A job is one unit of the
 // cache (fork == 0: its live rows, the new row, at most one eviction) or one

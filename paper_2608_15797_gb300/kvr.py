@@ -68,6 +68,7 @@ _SIGS = {
     "kvr_cache_set_fused": (_S, [_P, _I]),
     "kvr_cache_set_fused_tuning": (_S, [_P, _I, _I]),
     "kvr_cache_set_chunk_tuning": (_S, [_P, _I, _I]),
+    "kvr_fork_set_kernel": (_S, [_P, _I]),
     "kvr_sync_status": (_S, [_P, _P]),
     "kvr_last_error": (ctypes.c_char_p, []),
 }
@@ -191,6 +192,10 @@ def kvr_cache_set_fused(h, enable: bool):
 def kvr_cache_set_fused_tuning(h, groups: int, group_warps: int = 0):
     _check(lib.kvr_cache_set_fused_tuning(h, groups, group_warps),
            "kvr_cache_set_fused_tuning")
+
+
+def kvr_fork_set_kernel(h, kernel: int):
+    _check(lib.kvr_fork_set_kernel(h, kernel), "kvr_fork_set_kernel")
 
 
 def kvr_cache_set_chunk_tuning(h, groups: int, stages: int = 0):
@@ -359,7 +364,10 @@ def kvr_fork_destroy(fork):
 class Fork:
     """N candidates of a Cache sharing its live rows (owner of the buffer)."""
 
-    def __init__(self, cache: Cache, n_cand: int, tail_cap: int, stream=None):
+    def __init__(self, cache: Cache, n_cand: int, tail_cap: int, stream=None,
+                 kernel: int = 0):
+        """kernel: 0 the library's choice, 1 candidate-batched, 2 chunked,
+        3 one CTA per unit, 4 generic (kvr_fork_set_kernel)."""
         self.cache, self.N, self.tcap = cache, n_cand, tail_cap
         self.nbytes = kvr_fork_required_bytes(cache.handle, n_cand, tail_cap)
         if self.nbytes == 0:
@@ -368,6 +376,8 @@ class Fork:
                                device=cache.buf.device)
         self.handle = kvr_fork_candidates(cache.handle, n_cand, tail_cap,
                                           self.buf, self.nbytes, stream)
+        if kernel:
+            kvr_fork_set_kernel(self.handle, kernel)
 
     def __del__(self):
         h = getattr(self, "handle", None)

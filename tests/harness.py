@@ -77,7 +77,7 @@ def _unit_map(pos, score):
 
 def fork_lockstep(c: kvr.Cache, o: orc.OracleCache, w: inputs.Workload,
                   seed: int, n_cand: int, steps: int, budget: int, window: int,
-                  pick_step: int = 0, tail_cap=None):
+                  pick_step: int = 0, tail_cap=None, kernel: int = 0):
     """Fork both sides into n_cand candidates, decode `steps` tokens per
     candidate checking every candidate after every token (outputs; scores of
     every prefix and tail row, by position), then commit a seeded pick (the
@@ -85,7 +85,7 @@ def fork_lockstep(c: kvr.Cache, o: orc.OracleCache, w: inputs.Workload,
     Returns (oracle after commit, chosen, stats)."""
     S = c.S
     parent_pos = [c.export(s, kv=False) for s in range(S)]
-    f = kvr.Fork(c, n_cand, tail_cap or steps)
+    f = kvr.Fork(c, n_cand, tail_cap or steps, kernel=kernel)
     cands = o.fork(n_cand)
     stats = parity.Stats()
     for t in range(steps):

@@ -24,18 +24,14 @@ def _cuda():
     torch.cuda.set_device(0)
 
 
-# The candidate kernels: the chunked persistent kernel (default), the
-# one-CTA-per-unit tensor-core kernel, and the generic kernels.
-PATHS = {"chunked": dict(fused=True, chunk=(0, 0)),
-         "mma": dict(fused=True, chunk=(-1, 0)),
-         "generic": dict(fused=False, chunk=(0, 0))}
+# The candidate kernels (kvr_fork_set_kernel): candidate-batched (the
+# default), chunked, one CTA per unit, generic.
+PATHS = {"batch": 1, "chunked": 2, "mma": 3, "generic": 4}
 
 
-def _evicted_pair(w, seed, S, cap, prompt_lens, warm_steps, path="chunked"):
-    """Load prompts and run evicting steps so the parent sits at B + W rows;
-    the parent (and its forks) run on the kernels `path` names."""
-    c, o = harness.make_pair(w, seed, S, cap=cap, prompt_lens=prompt_lens,
-                             **PATHS[path])
+def _evicted_pair(w, seed, S, cap, prompt_lens, warm_steps):
+    """Load prompts and run evicting steps so the parent sits at B + W rows."""
+    c, o = harness.make_pair(w, seed, S, cap=cap, prompt_lens=prompt_lens)
     harness.lockstep(c, o, w, seed, warm_steps, w.budget, w.window)
     return c, o
 
@@ -46,11 +42,10 @@ def test_small_fork_commit_then_continue(n_cand, path):
     """Tail lengths cross the 16-row tile and 32-row chunk boundaries (7
     tokens from a ragged parent, 37 for N = 8)."""
     w = inputs.Workload("f", 2, 2, 3, 128, "bf16", 12, 4, 30, 0, sigma=1.0)
-    c, o = _evicted_pair(w, 21, 2, cap=60, prompt_lens=[30, 9], warm_steps=3,
-                         path=path)
+    c, o = _evicted_pair(w, 21, 2, cap=60, prompt_lens=[30, 9], warm_steps=3)
     o2, chosen, st = harness.fork_lockstep(c, o, w, 21, n_cand,
                                            37 if n_cand == 8 else 7, w.budget,
-                                           w.window)
+                                           w.window, kernel=PATHS[path])
     assert (c.lengths() == np.minimum(o2.len.max(axis=2), 16)).all()
     # the committed parent keeps decoding in lock-step
     harness.lockstep(c, o2, w, 21, 4, w.budget, w.window, step0=100)
@@ -114,34 +109,49 @@ def test_single_candidate_equals_plain_deferred_eviction():
                     assert abs(ma[p] - mb[p]) <= 1e-4 * max(abs(mb[p]), 1e-6)
 
 
-@pytest.mark.parametrize("path", ["chunked", "mma"])
+@pytest.mark.parametrize("path", ["batch", "chunked", "mma"])
 def test_7b_best_of_4(path):
     """7B geometry stepwise best-of-4: an evicted cache (prompt 512, B=128,
     W=8; heavy keys), forked to 4 candidates that decode a 16-token step
     sharing the prefix, then re-evicted and committed."""
     w = inputs.WORKLOADS["7b_bon4"]
     c, o = _evicted_pair(w, 25, 1, cap=w.prompt + 1, prompt_lens=[w.prompt],
-                         warm_steps=2, path=path)
+                         warm_steps=2)
     o2, chosen, st = harness.fork_lockstep(c, o, w, 25, w.n_cand, 16, w.budget,
-                                           w.window)
+                                           w.window, kernel=PATHS[path])
     assert (c.lengths() == w.budget + w.window).all()
 
 
-def test_72b_best_of_8():
+@pytest.mark.parametrize("path", ["batch", "chunked"])
+def test_72b_best_of_8(path):
     """72B geometry (80 layers, 8 KV heads, G=8), B=64, N=8 candidates, an
     8-token step (reduced from 64 to keep the oracle fast)."""
     w = inputs.Workload("72b_small", 80, 8, 8, 128, "bf16", 64, 8, 200, 0,
                         sigma=1.0 / np.sqrt(128.0))
     c, o = _evicted_pair(w, 26, 1, cap=w.prompt + 1, prompt_lens=[w.prompt],
                          warm_steps=1)
-    harness.fork_lockstep(c, o, w, 26, 8, 8, w.budget, w.window)
+    harness.fork_lockstep(c, o, w, 26, 8, 8, w.budget, w.window,
+                          kernel=PATHS[path])
     assert (c.lengths() == w.budget + w.window).all()
 
 
-def test_fork_empty_prefix_and_chunk_edges():
-    """A parent with no live rows (empty prompt: the prefix segment is empty)
-    and one whose prefix is an exact multiple of the 32-row chunk, forked and
-    decoded so the tails cross 32 rows, then committed."""
+@pytest.mark.parametrize("path", ["batch", "chunked"])
+def test_fork_empty_prefix_and_block_edges(path):
+    """A parent with no live rows (an empty prefix) and one whose prefix is
+    an exact multiple of the 32-row chunk, with 2 and 3 candidates (tail
+    blocks of 64 and 32 rows per candidate), decoded so the tails cross 32
+    and 64 rows, then committed."""
     w = inputs.Workload("fe", 1, 2, 2, 128, "bf16", 24, 8, 0, 0, sigma=1.0)
-    c, o = harness.make_pair(w, 27, 2, cap=80, prompt_lens=[0, 32])
-    harness.fork_lockstep(c, o, w, 27, 2, 34, w.budget, w.window)
+    for n_cand in (2, 3):
+        c, o = harness.make_pair(w, 27, 2, cap=110, prompt_lens=[0, 32])
+        harness.fork_lockstep(c, o, w, 27, n_cand, 70, w.budget, w.window,
+                              kernel=PATHS[path])
+
+
+def test_fork_prefix_longer_than_a_block():
+    """A prefix of 200 rows (a full 128-row prefix block and a partial one in
+    the candidate-batched kernel) with 4 candidates."""
+    w = inputs.Workload("fl", 1, 1, 3, 128, "bf16", 1 << 20, 0, 0, 0, sigma=1.0)
+    c, o = harness.make_pair(w, 28, 1, cap=240, prompt_lens=[200])
+    harness.fork_lockstep(c, o, w, 28, 4, 12, w.budget, w.window,
+                          kernel=PATHS["batch"])
