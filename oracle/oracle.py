@@ -126,6 +126,23 @@ class OracleCache:
                            for k, v in self.__dict__.items()})
         return c
 
+    def resized(self, cap) -> "OracleCache":
+        """The same state in a cache of capacity `cap` (at least every live
+        length); rows are compacted, so only slots [0, cap) are kept.  Data
+        movement only: lets long runs fork small copies after the first
+        eviction."""
+        if cap < int(self.len.max(initial=0)):
+            raise ValueError("capacity below a live length")
+        c = OracleCache(self.S, self.L, self.H, self.G, self.d, cap, self.scale)
+        k = min(cap, self.cap)
+        c.K[..., :k, :] = self.K[..., :k, :]
+        c.V[..., :k, :] = self.V[..., :k, :]
+        c.score[..., :k] = self.score[..., :k]
+        c.pos[..., :k] = self.pos[..., :k]
+        c.len[...] = self.len
+        c.next_pos[...] = self.next_pos
+        return c
+
     def load(self, seq, k, v, first_pos=0, scores=None):
         """Prompt rows [L][H][n][d] with positions first_pos.. and score 0."""
         n = k.shape[2]

@@ -391,3 +391,24 @@ def test_tiny_workload_invariants():
             live = set(c.pos[idx][:c.len[idx]].tolist())
             assert set(range(newest - w.window + 1, newest + 1)) <= live
     np.testing.assert_allclose(live_sum() + evicted, w.steps, rtol=1e-11)
+
+
+def test_resized_oracle_steps_identically():
+    """OracleCache.resized only moves data: a resized copy takes the same
+    next step (outputs, scores, retained rows) as the original."""
+    w = inputs.Workload("rs", 2, 2, 3, 16, "f32", 6, 2, 20, 0, sigma=1.0)
+    o = orc.OracleCache(1, 2, 2, 3, 16, cap=21)
+    k, v = inputs.prompt(w, 5, 0, 20)
+    o.load(0, k, v)
+    o.step(*inputs.step_inputs(w, 5, 0, 1), B=6, W=2)
+    r = o.resized(9)
+    q, kn, vn = inputs.step_inputs(w, 5, 1, 1)
+    a = o.step(q, kn, vn, B=6, W=2)
+    b = r.step(q, kn, vn, B=6, W=2)
+    assert np.array_equal(a, b)
+    for l in range(2):
+        for h in range(2):
+            for x, y in zip(o.unit_rows(0, l, h), r.unit_rows(0, l, h)):
+                assert np.array_equal(x, y)
+    with pytest.raises(ValueError):
+        o.resized(5)
