@@ -64,7 +64,8 @@ def parse():
     p.add_argument("--fused-groups", type=int, default=0,
                    help="units computed at once per SM by the fused kernel "
                         "(0: the library's choice)")
-    p.add_argument("--mode", default="step", choices=["step", "helper", "fork"],
+    p.add_argument("--mode", default="step",
+                   choices=["step", "helper", "fork", "crossover"],
                    help="step: the evicted decode step (the headline); "
                         "helper: full-context decode of the 1.5B helper at "
                         "16k context; fork: 72B best-of-8 candidate step")
@@ -487,6 +488,102 @@ def run_helper(args):
                 kernel="kvr_decode_attend (split partials + combine)")
 
 
+def run_crossover(args):
+    """The attention-side crossover of App. C (Eq. 14) measured on this GPU
+    at 7B geometry: full-context decode attention (append + attention over
+    every row, no scores; kvr_decode_attend) against the evicted step
+    (append + attention + scores + selection + compaction over B' = B + W
+    rows; kvr_decode_step), both over all 28 layers of S sequences.
+    t_full(l) is measured at contexts from 64 to 16384 and fitted as
+    a + b l; alpha = t_evict / t_full(B') - 1 and l* = (t_evict - a) / b,
+    the context past which the evicted step is the cheaper one."""
+    import torch
+    from paper_2608_15797_gb300 import kvr
+    w = inputs.WORKLOADS["7b_b64"]
+    S = args.seqs or 16
+    L, H, G, d = w.n_layers, w.n_kv_heads, w.group, w.head_dim
+    dev = torch.device("cuda", 0)
+    stream = torch.cuda.current_stream(dev)
+    K, Wm = max(1, min(args.steps, 40)), max(3, args.warmup)
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(args.seed + 31)
+
+    def inputs_for(S):
+        q = (torch.randn(S, L, H * G, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+        kn = (torch.randn(S, L, H, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+        vn = (torch.randn(S, L, H, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+        return q, kn, vn
+
+    def loaded(rows, cap):
+        cache = kvr.Cache(S, L, H, G, d, cap, "bf16", "bf16", device=dev)
+        for s in range(S):
+            k = (torch.randn(L, H, rows, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+            v = (torch.randn(L, H, rows, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+            cache.load(s, k, v)
+            del k, v
+        return cache
+
+    def timed(fn):
+        for i in range(Wm):
+            fn()
+        torch.cuda.synchronize()
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        t0.record(stream)
+        for i in range(K):
+            fn()
+        t1.record(stream)
+        torch.cuda.synchronize()
+        return t0.elapsed_time(t1) * 1e3 / K  # us per call
+
+    q, kn, vn = inputs_for(S)
+    out = torch.empty(S, L, H * G, d, dtype=torch.bfloat16, device=dev)
+    full = []
+    drift = Wm + (K + 1) // 2  # each call appends a row: centre the mean
+    for target in (72, 128, 256, 512, 640, 1024, 2048, 4096, 8192, 16384):
+        ell = target - drift
+        cache = loaded(ell, ell + Wm + K + 1)
+        need = kvr.kvr_decode_attend_workspace_bytes(cache.handle, 0, L, 0)
+        ws = torch.empty(max(need, 16), dtype=torch.uint8, device=dev)
+        t = timed(lambda: kvr.kvr_decode_attend(cache.handle, 0, L, q, kn, vn,
+                                                out, 0, ws, ws.numel(), stream))
+        cache.sync_status()
+        # mean rows attended over the timed calls
+        full.append((ell + Wm + (K + 1) / 2.0, t))
+        del cache, ws
+    evict = {}
+    for B, Wn in ((64, 8), (512, 128)):
+        cache = loaded(B + Wn, B + Wn + 1)
+        t = timed(lambda: kvr.kvr_decode_step(cache.handle, 0, L, q, kn, vn, out,
+                                              B, Wn, stream))
+        cache.sync_status()
+        evict[B + Wn] = t
+        del cache
+    ls = np.array([x for x, _ in full])
+    ts = np.array([y for _, y in full])
+    fit = ls >= 512  # the bandwidth-bound part of the curve
+    b, a = np.polyfit(ls[fit], ts[fit], 1)
+    res = {}
+    for bp, te in evict.items():
+        t_bp = float(np.interp(bp, ls, ts))
+        # first context at which full attention costs as much as the step
+        above = np.nonzero(ts >= te)[0]
+        if len(above) and above[0] > 0:
+            i = above[0]
+            lstar = float(ls[i - 1] + (te - ts[i - 1]) * (ls[i] - ls[i - 1]) /
+                          (ts[i] - ts[i - 1]))
+        elif len(above):
+            lstar = float(ls[0])
+        else:
+            lstar = float((te - a) / b)
+        res[bp] = {"t_evict_us": te, "t_full_at_Bphys_us": t_bp,
+                   "alpha": te / t_bp - 1.0, "lstar_rows": lstar,
+                   "lstar_over_Bphys": lstar / bp}
+    return dict(full=[{"context": float(x), "us_per_step": float(y)} for x, y in full],
+                fit={"a_us": float(a), "b_us_per_row": float(b)}, res=res, S=S,
+                K=K)
+
+
 def run_fork(args):
     """72B geometry (80 layers, 64 q / 8 kv heads, d 128), B=64, W=8: an
     evicted parent (B+W rows) forked to 8 candidates; one timed step is one
@@ -611,6 +708,27 @@ def main():
         return 0
 
     import torch
+    if args.mode == "crossover":
+        if rank == 0:
+            r = run_crossover(args)
+            r640, r72 = r["res"][640], r["res"][72]
+            print(json.dumps({
+                "metric": "attention-side crossover context l* at B'=640 "
+                          "(7B geometry, Eq. 14; lower: eviction pays sooner)",
+                "value": r640["lstar_rows"], "unit": "rows", "n_gpus": 1,
+                "steps": r["K"], "warmup": args.warmup,
+                "higher_is_better": False, "scaling": "weak",
+                "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+                "config": {"workload": "7b crossover", "n_seq": r["S"],
+                           "layers": 28, "kv_heads": 4, "group": 7,
+                           "head_dim": 128},
+                "alpha_640": r640["alpha"], "crossover_72": r72,
+                "crossover_640": r640, "full_context": r["full"],
+                "fit": r["fit"],
+                "paper": {"lstar_rows": 2500, "alpha": 2.9, "B_phys": 640,
+                          "note": "the paper's measurement on its own "
+                                  "system, end to end; context only"}}))
+        return 0
     if args.mode != "step":
         if rank == 0:
             r = run_helper(args) if args.mode == "helper" else run_fork(args)
