@@ -190,6 +190,28 @@ class OracleCache:
             arr[:, lb:le] = new
         return out.reshape(S, nl, H * G, d)
 
+    def absorb(self, q, k_new, v_new, B=0, W=0, evict=True, layer_begin=None,
+               layer_end=None):
+        """c tokens of every sequence in one call: the reading of Alg. 1's
+        single forward pass of the base model over an accepted helper step
+        (and of a prompt prefill whose attention seeds the scores).  Token j
+        is appended and attends every live row and the chunk's rows 0..j
+        (causal), adding its head-mean probabilities to the scores of every
+        row it attends -- c decode steps with the eviction to B + W applied
+        once, after the last.
+
+        q: [S][nl][c][H*G][d]; k_new, v_new: [S][nl][c][H][d].  Returns out
+        [S][nl][c][H*G][d].
+        """
+        lb, le = self._layers(layer_begin, layer_end)
+        c = q.shape[2]
+        outs = [self.step(q[:, :, j], k_new[:, :, j], v_new[:, :, j],
+                          evict=False, layer_begin=lb, layer_end=le)
+                for j in range(c)]
+        if evict:
+            self.evict(B, W, lb, le)
+        return np.stack(outs, axis=2)
+
     def evict(self, B, W, layer_begin=None, layer_end=None):
         lb, le = self._layers(layer_begin, layer_end)
         sub = [np.ascontiguousarray(a[:, lb:le]) for a in

@@ -412,3 +412,76 @@ def test_resized_oracle_steps_identically():
                 assert np.array_equal(x, y)
     with pytest.raises(ValueError):
         o.resized(5)
+
+
+# --------------------------------------------------------------------------
+# Absorbing a chunk (a token block attended causally in one call)
+# --------------------------------------------------------------------------
+
+def _chunk(rng, c, H, G, d):
+    q = rng.standard_normal((1, 1, c, H * G, d))
+    kn = rng.standard_normal((1, 1, c, H, d))
+    vn = rng.standard_normal((1, 1, c, H, d))
+    return q, kn, vn
+
+
+def test_absorb_equals_masked_sdpa_and_column_sums():
+    """Against the library: outputs are SDPA with a mask that lets token j
+    see every prompt row and chunk rows 0..j; scores are the column sums over
+    the chunk's tokens of the head-mean probabilities (SDPA with identity
+    values); each token adds exactly 1 per KV head."""
+    H, G, d, P, c = 2, 3, 16, 5, 6
+    rng = np.random.default_rng(21)
+    o = orc.OracleCache(1, 1, H, G, d, cap=P + c)
+    kp = rng.standard_normal((1, H, P, d))
+    vp = rng.standard_normal((1, H, P, d))
+    o.load(0, kp, vp)
+    q, kn, vn = _chunk(rng, c, H, G, d)
+    out = o.absorb(q, kn, vn, evict=False)
+    n = P + c
+    mask = torch.zeros(c, n, dtype=torch.bool)
+    for j in range(c):
+        mask[j, :P + j + 1] = True
+    for h in range(H):
+        K = torch.from_numpy(np.concatenate([kp[0, h], kn[0, 0, :, h]]))
+        V = torch.from_numpy(np.concatenate([vp[0, h], vn[0, 0, :, h]]))
+        Q = torch.from_numpy(np.ascontiguousarray(
+            q[0, 0, :, h * G:(h + 1) * G].transpose(1, 0, 2)))  # [G, c, d]
+        ref = F.scaled_dot_product_attention(Q, K[None].expand(G, n, d),
+                                             V[None].expand(G, n, d),
+                                             attn_mask=mask)
+        np.testing.assert_allclose(out[0, 0, :, h * G:(h + 1) * G],
+                                   ref.numpy().transpose(1, 0, 2),
+                                   rtol=1e-12, atol=1e-13)
+        eye = torch.eye(n, dtype=torch.float64)
+        prob = F.scaled_dot_product_attention(Q, K[None].expand(G, n, d),
+                                              eye[None].expand(G, n, n),
+                                              attn_mask=mask)  # [G, c, n]
+        want = prob.mean(0).sum(0).numpy()
+        np.testing.assert_allclose(o.score[0, 0, h, :n], want, rtol=1e-12,
+                                   atol=1e-14)
+        assert abs(o.score[0, 0, h, :n].sum() - c) < 1e-12
+    assert (o.len == n).all() and (o.next_pos == n).all()
+
+
+def test_absorb_then_evict_keeps_the_brute_force_set():
+    """After a chunk, the unit is cut to B + W once: the W newest positions
+    plus the top B of the rest under (score desc, position asc), found here
+    by subset enumeration on the pre-eviction scores."""
+    H, G, d, B, W = 2, 2, 8, 3, 2
+    rng = np.random.default_rng(22)
+    for P, c in ((4, 5), (0, 7), (6, 1), (2, 3)):
+        o = orc.OracleCache(1, 1, H, G, d, cap=P + c)
+        if P:
+            o.load(0, rng.standard_normal((1, H, P, d)),
+                   rng.standard_normal((1, H, P, d)))
+        q, kn, vn = _chunk(rng, c, H, G, d)
+        keep = o.copy()
+        keep.absorb(q, kn, vn, evict=False)
+        o.absorb(q, kn, vn, B=B, W=W)
+        for h in range(H):
+            n = P + c
+            sc, ps = keep.score[0, 0, h, :n], keep.pos[0, 0, h, :n]
+            want = {int(ps[i]) for i in _brute_keep(list(sc), list(ps), B, W)}
+            got = set(o.pos[0, 0, h, :o.len[0, 0, h]].tolist())
+            assert got == want
