@@ -250,6 +250,27 @@ kvr_status kvr_cache_set_fused_tuning(kvr_cache *cache, int groups,
 kvr_status kvr_cache_set_chunk_tuning(kvr_cache *cache, int groups,
                                       int stages);
 
+/* Absorb a chunk of `chunk` tokens per sequence in one call, and optionally
+ * cut every unit back to B + W once afterwards (Algorithm 1: when a helper
+ * step is accepted, the base model encodes its tokens in a single forward
+ * pass, so its KV absorbs the step; a prompt absorbed into an empty cache
+ * seeds the scores with its prefill attention).  The result is that of
+ * `chunk` kvr_decode_attend_score calls followed by one kvr_evict_compact:
+ * token j is appended as a new row and attends every live row and the
+ * chunk's rows 0..j (causal), adding the head-mean of its probabilities to
+ * the accumulated score of every row it attends (Sec. 2.1); then, if evict
+ * != 0, each unit keeps its W most recent positions and the best B others
+ * (score descending, position ascending; Eq. 1).
+ *   q:     [S][layer_end - layer_begin][chunk][H * G][d]
+ *   k_new: [S][layer_end - layer_begin][chunk][H][d]  (v_new likewise)
+ *   out:   [S][layer_end - layer_begin][chunk][H * G][d], out_dtype
+ * Every unit must have room for the chunk (live + chunk <= capacity), else
+ * KVR_ECAPACITY before anything runs.  Stream-ordered. */
+kvr_status kvr_absorb_chunk(kvr_cache *cache, int layer_begin, int layer_end,
+                            int chunk, const void *q, const void *k_new,
+                            const void *v_new, void *out, int budget,
+                            int window, int evict, void *stream);
+
 /* ---- the same step for callers that cannot allocate -------------------- */
 
 /* The paper has no counterpart to this call: it is a deployment variant.

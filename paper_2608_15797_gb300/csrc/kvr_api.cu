@@ -689,6 +689,44 @@ kvr_status kvr_evict_compact(kvr_cache *c, int lb, int le, int budget,
   return KVR_OK;
 }
 
+kvr_status kvr_absorb_chunk(kvr_cache *c, int lb, int le, int chunk,
+                            const void *q, const void *k_new,
+                            const void *v_new, void *out, int budget,
+                            int window, int evict, void *stream) {
+  if (!c) return fail(KVR_EINVAL, "null cache");
+  if (c->forks) return fail(KVR_ESTATE, "the cache has a live fork");
+  kvr_status st = check_layers(c, lb, le);
+  if (st != KVR_OK) return st;
+  if (!q || !k_new || !v_new || !out)
+    return fail(KVR_EINVAL, "null q, k_new, v_new or out");
+  if (chunk < 1) return fail(KVR_EINVAL, "chunk of %d tokens", chunk);
+  if (evict) {
+    st = check_evict(budget, window);
+    if (st != KVR_OK) return st;
+  }
+  const int m = max_len(c, lb, le);
+  if ((long long)m + chunk > c->desc.capacity)
+    return fail(KVR_ECAPACITY, "a unit holds %d rows; %d more exceed capacity "
+                "%d", m, chunk, c->desc.capacity);
+  for (int s = 0; s < c->desc.n_seq; ++s)
+    for (int l = lb; l < le; ++l)
+      if ((long long)c->next_pos[(size_t)s * c->desc.n_layers + l] + chunk >=
+          INT32_MAX)
+        return fail(KVR_ECAPACITY, "position counter exhausted");
+  // Token by token: each launch appends token j of every unit and attends
+  // over every live row, adding to the scores (eviction deferred).
+  for (int j = 0; j < chunk; ++j) {
+    StepArgs a = step_args(c, lb, le, q, k_new, v_new, out);
+    a.chunk = chunk;
+    a.tok = j;
+    cudaError_t e = kvr::launch_attend_score_generic(c->view, a, as_stream(stream));
+    if (e != cudaSuccess) return cuda_fail("kvr_absorb_chunk", e);
+    c->launches += 1;
+    mirror_append(c, lb, le);
+  }
+  return evict ? kvr_evict_compact(c, lb, le, budget, window, stream) : KVR_OK;
+}
+
 kvr_status kvr_decode_step(kvr_cache *c, int lb, int le, const void *q,
                            const void *k_new, const void *v_new, void *out,
                            int budget, int window, void *stream) {

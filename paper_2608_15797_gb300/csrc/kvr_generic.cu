@@ -77,7 +77,8 @@ __global__ void __launch_bounds__(kThreads)
   T *Vu = reinterpret_cast<T *>(c.V) + x.u * (size_t)c.cap * D;
   float *su = c.score + x.u * (size_t)c.sstride;
   int32_t *pu = c.pos + x.u * (size_t)c.sstride;
-  const size_t kv_row = ((size_t)x.s * a.nl + x.lr) * c.H + x.h;
+  const size_t kv_row =
+      (((size_t)x.s * a.nl + x.lr) * a.chunk + a.tok) * c.H + x.h;
   const size_t q_row = kv_row * G;
   const T *qg = reinterpret_cast<const T *>(a.q) + q_row * D;
   const T *kn = reinterpret_cast<const T *>(a.k_new) + kv_row * D;

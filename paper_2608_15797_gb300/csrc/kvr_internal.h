@@ -72,6 +72,9 @@ struct StepArgs {
   int max_rows;       // largest live length after the append over the units
   int budget, window; // eviction target (evict only when evict != 0)
   int evict;
+  // Inputs holding `chunk` tokens per (sequence, layer) row, [S][nl][chunk]
+  // [...] (kvr_absorb_chunk); this call reads token `tok` of each.
+  int chunk = 1, tok = 0;
 };
 
 // Generic kernels (any d in {64,128}, G <= 8, fp32 or bf16): one CTA per unit.

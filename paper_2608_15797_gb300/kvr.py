@@ -62,6 +62,7 @@ _SIGS = {
     "kvr_decode_attend_score_noalloc": (_S, [_P, _I, _I, _P, _P, _P, _P, _P]),
     "kvr_evict_compact": (_S, [_P, _I, _I, _I, _I, _P]),
     "kvr_decode_step": (_S, [_P, _I, _I, _P, _P, _P, _P, _I, _I, _P]),
+    "kvr_absorb_chunk": (_S, [_P, _I, _I, _I, _P, _P, _P, _P, _I, _I, _I, _P]),
     "kvr_cache_export": (_S, [_P, _I, _P, _P, _P, _P, _P, _P, _P]),
     "kvr_cache_lengths": (_S, [_P, _P]),
     "kvr_cache_launch_count": (_S, [_P, _P]),
@@ -166,6 +167,14 @@ def kvr_decode_step(h, layer_begin, layer_end, q, k_new, v_new, out, budget,
                                _stream(stream)), "kvr_decode_step")
 
 
+def kvr_absorb_chunk(h, layer_begin, layer_end, chunk, q, k_new, v_new, out,
+                     budget, window, evict=True, stream=None):
+    _check(lib.kvr_absorb_chunk(h, layer_begin, layer_end, chunk, _ptr(q),
+                                _ptr(k_new), _ptr(v_new), _ptr(out), budget,
+                                window, 1 if evict else 0, _stream(stream)),
+           "kvr_absorb_chunk")
+
+
 def kvr_cache_export(h, seq, host_k, host_v, host_score, host_pos, host_len,
                      host_next_pos, stream=None):
     _check(lib.kvr_cache_export(h, seq, _ptr(host_k), _ptr(host_v),
@@ -268,6 +277,19 @@ class Cache:
         out = self.new_out(le - lb) if out is None else out
         kvr_decode_step(self.handle, lb, le, q, k_new, v_new, out, budget,
                         window, stream)
+        return out
+
+    def absorb(self, q, k_new, v_new, budget=0, window=0, evict=True,
+               out=None, layers=None, stream=None):
+        """q [S][nl][c][H*G][d], k_new/v_new [S][nl][c][H][d] -> out
+        [S][nl][c][H*G][d] (kvr_absorb_chunk)."""
+        lb, le = self._layers(layers)
+        c = q.shape[2]
+        if out is None:
+            out = torch.empty(self.S, le - lb, c, self.H * self.G, self.d,
+                              dtype=self.out_torch_dtype, device=self.buf.device)
+        kvr_absorb_chunk(self.handle, lb, le, c, q, k_new, v_new, out, budget,
+                         window, evict, stream)
         return out
 
     def lengths(self):

@@ -1,0 +1,98 @@
+"""Absorbing a chunk of tokens (kvr_absorb_chunk) against the oracle: c
+tokens attended causally in one call, scores accumulated from every token,
+one eviction to B + W at the end; then ordinary decode steps continue from
+the resulting state in lock-step."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import parity
+from paper_2608_15797_gb300 import inputs, kvr
+from tests import harness
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(autouse=True)
+def _cuda():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA device")
+    torch.cuda.set_device(0)
+
+
+def absorb_lockstep(c, o, w, seed, chunk, B, W, evict=True, step0=20_000):
+    """One absorb call on both sides, checking every token's output, then the
+    retained rows and scores of every unit."""
+    S = c.S
+    toks = [inputs.step_inputs(w, seed, step0 + j, S) for j in range(chunk)]
+    q, kn, vn = (np.stack([t[i] for t in toks], axis=2) for i in range(3))
+    out = c.absorb(harness.dev(q, w.dtype), harness.dev(kn, w.dtype),
+                   harness.dev(vn, w.dtype), B, W, evict=evict)
+    ref = o.absorb(q, kn, vn, B=B, W=W, evict=False)
+    torch.cuda.synchronize()
+    got = out.float().cpu().numpy()
+    for j in range(chunk):
+        parity.check_out(got[:, :, j], ref[:, :, j], what=f"token {j} of the chunk")
+    exports = [c.export(s, kv=False) for s in range(S)]
+    st = parity.check_and_adopt(o, exports, B, W, evict=evict)
+    c.sync_status()
+    return st
+
+
+@pytest.mark.parametrize("G,d,dtype", [(7, 128, "bf16"), (1, 128, "bf16"),
+                                       (8, 128, "bf16"), (3, 64, "f32")])
+@pytest.mark.parametrize("chunk", [1, 5, 33])
+def test_absorb_shapes(G, d, dtype, chunk):
+    """Ragged units (an empty one included), chunks crossing tile ends, then
+    three decode steps."""
+    B, W = 12, 4
+    w = inputs.Workload("ab", 2, 2, G, d, dtype, B, W, 20, 0, sigma=1.0)
+    c, o = harness.make_pair(w, 50, 3, cap=20 + chunk + 4,
+                             prompt_lens=[20, 0, 9])
+    absorb_lockstep(c, o, w, 50, chunk, B, W)
+    harness.lockstep(c, o, w, 50, 3, B, W, step0=100)
+
+
+def test_absorb_without_eviction_grows_every_unit():
+    w = inputs.Workload("ab", 1, 2, 4, 128, "bf16", 8, 2, 10, 0, sigma=1.0)
+    c, o = harness.make_pair(w, 51, 2, cap=40, prompt_lens=[10, 3])
+    absorb_lockstep(c, o, w, 51, 17, 8, 2, evict=False)
+    assert c.lengths().tolist() == [[27], [20]]
+
+
+def test_absorb_7b_helper_step():
+    """7B geometry (28 layers, G=7), an evicted cache at B+W = 72 rows absorbs
+    an accepted 64-token step in one call, evicts back to 72, then decodes."""
+    w = inputs.WORKLOADS["7b_unscaled"]
+    B, W = w.budget, w.window
+    c, o = harness.make_pair(w, 52, 2, cap=B + W + 64 + 1,
+                             prompt_lens=[B + W, B + W - 30])
+    absorb_lockstep(c, o, w, 52, 64, B, W)
+    assert (c.lengths() <= B + W).all()
+    harness.lockstep(c, o, w, 52, 4, B, W, step0=200)
+
+
+def test_absorb_prompt_seeds_scores():
+    """An empty cache absorbs a 200-token prompt: the scores it keeps are the
+    prompt's own causal attention (not zeros), and the cut to B + W keeps
+    the window and the best-attended rows."""
+    w = inputs.Workload("pp", 2, 2, 7, 128, "bf16", 24, 8, 0, 0, sigma=1.0)
+    c, o = harness.make_pair(w, 53, 2, cap=201, prompt_lens=[0, 0])
+    absorb_lockstep(c, o, w, 53, 200, w.budget, w.window)
+    e = c.export(0, kv=False)
+    assert (e["len"] == 32).all()
+    assert (e["score"][:, :, :32] > 0).all()
+
+
+def test_absorb_errors():
+    w = inputs.Workload("er", 1, 1, 2, 128, "bf16", 4, 2, 8, 0, sigma=1.0)
+    c, _ = harness.make_pair(w, 54, 1, cap=12)
+    q = torch.zeros(1, 1, 5, 2, 128, dtype=torch.bfloat16, device="cuda")
+    k = torch.zeros(1, 1, 5, 1, 128, dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(kvr.KvrError) as e:
+        c.absorb(q, k, k, 4, 2)
+    assert e.value.status == kvr.KVR_ECAPACITY
+    with pytest.raises(kvr.KvrError) as e:
+        kvr.kvr_absorb_chunk(c.handle, 0, 1, 0, q, k, k, q, 4, 2)
+    assert e.value.status == kvr.KVR_EINVAL
+    assert c.lengths().tolist() == [[8]]
