@@ -713,6 +713,31 @@ kvr_status kvr_absorb_chunk(kvr_cache *c, int lb, int le, int chunk,
       if ((long long)c->next_pos[(size_t)s * c->desc.n_layers + l] + chunk >=
           INT32_MAX)
         return fail(KVR_ECAPACITY, "position counter exhausted");
+  const CacheView &v = c->view;
+  if (c->fused && v.kv_bf16 && v.d == 128 && v.G <= 8 &&
+      chunk <= kvr::absorb_max_chunk() && m + chunk <= kvr::absorb_max_rows() &&
+      aligned16(q) && aligned16(k_new) && aligned16(v_new) && aligned16(out)) {
+    kvr::AbsorbParams p{};
+    p.c = v;
+    p.q = static_cast<const __nv_bfloat16 *>(q);
+    p.k_new = static_cast<const __nv_bfloat16 *>(k_new);
+    p.v_new = static_cast<const __nv_bfloat16 *>(v_new);
+    p.out = out;
+    p.lb = lb;
+    p.nl = le - lb;
+    p.chunk = chunk;
+    p.budget = budget;
+    p.window = window;
+    p.evict = evict ? 1 : 0;
+    p.scale_log2e = v.scale * 1.4426950408889634f;
+    p.inv_g = 1.f / (float)v.G;
+    cudaError_t e = kvr::launch_absorb(p, as_stream(stream));
+    if (e != cudaSuccess) return cuda_fail("kvr_absorb_chunk", e);
+    c->launches += 1;
+    for (int j = 0; j < chunk; ++j) mirror_append(c, lb, le);
+    if (evict) mirror_evict(c, lb, le, budget, window);
+    return KVR_OK;
+  }
   // Token by token: each launch appends token j of every unit and attends
   // over every live row, adding to the scores (eviction deferred).
   for (int j = 0; j < chunk; ++j) {

@@ -216,6 +216,20 @@ cudaError_t launch_fork_batch(const CUtensorMap &tmK, const CUtensorMap &tmV,
                               const ForkBatchParams &p, int grid,
                               cudaStream_t st);
 
+// Absorbing a chunk of tokens (kvr_absorb.cu): bf16, d = 128, G <= 8,
+// chunk <= absorb_max_chunk(), at most absorb_max_rows() rows after it.
+struct AbsorbParams {
+  CacheView c;
+  const __nv_bfloat16 *q, *k_new, *v_new;  // [S][nl][chunk][...][128]
+  void *out;
+  int lb, nl, chunk;
+  int budget, window, evict;
+  float scale_log2e, inv_g;
+};
+int absorb_max_chunk();
+int absorb_max_rows();
+cudaError_t launch_absorb(const AbsorbParams &p, cudaStream_t st);
+
 // Persistent chunked step (kvr_chunked.cu): bf16, d = 128, G <= 8, at most
 // chunk_max_rows() rows per job with the new row.  A job is one unit of the
 // cache (fork == 0: its live rows, the new row, at most one eviction) or one

@@ -39,35 +39,41 @@ def absorb_lockstep(c, o, w, seed, chunk, B, W, evict=True, step0=20_000):
     return st
 
 
+@pytest.mark.parametrize("fused", [True, False], ids=["fused", "tokenwise"])
 @pytest.mark.parametrize("G,d,dtype", [(7, 128, "bf16"), (1, 128, "bf16"),
                                        (8, 128, "bf16"), (3, 64, "f32")])
-@pytest.mark.parametrize("chunk", [1, 5, 33])
-def test_absorb_shapes(G, d, dtype, chunk):
+@pytest.mark.parametrize("chunk", [1, 5, 33, 64])
+def test_absorb_shapes(G, d, dtype, chunk, fused):
     """Ragged units (an empty one included), chunks crossing tile ends, then
-    three decode steps."""
+    three decode steps.  fused=False runs the token-by-token path."""
     B, W = 12, 4
     w = inputs.Workload("ab", 2, 2, G, d, dtype, B, W, 20, 0, sigma=1.0)
     c, o = harness.make_pair(w, 50, 3, cap=20 + chunk + 4,
-                             prompt_lens=[20, 0, 9])
+                             prompt_lens=[20, 0, 9], fused=fused)
     absorb_lockstep(c, o, w, 50, chunk, B, W)
     harness.lockstep(c, o, w, 50, 3, B, W, step0=100)
 
 
-def test_absorb_without_eviction_grows_every_unit():
+@pytest.mark.parametrize("fused", [True, False], ids=["fused", "tokenwise"])
+def test_absorb_without_eviction_grows_every_unit(fused):
     w = inputs.Workload("ab", 1, 2, 4, 128, "bf16", 8, 2, 10, 0, sigma=1.0)
-    c, o = harness.make_pair(w, 51, 2, cap=40, prompt_lens=[10, 3])
+    c, o = harness.make_pair(w, 51, 2, cap=40, prompt_lens=[10, 3], fused=fused)
     absorb_lockstep(c, o, w, 51, 17, 8, 2, evict=False)
     assert c.lengths().tolist() == [[27], [20]]
 
 
-def test_absorb_7b_helper_step():
+@pytest.mark.parametrize("fused", [True, False], ids=["fused", "tokenwise"])
+def test_absorb_7b_helper_step(fused):
     """7B geometry (28 layers, G=7), an evicted cache at B+W = 72 rows absorbs
     an accepted 64-token step in one call, evicts back to 72, then decodes."""
     w = inputs.WORKLOADS["7b_unscaled"]
     B, W = w.budget, w.window
     c, o = harness.make_pair(w, 52, 2, cap=B + W + 64 + 1,
-                             prompt_lens=[B + W, B + W - 30])
+                             prompt_lens=[B + W, B + W - 30], fused=fused)
+    n0 = c.launch_count()
     absorb_lockstep(c, o, w, 52, 64, B, W)
+    if fused:
+        assert c.launch_count() - n0 == 1  # one launch for the whole chunk
     assert (c.lengths() <= B + W).all()
     harness.lockstep(c, o, w, 52, 4, B, W, step0=200)
 
@@ -96,3 +102,12 @@ def test_absorb_errors():
         kvr.kvr_absorb_chunk(c.handle, 0, 1, 0, q, k, k, q, 4, 2)
     assert e.value.status == kvr.KVR_EINVAL
     assert c.lengths().tolist() == [[8]]
+
+
+def test_absorb_into_a_longer_than_budget_unit():
+    """Units above B + W before the chunk (a prompt loaded with zero scores):
+    the cut moves surviving old rows as well as placing new ones."""
+    w = inputs.Workload("lo", 1, 2, 5, 128, "bf16", 16, 4, 60, 0, sigma=1.0)
+    c, o = harness.make_pair(w, 55, 2, cap=100, prompt_lens=[60, 25])
+    absorb_lockstep(c, o, w, 55, 40, w.budget, w.window)
+    harness.lockstep(c, o, w, 55, 2, w.budget, w.window, step0=300)
