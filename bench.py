@@ -65,7 +65,7 @@ def parse():
                    help="units computed at once per SM by the fused kernel "
                         "(0: the library's choice)")
     p.add_argument("--mode", default="step",
-                   choices=["step", "helper", "fork", "crossover"],
+                   choices=["step", "helper", "fork", "crossover", "absorb"],
                    help="step: the evicted decode step (the headline); "
                         "helper: full-context decode of the 1.5B helper at "
                         "16k context; fork: 72B best-of-8 candidate step")
@@ -584,6 +584,68 @@ def run_crossover(args):
                 K=K)
 
 
+def run_absorb(args):
+    """An accepted 64-token step absorbed by the evicted 7B base model in one
+    call (kvr_absorb_chunk): 64 sequences x 28 layers, each unit at B+W = 72
+    rows takes 64 new rows with causal attention and accumulated scores, then
+    is cut back to 72.  One timed step = one call."""
+    import torch
+    from paper_2608_15797_gb300 import kvr
+    w = inputs.WORKLOADS["7b_b64"]
+    S = args.seqs or 64
+    L, H, G, d, B, Wn, C = w.n_layers, w.n_kv_heads, w.group, w.head_dim, w.budget, w.window, 64
+    dev = torch.device("cuda", 0)
+    cache = kvr.Cache(S, L, H, G, d, B + Wn + C, "bf16", "bf16", device=dev)
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(args.seed + 37)
+    for s in range(S):
+        k = (torch.randn(L, H, B + Wn, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+        v = (torch.randn(L, H, B + Wn, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+        cache.load(s, k, v)
+    pool = []
+    for _ in range(4):
+        q = (torch.randn(S, L, C, H * G, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+        kn = (torch.randn(S, L, C, H, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+        vn = (torch.randn(S, L, C, H, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+        pool.append((q, kn, vn))
+    out = torch.empty(S, L, C, H * G, d, dtype=torch.bfloat16, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step(i):
+        q, kn, vn = pool[i % 4]
+        kvr.kvr_absorb_chunk(cache.handle, 0, L, C, q, kn, vn, out, B, Wn, True,
+                             stream)
+
+    K, Wm = args.steps, max(3, args.warmup)
+    for i in range(Wm):
+        step(i)
+    torch.cuda.synchronize()
+    n0 = cache.launch_count()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for i in range(K):
+        step(i)
+    t1.record(stream)
+    torch.cuda.synchronize()
+    total = t0.elapsed_time(t1)
+    launches = cache.launch_count() - n0
+    cache.sync_status()
+    units = S * L * H
+    m = B + Wn
+    # bytes: old K/V rows read, new k/v read, kept new rows written (at most
+    # B + W of them, bounded by the chunk), q read, out written, scores and
+    # positions read and written, state
+    per_unit = (2 * m * d * 2 + 2 * C * d * 2 + 2 * min(C, m) * d * 2 +
+                2 * C * G * d * 2 + 8 * m + 8 * m + 16)
+    # flops: QK^T twice (statistics pass, probability pass) and PV (hi + lo
+    # terms) over the causal triangle's mean width m + C/2
+    flops = C * G * (m + C / 2.0) * d * 2 * (2 + 2)
+    return dict(total_ms=total, per_ms=total / max(1, launches), K=K,
+                launches=launches, launch_bytes=per_unit * units,
+                launch_flops=flops * units, S=S, C=C)
+
+
 def run_fork(args):
     """72B geometry (80 layers, 64 q / 8 kv heads, d 128), B=64, W=8: an
     evicted parent (B+W rows) forked to 8 candidates; one timed step is one
@@ -728,6 +790,39 @@ def main():
                 "paper": {"lstar_rows": 2500, "alpha": 2.9, "B_phys": 640,
                           "note": "the paper's measurement on its own "
                                   "system, end to end; context only"}}))
+        return 0
+    if args.mode == "absorb":
+        if rank == 0:
+            r = run_absorb(args)
+            peaks, peak_kind = measured_peaks()
+            sec = r["per_ms"] / 1e3
+            gbs = r["launch_bytes"] / sec / 1e9
+            tfs = r["launch_flops"] / sec / 1e12
+            print(json.dumps({
+                "metric": f"absorbed 64-token steps/s (7B geometry, B=64, W=8, "
+                          f"{r['S']} sequences x 28 layers per call)",
+                "value": r["K"] / (r["total_ms"] / 1e3), "unit": "calls/s",
+                "n_gpus": 1, "steps": r["K"], "warmup": args.warmup,
+                "ms_per_step": r["total_ms"] / r["K"], "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+                "data": "synthetic",
+                "config": {"workload": "7b absorb", "n_seq": r["S"], "layers": 28,
+                           "kv_heads": 4, "group": 7, "head_dim": 128,
+                           "chunk": r["C"], "budget": 64, "window": 8},
+                "tokens_per_s": r["K"] * r["S"] * r["C"] / (r["total_ms"] / 1e3),
+                "roofline": {"bound": "hbm", "achieved": gbs,
+                             "peak": float(peaks["hbm_gbs"]), "unit": "GB/s",
+                             "frac": gbs / float(peaks["hbm_gbs"]),
+                             "peak_kind": peak_kind, "traffic": None,
+                             "algorithmic_bytes_per_launch": r["launch_bytes"],
+                             "launch_ms": r["per_ms"],
+                             "kernel": "kvr_absorb_chunk"},
+                "tensor": {"achieved_tflops": tfs,
+                           "peak_tflops": float(peaks.get("bf16_tflops", 0)),
+                           "frac": tfs / float(peaks.get("bf16_tflops", 1)),
+                           "note": "mma.sync flops incl. the second QK pass "
+                                   "and the lo term of P"},
+                "gpu_launches": r["launches"]}))
         return 0
     if args.mode != "step":
         if rank == 0:

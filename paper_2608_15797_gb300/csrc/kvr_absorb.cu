@@ -40,6 +40,7 @@ using dev::kWarps;
 
 constexpr int kMaxChunk = 64;
 constexpr int kMaxRows = 192;
+static_assert(kMaxRows <= kThreads, "one row per thread in the selection");
 
 __device__ __forceinline__ void cp_async_commit_wait_all() {
   asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
@@ -58,7 +59,9 @@ struct AbsorbSmem {
   static constexpr int ps = sc + 4 * kMaxRows;         // positions
   static constexpr int acc = ps + 4 * kMaxRows;        // score increments
   static constexpr int lists = acc + 4 * kMaxRows;     // holes | movers
-  static constexpr int bytes = lists + 8 * kMaxRows;
+  static constexpr int key = lists + 8 * kMaxRows;     // selection keys
+  static constexpr int kept = key + 8 * kMaxRows;      // kept flags
+  static constexpr int bytes = kept + 4 * kMaxRows;
 };
 
 template <bool kOutBf16>
@@ -66,9 +69,7 @@ __global__ void __launch_bounds__(kThreads)
     absorb_kernel(const AbsorbParams p) {
   pdl_begin();
   extern __shared__ __align__(1024) unsigned char smem[];
-  __shared__ unsigned hist[256];
-  __shared__ unsigned long long s_prefix;
-  __shared__ int s_need, s_base, s_count;
+  __shared__ int s_base, s_count;
   __shared__ int s_wsum[kWarps];
   const CacheView &c = p.c;
   const int G = c.G, C = p.chunk;
@@ -153,18 +154,25 @@ __global__ void __launch_bounds__(kThreads)
     }
     // S tile for key rows [kt*16, kt*16 + 16): two n8 halves, scaled log2.
     auto logits = [&](int kt, float (&s)[2][4]) {
+      float s2[2][4];  // odd k-steps on a second chain
 #pragma unroll
       for (int hf = 0; hf < 2; ++hf)
-        s[hf][0] = s[hf][1] = s[hf][2] = s[hf][3] = 0.f;
+        s[hf][0] = s[hf][1] = s[hf][2] = s[hf][3] = s2[hf][0] = s2[hf][1] =
+            s2[hf][2] = s2[hf][3] = 0.f;
       const int kr = kt * 16 + (lane & 7) + ((lane >> 4) << 3);
 #pragma unroll
       for (int ks = 0; ks < 8; ++ks) {
         const int ch = 2 * ks + ((lane >> 3) & 1);
         uint32_t b0, b1, b2, b3;
         ldsm_x4(sK + swz(kr, ch), b0, b1, b2, b3);
-        mma_bf16(s[0], qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3], b0, b1);
-        mma_bf16(s[1], qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3], b2, b3);
+        float(&t)[2][4] = (ks & 1) ? s2 : s;
+        mma_bf16(t[0], qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3], b0, b1);
+        mma_bf16(t[1], qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3], b2, b3);
       }
+#pragma unroll
+      for (int hf = 0; hf < 2; ++hf)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) s[hf][e] += s2[hf][e];
 #pragma unroll
       for (int hf = 0; hf < 2; ++hf) {
         const int col = kt * 16 + hf * 8 + c2;
@@ -285,15 +293,26 @@ __global__ void __launch_bounds__(kThreads)
   const int B = p.budget, W = p.window;
   const bool cut = p.evict && n > B + W;
   const int wlo = t0 + C - 1 - W;  // a row is a candidate iff pos <= wlo
-  unsigned long long thr = ~0ull;
-  if (cut && B > 0)
-    thr = dev::block_select(
-        n, B, [&](int i) { return PS[i] <= wlo; },
-        [&](int i) { return dev::rank_key(SC[i], PS[i]); }, hist, &s_prefix,
-        &s_need);
-  auto keep = [&](int i) {
-    return !cut || PS[i] > wlo || (B > 0 && dev::rank_key(SC[i], PS[i]) >= thr);
-  };
+  // TopB by rank (n <= kMaxRows <= kThreads rows, one per thread): a
+  // candidate stays iff fewer than B candidates have a larger key (keys are
+  // distinct: positions are).  Rows outside the window-free set always stay.
+  unsigned long long *KEY = reinterpret_cast<unsigned long long *>(smem + AbsorbSmem::key);
+  int *KEPT = reinterpret_cast<int *>(smem + AbsorbSmem::kept);
+  for (int r = tid; r < n; r += kThreads)
+    KEY[r] = PS[r] <= wlo ? dev::rank_key(SC[r], PS[r]) : 0ull;
+  __syncthreads();
+  for (int r = tid; r < n; r += kThreads) {
+    int k = 1;
+    if (cut && PS[r] <= wlo) {
+      const unsigned long long mine_key = KEY[r];
+      int above = 0;
+      for (int j = 0; j < n; ++j) above += KEY[j] > mine_key ? 1 : 0;
+      k = above < B ? 1 : 0;
+    }
+    KEPT[r] = k;
+  }
+  __syncthreads();
+  auto keep = [&](int i) { return KEPT[i] != 0; };
   if (tid == 0) s_count = 0;
   __syncthreads();
   int mine = 0;
