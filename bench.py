@@ -65,10 +65,13 @@ def parse():
                    help="units computed at once per SM by the fused kernel "
                         "(0: the library's choice)")
     p.add_argument("--mode", default="step",
-                   choices=["step", "helper", "fork", "crossover", "absorb"],
+                   choices=["step", "helper", "fork", "crossover", "absorb",
+                            "entropy"],
                    help="step: the evicted decode step (the headline); "
                         "helper: full-context decode of the 1.5B helper at "
                         "16k context; fork: 72B best-of-8 candidate step")
+    p.add_argument("--entropy-dtype", default="bf16", choices=["bf16", "f32"],
+                   help="logit element type for --mode entropy")
     p.add_argument("--seqs", type=int, default=0,
                    help="sequences for --mode helper/fork (0: 16 / 4)")
     p.add_argument("--chunk-groups", type=int, default=0,
@@ -646,6 +649,90 @@ def run_absorb(args):
                 launch_flops=flops * units, S=S, C=C)
 
 
+def run_entropy(args):
+    """The detector's entropy test on the candidates' next-token logits:
+    64 problems x 8 candidates = 512 rows of 152,064 logits (Qwen2.5-Math's
+    output width) per generated token, one kvr_entropy_step launch.  Rows
+    have spreads in [3.6, 5.0] (entropy about 2.5-6.5 nats, below tau), so
+    no row stops and every launch reads every row.  Three logit buffers
+    rotate (each larger than L2)."""
+    import torch
+    from paper_2608_15797_gb300 import kvr
+    rows, V = 512, inputs.VOCAB
+    dt = args.entropy_dtype
+    tdt = torch.bfloat16 if dt == "bf16" else torch.float32
+    dev = torch.device("cuda", 0)
+    det = kvr.EntropyDetector(rows, V, logits_dtype=dt, device=dev)
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(args.seed + 41)
+    sig = torch.linspace(3.6, 5.0, rows, device=dev).unsqueeze(1)
+    bufs = [(torch.randn(rows, V, generator=gen, device=dev) * sig).to(tdt)
+            for _ in range(3)]
+    H = torch.empty(rows, dtype=torch.float32, device=dev)
+    M = torch.empty_like(H)
+    St = torch.empty(rows, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step(i, x=None):
+        det.step(bufs[i % 3] if x is None else x, H, M, St, stream)
+
+    K, Wm = args.steps, max(3, args.warmup)
+    for i in range(Wm):
+        step(i)
+    torch.cuda.synchronize()
+    n0 = det.launch_count()
+    clocks = ClockSampler(0)
+    clocks.start()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    tb = clocks.mark()
+    t0.record(stream)
+    for i in range(K):
+        step(i)
+    t1.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop(tb, clocks.mark())
+    total = t0.elapsed_time(t1)
+    launches = det.launch_count() - n0
+    det.sync_status()
+    stopped = int((St != 0).sum().item())
+    # end to end: logits from pinned host memory, stop flags back, per token
+    host = [b.cpu().pin_memory() for b in bufs[:2]]
+    flags = torch.empty(rows, dtype=torch.int32).pin_memory()
+    xd = torch.empty_like(bufs[0])
+    Ke = max(3, args.e2e_steps // 50)
+    step(0, bufs[0])
+    torch.cuda.synchronize()
+    t0.record(stream)
+    for i in range(Ke):
+        xd.copy_(host[i % 2], non_blocking=True)
+        step(i, xd)
+        flags.copy_(St, non_blocking=True)
+    t1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = t0.elapsed_time(t1)
+    esz = 2 if dt == "bf16" else 4
+    per_launch = rows * V * esz + rows * (4 * 12 + 16)
+    return dict(total_ms=total, per_ms=total / max(1, launches), K=K,
+                launches=launches, launch_bytes=per_launch, rows=rows, V=V,
+                dtype=dt, stopped=stopped, clocks=clk, Ke=Ke, e2e_ms=e2e_ms,
+                bi=rows * V * esz, bo=rows * 4)
+
+
+def entropy_cpu_baseline(seconds):
+    """The fp64 oracle's token_entropy on bounded samples of the same rows
+    (8 rows of 152,064 logits per call), scaled to tokens/s."""
+    import time
+    from oracle import entropy as ent
+    x = inputs.candidate_logits(0, 0, 8, inputs.VOCAB, 4.0)
+    n, t0 = 0, time.perf_counter()
+    while time.perf_counter() - t0 < seconds:
+        ent.token_entropy(x)
+        n += 8
+    spent = time.perf_counter() - t0
+    return n / spent, n, spent
+
+
 def run_fork(args):
     """72B geometry (80 layers, 64 q / 8 kv heads, d 128), B=64, W=8: an
     evicted parent (B+W rows) forked to 8 candidates; one timed step is one
@@ -823,6 +910,51 @@ def main():
                            "note": "mma.sync flops incl. the second QK pass "
                                    "and the lo term of P"},
                 "gpu_launches": r["launches"]}))
+        return 0
+    if args.mode == "entropy":
+        if rank == 0:
+            r = run_entropy(args)
+            peaks, peak_kind = measured_peaks()
+            sec = r["per_ms"] / 1e3
+            gbs = r["launch_bytes"] / sec / 1e9
+            line = {
+                "metric": "candidate tokens screened/s by the entropy test "
+                          f"({r['rows']} candidate rows x {r['V']} "
+                          f"{r['dtype']} logits per launch)",
+                "value": r["K"] * r["rows"] / (r["total_ms"] / 1e3),
+                "unit": "tokens/s", "n_gpus": 1, "steps": r["K"],
+                "warmup": args.warmup, "ms_per_step": r["total_ms"] / r["K"],
+                "higher_is_better": True, "scaling": "weak",
+                "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+                "config": {"workload": "entropy detector, 64 problems x 8 "
+                                       "candidates", "rows": r["rows"],
+                           "vocab": r["V"], "logits": r["dtype"],
+                           "window": 12, "guard": 24, "tau": 7.0,
+                           "l2": "3 rotating logit buffers, each larger "
+                                 "than L2"},
+                "rows_stopped": r["stopped"],
+                "roofline": {"bound": "hbm", "achieved": gbs,
+                             "peak": float(peaks["hbm_gbs"]), "unit": "GB/s",
+                             "frac": gbs / float(peaks["hbm_gbs"]),
+                             "peak_kind": peak_kind, "traffic": None,
+                             "algorithmic_bytes_per_launch": r["launch_bytes"],
+                             "launch_ms": r["per_ms"],
+                             "kernel": "entropy_kernel"},
+                "e2e": {"value": r["Ke"] * r["rows"] / (r["e2e_ms"] / 1e3),
+                        "unit": "tokens/s", "h2d_bytes_per_step": r["bi"],
+                        "d2h_bytes_per_step": r["bo"]},
+                "gpu_launches": r["launches"],
+                "clocks": r["clocks"],
+            }
+            if not args.no_cpu_baseline:
+                rate, n, spent = entropy_cpu_baseline(min(args.cpu_seconds,
+                                                          10.0))
+                line["cpu_baseline"] = {
+                    "value": rate, "unit": "tokens/s", "cores": 1,
+                    "kind": "oracle",
+                    "sample": f"{n} rows of {inputs.VOCAB} logits through the "
+                              f"fp64 oracle in {spent:.1f} s"}
+            print(json.dumps(line))
         return 0
     if args.mode != "step":
         if rank == 0:

@@ -271,6 +271,82 @@ kvr_status kvr_absorb_chunk(kvr_cache *cache, int layer_begin, int layer_end,
                             const void *v_new, void *out, int budget,
                             int window, int evict, void *stream);
 
+/* ---- degeneration detector: the entropy test ---------------------------- */
+
+/* Sec. 3.3 ("Incoherent generation") and App. Impl. ("Online degeneration
+ * detection"): each base candidate is screened while it decodes.  At its e-th
+ * generated token (e = 1, 2, ... since the row's last reset) the detector
+ * takes the predictive entropy
+ *   H_e = -sum_v p_e(v) ln p_e(v),  p_e = softmax(logits / temperature)
+ * over the whole vocabulary (natural log; nats), and its moving mean H-bar_e
+ * over the last min(e, window) tokens.  The row stops at the first e > guard
+ * with H-bar_e > tau; a stopped row stays stopped and its later logits are
+ * not read.  App. Impl. uses tau = 7.0, window 12, guard 24.  (The paper's
+ * second test, the gzip ratio of the candidate's text, is host text work and
+ * not part of this library.)
+ *
+ * The decision is taken in fp32: the window's entropies are summed oldest
+ * first and the row stops when e > guard and sum > tau * min(e, window). */
+typedef struct {
+  int rows;        /* candidate rows tracked, 1..65535 */
+  int vocab;       /* logits per row, >= 1 */
+  int window;      /* |W_e|, 1..64 */
+  int guard;       /* positions never tested (e <= guard), >= 0 */
+  float tau;       /* threshold on the moving mean, nats */
+  float temperature; /* softmax temperature, > 0; 0 means 1 */
+  kvr_dtype logits_dtype;
+} kvr_entropy_desc;
+
+typedef struct kvr_entropy kvr_entropy; /* opaque host handle */
+
+/* Device bytes the detector's state needs (0 for an invalid descriptor). */
+size_t kvr_entropy_required_bytes(const kvr_entropy_desc *desc);
+
+/* Lay the state out in the caller's device buffer dev_buf (256-byte aligned,
+ * >= required bytes; the caller keeps ownership) and clear it on stream:
+ * every row starts live with no tokens seen.  The handle owns host
+ * metadata only. */
+kvr_status kvr_entropy_create(const kvr_entropy_desc *desc, void *dev_buf,
+                              size_t bytes, void *stream, kvr_entropy **out);
+
+/* Rows [row_begin, row_end) take new candidates: no tokens seen, live.
+ * Stream-ordered. */
+kvr_status kvr_entropy_reset(kvr_entropy *det, int row_begin, int row_end,
+                             void *stream);
+
+/* One generated token for every row, in one launch.
+ *   logits     dev [rows][row_stride] of logits_dtype; the first vocab of
+ *              each row are read.  row_stride >= vocab (elements).
+ *   entropy    dev [rows] fp32 or NULL: H_e (NaN for a row already stopped
+ *              before this call, whose logits are not read).
+ *   mean       dev [rows] fp32 or NULL: H-bar_e (NaN for such a row).
+ *   stopped    dev [rows] int32 or NULL: after this token, the position e
+ *              at which the row stopped, or 0 while it is live.
+ * Rows whose logits hold a NaN or +inf, or only -inf, get H_e = NaN, never
+ * stop on it, and set the device error word (kvr_entropy_sync_status).
+ * Stream-ordered; calls on one handle must be ordered on one stream. */
+kvr_status kvr_entropy_step(kvr_entropy *det, const void *logits,
+                            int64_t row_stride, float *entropy, float *mean,
+                            int32_t *stopped, void *stream);
+
+/* Synchronising: wait for stream, then copy the state to host.
+ * host_hist [rows][window] fp32: each row's last min(count, window)
+ * entropies, oldest first, then zeros; host_count [rows] int32: tokens seen
+ * since the row's reset; host_stopped [rows] int32 as in kvr_entropy_step.
+ * Any pointer may be NULL. */
+kvr_status kvr_entropy_export(kvr_entropy *det, float *host_hist,
+                              int32_t *host_count, int32_t *host_stopped,
+                              void *stream);
+
+/* Synchronising: wait for stream, read and clear the detector's device
+ * error word (KVR_EDEVICE if a row's logits were not finite). */
+kvr_status kvr_entropy_sync_status(kvr_entropy *det, void *stream);
+
+/* Number of kernels this handle has launched since it was created. */
+kvr_status kvr_entropy_launch_count(const kvr_entropy *det, uint64_t *count);
+
+void kvr_entropy_destroy(kvr_entropy *det);
+
 /* ---- the same step for callers that cannot allocate -------------------- */
 
 /* The paper has no counterpart to this call: it is a deployment variant.

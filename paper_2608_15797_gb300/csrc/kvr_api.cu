@@ -642,6 +642,10 @@ int kvr::report_cuda_error(const char *where, cudaError_t e) {
   return cuda_fail(where, e);
 }
 
+int kvr::report_error(int st, const char *msg) {
+  return fail(static_cast<kvr_status>(st), "%s", msg);
+}
+
 int kvr::decode_attend_score_ext(kvr_cache *c, int lb, int le, const void *q,
                                  const void *k_new, const void *v_new,
                                  void *out, float *ext, size_t ext_floats,

@@ -268,4 +268,6 @@ int decode_attend_score_ext(kvr_cache *c, int lb, int le, const void *q,
                             float *ext, size_t ext_floats, void *stream);
 // Record a CUDA failure as the thread's last error; returns KVR_ECUDA.
 int report_cuda_error(const char *where, cudaError_t e);
+// Record msg as the thread's last error; returns st.
+int report_error(int st, const char *msg);
 }  // namespace kvr

@@ -165,3 +165,32 @@ def prior_lengths(seed: int, n_seq: int, lo: int = PRIOR_LEN_RANGE[0],
 def candidate_pick(seed: int, step: int, n_seq: int, n_cand: int) -> np.ndarray:
     """Seeded stand-in for the PRM argmax of Eq. 2: the committed candidate."""
     return _rng(seed, _TAG_PICK, step).integers(0, n_cand, size=n_seq).astype(np.int32)
+
+
+# Next-token logits of candidate rows (the degeneration detector's input).
+# The paper's models are Qwen2.5-Math; their output layer has 152,064 logits
+# (the tokenizer's vocabulary padded), which fixes the row length.
+VOCAB = 152064
+_TAG_LOGITS = 6
+
+
+def candidate_logits(seed: int, step: int, rows: int, vocab: int = VOCAB,
+                     sigma=3.0, boost=0.0, dtype: str = "bf16") -> np.ndarray:
+    """Synthetic logits [rows][vocab] for one generated position (float32,
+    element-type exact): N(0,1) * sigma[row], plus boost[row] on one token
+    per row drawn uniformly.  sigma and boost are scalars or per-row arrays.
+
+    The spread sets where a row sits against the detector's threshold: a
+    wide spread concentrates the distribution on few tokens (a coherent,
+    confident candidate), a narrow one spreads it over many (an incoherent
+    one).  These Gaussian rows stand in for the Qwen2.5-Math logits of the
+    paper's candidates."""
+    rng = _rng(seed, _TAG_LOGITS, step)
+    x = rng.standard_normal((rows, vocab), dtype=np.float32)
+    x *= np.asarray(sigma, np.float32).reshape(-1, 1) if np.ndim(sigma) else \
+        np.float32(sigma)
+    b = np.broadcast_to(np.asarray(boost, np.float32), (rows,))
+    if np.any(b != 0):
+        hot = rng.integers(0, vocab, size=rows)
+        x[np.arange(rows), hot] += b
+    return round_to(x, dtype)

@@ -476,3 +476,140 @@ def attend_full(cache: Cache, q, k_new, v_new, out=None, layers=None,
     kvr_decode_attend(cache.handle, lb, le, q, k_new, v_new, out, n_splits,
                       workspace, workspace.numel(), stream)
     return out
+
+
+# ---- degeneration detector: the entropy test --------------------------------
+
+class kvr_entropy_desc(ctypes.Structure):
+    _fields_ = [("rows", ctypes.c_int), ("vocab", ctypes.c_int),
+                ("window", ctypes.c_int), ("guard", ctypes.c_int),
+                ("tau", ctypes.c_float), ("temperature", ctypes.c_float),
+                ("logits_dtype", ctypes.c_int)]
+
+
+for _name, (_res, _args) in {
+    "kvr_entropy_required_bytes": (ctypes.c_size_t,
+                                   [ctypes.POINTER(kvr_entropy_desc)]),
+    "kvr_entropy_create": (_S, [ctypes.POINTER(kvr_entropy_desc), _P,
+                                ctypes.c_size_t, _P, ctypes.POINTER(_P)]),
+    "kvr_entropy_reset": (_S, [_P, _I, _I, _P]),
+    "kvr_entropy_step": (_S, [_P, _P, ctypes.c_int64, _P, _P, _P, _P]),
+    "kvr_entropy_export": (_S, [_P, _P, _P, _P, _P]),
+    "kvr_entropy_sync_status": (_S, [_P, _P]),
+    "kvr_entropy_launch_count": (_S, [_P, _P]),
+    "kvr_entropy_destroy": (None, [_P]),
+}.items():
+    _f = getattr(lib, _name)
+    _f.restype = _res
+    _f.argtypes = _args
+
+
+def kvr_entropy_required_bytes(desc: kvr_entropy_desc) -> int:
+    return int(lib.kvr_entropy_required_bytes(ctypes.byref(desc)))
+
+
+def kvr_entropy_create(desc, dev_buf, nbytes, stream=None):
+    h = _P()
+    _check(lib.kvr_entropy_create(ctypes.byref(desc), _ptr(dev_buf), nbytes,
+                                  _stream(stream), ctypes.byref(h)),
+           "kvr_entropy_create")
+    return h
+
+
+def kvr_entropy_reset(h, row_begin, row_end, stream=None):
+    _check(lib.kvr_entropy_reset(h, row_begin, row_end, _stream(stream)),
+           "kvr_entropy_reset")
+
+
+def kvr_entropy_step(h, logits, row_stride, entropy=None, mean=None,
+                     stopped=None, stream=None):
+    _check(lib.kvr_entropy_step(h, _ptr(logits), int(row_stride),
+                                _ptr(entropy), _ptr(mean), _ptr(stopped),
+                                _stream(stream)), "kvr_entropy_step")
+
+
+def kvr_entropy_export(h, host_hist, host_count, host_stopped, stream=None):
+    _check(lib.kvr_entropy_export(h, _ptr(host_hist), _ptr(host_count),
+                                  _ptr(host_stopped), _stream(stream)),
+           "kvr_entropy_export")
+
+
+def kvr_entropy_sync_status(h, stream=None):
+    _check(lib.kvr_entropy_sync_status(h, _stream(stream)),
+           "kvr_entropy_sync_status")
+
+
+def kvr_entropy_launch_count(h) -> int:
+    n = ctypes.c_uint64()
+    _check(lib.kvr_entropy_launch_count(h, ctypes.byref(n)),
+           "kvr_entropy_launch_count")
+    return n.value
+
+
+def kvr_entropy_destroy(h):
+    lib.kvr_entropy_destroy(h)
+
+
+class EntropyDetector:
+    """Owner of one kvr_entropy handle and the torch buffer it lives in
+    (Sec. 3.3 entropy test; App. Impl. tau 7.0, window 12, guard 24)."""
+
+    def __init__(self, rows, vocab, window=12, guard=24, tau=7.0,
+                 temperature=1.0, logits_dtype="bf16", device="cuda",
+                 stream=None):
+        self.desc = kvr_entropy_desc(rows, vocab, window, guard, float(tau),
+                                     float(temperature), DTYPES[logits_dtype])
+        self.rows, self.vocab, self.window = rows, vocab, window
+        self.logits_dtype = logits_dtype
+        self.nbytes = kvr_entropy_required_bytes(self.desc)
+        if self.nbytes == 0:
+            raise KvrError(KVR_EINVAL, "EntropyDetector", "invalid descriptor")
+        self.buf = torch.empty(self.nbytes, dtype=torch.uint8, device=device)
+        self.handle = kvr_entropy_create(self.desc, self.buf, self.nbytes,
+                                         stream)
+
+    def __del__(self):
+        h = getattr(self, "handle", None)
+        if h:
+            kvr_entropy_destroy(h)
+            self.handle = None
+
+    def reset(self, begin=0, end=None, stream=None):
+        kvr_entropy_reset(self.handle, begin, self.rows if end is None else end,
+                          stream)
+
+    def step(self, logits, entropy=None, mean=None, stopped=None, stream=None):
+        """One generated token: logits [rows][>= vocab] (row stride taken
+        from the tensor).  Returns (entropy, mean, stopped) device tensors."""
+        if logits.dim() != 2 or logits.shape[0] != self.rows or \
+                logits.shape[1] < self.vocab or logits.stride(1) != 1:
+            raise ValueError("logits must be [rows][>= vocab] with unit "
+                             "column stride")
+        if logits.dtype != TORCH_DTYPES[self.logits_dtype]:
+            raise ValueError("logits dtype does not match the descriptor")
+        dev = logits.device
+        entropy = torch.empty(self.rows, dtype=torch.float32, device=dev) \
+            if entropy is None else entropy
+        mean = torch.empty(self.rows, dtype=torch.float32, device=dev) \
+            if mean is None else mean
+        stopped = torch.empty(self.rows, dtype=torch.int32, device=dev) \
+            if stopped is None else stopped
+        _check(lib.kvr_entropy_step(self.handle,
+                                    ctypes.c_void_p(logits.data_ptr()),
+                                    int(logits.stride(0)), _ptr(entropy),
+                                    _ptr(mean), _ptr(stopped),
+                                    _stream(stream)), "kvr_entropy_step")
+        return entropy, mean, stopped
+
+    def export(self, stream=None):
+        hist = np.zeros((self.rows, self.window), np.float32)
+        count = np.zeros(self.rows, np.int32)
+        stopped = np.zeros(self.rows, np.int32)
+        kvr_entropy_export(self.handle, hist, count, stopped, stream)
+        return hist, count, stopped
+
+    def launch_count(self):
+        return kvr_entropy_launch_count(self.handle)
+
+    def sync_status(self, stream=None):
+        kvr_entropy_sync_status(self.handle, stream)
