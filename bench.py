@@ -72,6 +72,9 @@ def parse():
                         "16k context; fork: 72B best-of-8 candidate step")
     p.add_argument("--entropy-dtype", default="bf16", choices=["bf16", "f32"],
                    help="logit element type for --mode entropy")
+    p.add_argument("--entropy-kernel", type=int, default=0, choices=[0, 1, 2],
+                   help="--mode entropy kernel: 0 library's choice, "
+                        "1 persistent streaming, 2 one CTA per piece")
     p.add_argument("--seqs", type=int, default=0,
                    help="sequences for --mode helper/fork (0: 16 / 4)")
     p.add_argument("--chunk-groups", type=int, default=0,
@@ -663,6 +666,7 @@ def run_entropy(args):
     tdt = torch.bfloat16 if dt == "bf16" else torch.float32
     dev = torch.device("cuda", 0)
     det = kvr.EntropyDetector(rows, V, logits_dtype=dt, device=dev)
+    det.set_kernel(args.entropy_kernel)
     gen = torch.Generator(device=dev)
     gen.manual_seed(args.seed + 41)
     sig = torch.linspace(3.6, 5.0, rows, device=dev).unsqueeze(1)

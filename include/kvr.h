@@ -342,6 +342,13 @@ kvr_status kvr_entropy_export(kvr_entropy *det, float *host_hist,
  * error word (KVR_EDEVICE if a row's logits were not finite). */
 kvr_status kvr_entropy_sync_status(kvr_entropy *det, void *stream);
 
+/* Kernel choice (results agree within rounding): 0 = the library's choice
+ * (the piece kernel for bf16 logits, the streaming kernel for fp32),
+ * 1 = the persistent streaming kernel wherever the rows are 16-byte aligned
+ * and hold at least one 16-byte vector (the piece kernel otherwise),
+ * 2 = the piece kernel (one CTA per 16,384 bf16 / 8,192 fp32 logits). */
+kvr_status kvr_entropy_set_kernel(kvr_entropy *det, int kernel);
+
 /* Number of kernels this handle has launched since it was created. */
 kvr_status kvr_entropy_launch_count(const kvr_entropy *det, uint64_t *count);
 

@@ -497,6 +497,7 @@ for _name, (_res, _args) in {
     "kvr_entropy_export": (_S, [_P, _P, _P, _P, _P]),
     "kvr_entropy_sync_status": (_S, [_P, _P]),
     "kvr_entropy_launch_count": (_S, [_P, _P]),
+    "kvr_entropy_set_kernel": (_S, [_P, _I]),
     "kvr_entropy_destroy": (None, [_P]),
 }.items():
     _f = getattr(lib, _name)
@@ -607,6 +608,12 @@ class EntropyDetector:
         stopped = np.zeros(self.rows, np.int32)
         kvr_entropy_export(self.handle, hist, count, stopped, stream)
         return hist, count, stopped
+
+    def set_kernel(self, kernel: int):
+        """0: the library's choice, 1: persistent streaming kernel, 2: one CTA
+        per piece of a row."""
+        _check(lib.kvr_entropy_set_kernel(self.handle, kernel),
+               "kvr_entropy_set_kernel")
 
     def launch_count(self):
         return kvr_entropy_launch_count(self.handle)

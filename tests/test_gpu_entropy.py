@@ -60,11 +60,12 @@ def _sigma_schedule(rows, e):
 
 def run_lockstep(rows, vocab, steps, dtype="bf16", stride=None, window=12,
                  guard=24, tau=7.0, temperature=1.0, seed=0, offset=None,
-                 resets=()):
+                 resets=(), kernel=0):
     """Drive the kernel and the oracle through `steps` tokens; check every
     output.  Returns (near_ties, stops)."""
     det = kvr.EntropyDetector(rows, vocab, window, guard, tau, temperature,
                               dtype)
+    det.set_kernel(kernel)
     ref = ent.EntropyDetector(rows, window, guard, tau)
     hist32 = [[] for _ in range(rows)]  # the kernel's entropies, per row
     stop32 = np.zeros(rows, np.int64)
@@ -123,16 +124,29 @@ def run_lockstep(rows, vocab, steps, dtype="bf16", stride=None, window=12,
     return near, stop32
 
 
+KERNELS = {"stream": 1, "pieces": 2}
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])
 @pytest.mark.parametrize("vocab", [7, 1000, 16385, 40000])
-def test_entropy_lockstep_shapes(dtype, vocab):
-    near, stops = run_lockstep(12, vocab, 40, dtype)
+def test_entropy_lockstep_shapes(dtype, vocab, kernel):
+    near, stops = run_lockstep(12, vocab, 40, dtype, kernel=KERNELS[kernel])
     assert near <= 6
 
 
+@pytest.mark.parametrize("kernel", KERNELS)
+@pytest.mark.parametrize("rows", [1, 3, 200])
+def test_entropy_row_counts(rows, kernel):
+    """One row spread over many CTAs' segments, and many rows."""
+    run_lockstep(rows, 33333, 27, "bf16", kernel=KERNELS[kernel])
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])
-def test_entropy_qwen_vocab(dtype):
-    near, stops = run_lockstep(16, inputs.VOCAB, 40, dtype)
+def test_entropy_qwen_vocab(dtype, kernel):
+    near, stops = run_lockstep(16, inputs.VOCAB, 40, dtype,
+                               kernel=KERNELS[kernel])
     assert near <= 8
     # the schedule's incoherent rows stop at the first tested position
     assert all(stops[r] == 25 for r in range(1, 16, 4))
@@ -140,7 +154,8 @@ def test_entropy_qwen_vocab(dtype):
 
 
 @pytest.mark.parametrize("dtype,stride", [("bf16", 1001), ("bf16", 1003),
-                                          ("f32", 1001), ("f32", 1008)])
+                                          ("bf16", 1016), ("f32", 1001),
+                                          ("f32", 1008)])
 def test_entropy_padded_and_unaligned_rows(dtype, stride):
     run_lockstep(8, 1000, 30, dtype, stride=stride)
 
@@ -158,15 +173,19 @@ def test_entropy_large_logit_offset():
     run_lockstep(8, 3000, 26, "f32", offset=-900.0)
 
 
-def test_entropy_reset_rows():
-    run_lockstep(8, 2000, 60, "bf16", resets=((30, 1, 3), (45, 0, 8)))
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_entropy_reset_rows(kernel):
+    run_lockstep(8, 2000, 60, "bf16", resets=((30, 1, 3), (45, 0, 8)),
+                 kernel=KERNELS[kernel])
 
 
-def test_entropy_full_size_sampled():
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_entropy_full_size_sampled(kernel):
     """The bench's launch: 512 rows of 152,064 bf16 logits (64 problems x 8
     candidates), every row checked against the oracle for 3 tokens."""
     rows, V = 512, inputs.VOCAB
     det = kvr.EntropyDetector(rows, V)
+    det.set_kernel(KERNELS[kernel])
     gen = torch.Generator(device="cuda")
     gen.manual_seed(5)
     sig = torch.linspace(1.5, 5.0, rows, device="cuda").unsqueeze(1)
