@@ -215,25 +215,27 @@ class ClockSampler:
 # the CUDA arm
 # --------------------------------------------------------------------------
 
-def kernel_source_hash():
+def kernel_source_hash(files):
+    """sha256 (16 hex digits) of the named files under csrc/, in order."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2608_15797_gb300", "csrc")
-    for fn in sorted(os.listdir(csrc)):
-        if fn.endswith((".cu", ".cuh", ".h")):
-            with open(os.path.join(csrc, fn), "rb") as f:
-                h.update(f.read())
+    for fn in files:
+        with open(os.path.join(csrc, fn), "rb") as f:
+            h.update(f.read())
     return h.hexdigest()[:16]
 
 
-def committed_traffic(workload):
-    """DRAM bytes per launch from the committed ncu summary, if it was taken
-    on the current kernel sources."""
-    path = os.path.join(ROOT, "profiles", f"decode_step_{workload}.json")
+def committed_traffic(name):
+    """DRAM bytes per launch from the committed ncu summary profiles/<name>
+    .json, if it was taken on the current sources of that kernel (the files
+    it lists)."""
+    path = os.path.join(ROOT, "profiles", f"{name}.json")
     if not os.path.exists(path):
         return None
     with open(path) as f:
         d = json.load(f)
-    if d.get("kernel_sources_sha") != kernel_source_hash():
+    files = d.get("kernel_sources")
+    if not files or d.get("kernel_sources_sha") != kernel_source_hash(files):
         return None
     return d.get("dram_bytes_per_launch")
 
@@ -940,10 +942,16 @@ def main():
                 "roofline": {"bound": "hbm", "achieved": gbs,
                              "peak": float(peaks["hbm_gbs"]), "unit": "GB/s",
                              "frac": gbs / float(peaks["hbm_gbs"]),
-                             "peak_kind": peak_kind, "traffic": None,
+                             "peak_kind": peak_kind,
+                             "traffic": committed_traffic(
+                                 f"entropy_stream_{r['rows']}x{r['V']}_"
+                                 f"{r['dtype']}")
+                             if args.entropy_kernel in (0, 1) else None,
                              "algorithmic_bytes_per_launch": r["launch_bytes"],
                              "launch_ms": r["per_ms"],
-                             "kernel": "entropy_kernel"},
+                             "kernel": "entropy_stream_kernel"
+                             if args.entropy_kernel in (0, 1)
+                             else "entropy_kernel"},
                 "e2e": {"value": r["Ke"] * r["rows"] / (r["e2e_ms"] / 1e3),
                         "unit": "tokens/s", "h2d_bytes_per_step": r["bi"],
                         "d2h_bytes_per_step": r["bo"]},
@@ -1016,7 +1024,8 @@ def main():
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak,
                      "unit": "GB/s", "frac": achieved / peak,
                      "peak_kind": peak_kind,
-                     "traffic": committed_traffic(args.workload),
+                     "traffic": committed_traffic(
+                         f"decode_step_{args.workload}"),
                      "algorithmic_bytes_per_launch": r["launch_bytes"],
                      "launch_ms": r["per_launch_ms"],
                      "launch_timing": "timed region / launches in it",

@@ -343,7 +343,7 @@ kvr_status kvr_entropy_export(kvr_entropy *det, float *host_hist,
 kvr_status kvr_entropy_sync_status(kvr_entropy *det, void *stream);
 
 /* Kernel choice (results agree within rounding): 0 = the library's choice
- * (the piece kernel for bf16 logits, the streaming kernel for fp32),
+ * (the streaming kernel where the rows allow it),
  * 1 = the persistent streaming kernel wherever the rows are 16-byte aligned
  * and hold at least one 16-byte vector (the piece kernel otherwise),
  * 2 = the piece kernel (one CTA per 16,384 bf16 / 8,192 fp32 logits). */

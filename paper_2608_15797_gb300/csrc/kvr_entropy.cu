@@ -67,6 +67,27 @@ struct StepIO {
   int32_t *stopped;
 };
 
+// Packed fp32 pairs (sm_100 and later): one instruction adds or fuses two
+// lanes' worth of arithmetic.
+__device__ __forceinline__ uint64_t pk(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void upk(uint64_t v, float &lo, float &hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.ftz.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t add2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.ftz.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
 __device__ __forceinline__ float max_nan(float a, float b) {
   float r;
   asm("max.NaN.f32 %0, %1, %2;" : "=f"(r) : "f"(a), "f"(b));
@@ -115,27 +136,28 @@ struct Online {
     }
   }
 
-  // Two partial sums each (even and odd terms) shorten the dependency
-  // chains.
+  // Terms in pairs with packed fp32 arithmetic: the pair sums (even and
+  // odd terms) are added into s and t at the end.
   template <int N>
   __device__ __forceinline__ void add_fast(const float (&x)[N], float c,
                                            float nm) {
-    float sa = 0.f, ta = 0.f, sb = 0.f, tb = 0.f;
+    static_assert(N % 2 == 0, "pairs");
+    const uint64_t cc = pk(c, c), mm = pk(nm, nm);
+    uint64_t s2 = pk(0.f, 0.f), t2 = pk(0.f, 0.f);
 #pragma unroll
     for (int j = 0; j < N; j += 2) {
-      const float d = fmaf(x[j], c, nm);
-      const float e = kvr::ptx::ex2(d);
-      sa += e;
-      ta = fmaf(e, d, ta);
-      if (j + 1 < N) {
-        const float d2 = fmaf(x[j + 1], c, nm);
-        const float e2 = kvr::ptx::ex2(d2);
-        sb += e2;
-        tb = fmaf(e2, d2, tb);
-      }
+      const uint64_t d = fma2(pk(x[j], x[j + 1]), cc, mm);
+      float d0, d1;
+      upk(d, d0, d1);
+      const uint64_t e = pk(kvr::ptx::ex2(d0), kvr::ptx::ex2(d1));
+      s2 = add2(s2, e);
+      t2 = fma2(e, d, t2);
     }
-    s += sa + sb;
-    t += ta + tb;
+    float s0, s1, t0, t1;
+    upk(s2, s0, s1);
+    upk(t2, t0, t1);
+    s += s0 + s1;
+    t += t0 + t1;
   }
 
   __device__ __forceinline__ bool finite() const {
@@ -755,9 +777,9 @@ kvr_status kvr_entropy_step(kvr_entropy *det, const void *logits,
   cudaStream_t st = as_stream(stream);
   cudaError_t e;
   const int nvf = det->d.vocab / (bf16 ? 8 : 4);
-  // Measured at 512 rows x 152,064 logits: the piece kernel is faster for
-  // bf16 logits, the streaming kernel for fp32.
-  const bool stream_k = det->kernel == 1 || (det->kernel == 0 && !bf16);
+  // Measured at 512 rows x 152,064 logits, the streaming kernel is the
+  // faster one for both element types.
+  const bool stream_k = det->kernel != 2;
   if (vec && nvf >= 1 && stream_k) {
     if (!det->stream_grid) {
       e = stream_setup(&det->stream_grid);
