@@ -497,7 +497,7 @@ def run_helper(args):
 
 
 def run_crossover(args):
-    """The attention-side crossover of App. C (Eq. 14) measured on this GPU
+    """The attention-side crossover of App. D (Eq. 14) measured on this GPU
     at 7B geometry: full-context decode attention (append + attention over
     every row, no scores; kvr_decode_attend) against the evicted step
     (append + attention + scores + selection + compaction over B' = B + W

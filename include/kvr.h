@@ -9,11 +9,11 @@
  *      (grouped-query attention; softmax scale 1/sqrt(d) by default),
  *   3. adds to every live row's importance score s_i ("accumulated attention",
  *      Sec. 2.1) the mean over the G query heads of that row's probability,
- *   4. once the live length exceeds B' = B + W (App. C: eviction then runs on
+ *   4. once the live length exceeds B' = B + W (App. D: eviction then runs on
  *      every step), keeps the W most recent rows (the protected window of
- *      Sec. 4.1 / App. Impl.) plus the B best-scored others (TopB of Eq. 1;
+ *      Sec. 4.1 / App. C) plus the B best-scored others (TopB of Eq. 1;
  *      equal scores keep the lower position) and compacts K/V in place.
- * Candidates (Sec. 2.2, Eq. 2; App. Impl., best-of-(N+N)) fork from one cache
+ * Candidates (Sec. 2.2, Eq. 2; App. C, best-of-(N+N)) fork from one cache
  * state, decode a step each, and the chosen one becomes the persistent state
  * (Algorithm 1).
  *
@@ -130,7 +130,7 @@ kvr_status kvr_decode_step(kvr_cache *cache, int layer_begin, int layer_end,
 /* ---- full-context decode (the helper's cache: no scores, no eviction) -- */
 
 /* The full-context helper of KV-Rescue keeps its whole cache (Sec. 3.1;
- * App. C, Eq. 11): its decode step is Attn(q_t, C_t) of Eq. 1 over every
+ * App. D, Eq. 11): its decode step is Attn(q_t, C_t) of Eq. 1 over every
  * cached row, with no importance scores and no eviction.  This call appends
  * the new row (position = next position, score 0) and attends over all
  * rows, splitting each unit's rows over n_splits CTAs whose partial softmax
@@ -151,7 +151,7 @@ kvr_status kvr_decode_attend(kvr_cache *cache, int layer_begin, int layer_end,
 
 /* ---- candidates: stepwise best-of-N over one shared cache state -------- */
 
-/* Sec. 2.2 (Eq. 2) and App. Impl. (best-of-(N+N)): each reasoning step draws
+/* Sec. 2.2 (Eq. 2) and App. C (best-of-(N+N)): each reasoning step draws
  * N candidates from the same committed (evicted) cache state; the selected
  * one becomes the persistent state (Algorithm 1).  The paper forks by
  * copying the live rows; here the candidates share the parent's live rows
@@ -273,7 +273,7 @@ kvr_status kvr_absorb_chunk(kvr_cache *cache, int layer_begin, int layer_end,
 
 /* ---- degeneration detector: the entropy test ---------------------------- */
 
-/* Sec. 3.3 ("Incoherent generation") and App. Impl. ("Online degeneration
+/* Sec. 3.2 ("Incoherent generation") and App. C ("Online degeneration
  * detection"): each base candidate is screened while it decodes.  At its e-th
  * generated token (e = 1, 2, ... since the row's last reset) the detector
  * takes the predictive entropy
@@ -281,7 +281,7 @@ kvr_status kvr_absorb_chunk(kvr_cache *cache, int layer_begin, int layer_end,
  * over the whole vocabulary (natural log; nats), and its moving mean H-bar_e
  * over the last min(e, window) tokens.  The row stops at the first e > guard
  * with H-bar_e > tau; a stopped row stays stopped and its later logits are
- * not read.  App. Impl. uses tau = 7.0, window 12, guard 24.  (The paper's
+ * not read.  App. C uses tau = 7.0, window 12, guard 24.  (The paper's
  * second test, the gzip ratio of the candidate's text, is host text work and
  * not part of this library.)
  *

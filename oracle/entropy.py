@@ -4,7 +4,7 @@ TEST INFRASTRUCTURE ONLY: the tests, ``__graft_entry__.smoke()`` and the
 ``cpu_baseline`` leg of ``bench.py`` may use this module; the product path
 never imports it.  It shares no code with the CUDA library.
 
-What it computes (Sec. 3.3, "Incoherent generation"; App. Impl., "Online
+What it computes (Sec. 3.2, "Incoherent generation"; App. C, "Online
 degeneration detection"):
 
 * ``token_entropy`` -- H_e = -sum_v p_e(v) log p_e(v), the predictive
@@ -13,7 +13,7 @@ degeneration detection"):
   vocabulary.
 * ``EntropyDetector`` -- the moving mean of H over a recent window of |W_e|
   positions, and termination of a candidate once that mean exceeds
-  tau_ent.  App. Impl. fixes tau_ent = 7.0, a window of 12 and a guard of 24
+  tau_ent.  App. C fixes tau_ent = 7.0, a window of 12 and a guard of 24
   tokens.
 
 Readings where the paper is silent:
@@ -31,7 +31,7 @@ Readings where the paper is silent:
 arithmetic (a sum over the window from oldest to newest, compared with
 tau * |W_e|), the precision in which the kernel decides.
 
-Pins: ``tests/test_oracle_pins.py`` (scipy's entropy of scipy's softmax,
+Pins: ``tests/test_entropy_oracle_pins.py`` (scipy's entropy of scipy's softmax,
 closed forms, invariances) and ``tests/golden/entropy_detector_worked.json``
 (hand-derived stop positions).
 """

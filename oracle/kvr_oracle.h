@@ -11,10 +11,10 @@
  *   - the accumulated-attention importance s_i named in Sec. 2.1 (the example
  *     score of Eq. 1), updated every step by the mean over the G query heads of
  *     that step's attention probability;
- *   - TopB of Eq. 1 with the protected recent window of Sec. 4.1 / App. C
+ *   - TopB of Eq. 1 with the protected recent window of Sec. 4.1 / App. D
  *     (physical bound B' = B + w): the W most recent tokens are always kept,
  *     the B best of the rest are kept, ties go to the lower position;
- *   - eviction fires every step once the live length exceeds B' (App. C,
+ *   - eviction fires every step once the live length exceeds B' (App. D,
  *     "Decode compute").
  *
  * Layout: a "unit" is one (sequence, layer, KV head).  Every array is

@@ -12,9 +12,9 @@ per-unit cache state:
 * ``OracleCache.step``   -- Eq. 1 (Sec. 2.1): append the step's key/value,
   attend over every live row, add the mean over the G query heads of the
   attention probability to each row's accumulated-attention score, and, when
-  the live length exceeds B' = B + W (App. C), keep the W most recent rows
+  the live length exceeds B' = B + W (App. D), keep the W most recent rows
   (Sec. 4.1 window) plus the B best-scored others (ties: lower position).
-* ``OracleCache.fork``   -- App. Impl., "Best-of-(N+N)": a candidate is a
+* ``OracleCache.fork``   -- App. C, "Best-of-(N+N)": a candidate is a
   physical copy of the parent's live rows.
 * ``OracleCache.evict``  -- TopB of Eq. 1 on the current state.
 
@@ -240,7 +240,7 @@ class OracleCache:
                                _p(self.len), _p(keep))
 
     def fork(self, n_cand):
-        """App. Impl. "Best-of-(N+N)": N physical copies of the live state."""
+        """App. C "Best-of-(N+N)": N physical copies of the live state."""
         return [self.copy() for _ in range(n_cand)]
 
     def unit_rows(self, s, l, h):

@@ -1,7 +1,7 @@
 """Analytic memory / compute model of evicted decoding, and the algorithmic
 byte counts of the decode-step kernels.
 
-Part 1 restates the paper's App. C ("Overhead Derivation"):
+Part 1 restates the paper's App. D ("Overhead Derivation"):
   Eq. 8   m_kv = 2 L h_kv d_h b                  (KV bytes per token)
   Eq. 9   M_full(l) = m_kv l,  M_evict = m_kv B'  (B' = B + w)
   Eq. 10  M_full / M_evict = l / B'

@@ -1,5 +1,5 @@
 // kvr_entropy.cu -- the entropy test of the online degeneration detector
-// (Sec. 3.3, "Incoherent generation"; App. Impl., "Online degeneration
+// (Sec. 3.2, "Incoherent generation"; App. C, "Online degeneration
 // detection") and its C ABI (include/kvr.h, kvr_entropy_*).
 //
 // One launch per generated token screens every candidate row:

@@ -1,5 +1,5 @@
 // kvr_fork.cu -- candidate kernels of libkvr (stepwise best-of-N, Sec. 2.2
-// Eq. 2 and App. Impl.): N candidates share the parent's live rows as a
+// Eq. 2 and App. C): N candidates share the parent's live rows as a
 // read-only prefix and keep private tails and private score copies.
 //
 // fork_attend_kernel: one CTA per (sequence, layer, KV head).  The prefix K

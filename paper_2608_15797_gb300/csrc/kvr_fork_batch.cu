@@ -1,5 +1,5 @@
 // kvr_fork_batch.cu -- the candidate-batched decode step of stepwise best-of-N
-// (Sec. 2.2 Eq. 2, App. Impl.): N candidates share the parent's live rows as
+// (Sec. 2.2 Eq. 2, App. C): N candidates share the parent's live rows as
 // a read-only prefix and each has a private tail.  Per candidate: append +
 // Attn(q_t, C) (Eq. 1) over prefix + tail + new row, the candidate's
 // accumulated attention (Sec. 2.1, mean over the G heads) of every row, and

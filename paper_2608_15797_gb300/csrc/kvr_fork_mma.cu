@@ -1,5 +1,5 @@
 // kvr_fork_mma.cu -- the candidate-batched decode step on tensor cores
-// (stepwise best-of-N, Sec. 2.2 Eq. 2 and App. Impl.): N candidates share
+// (stepwise best-of-N, Sec. 2.2 Eq. 2 and App. C): N candidates share
 // the parent's live rows as a read-only prefix; each has a private tail.
 // bf16, head_dim 128, G <= 8, N <= 8.
 //

@@ -1,5 +1,5 @@
 // kvr_split.cu -- full-context decode attention split over the rows (the
-// KV-Rescue helper keeps its full cache, Sec. 3.1 / App. C): append the new
+// KV-Rescue helper keeps its full cache, Sec. 3.1 / App. D): append the new
 // row and compute Attn(q_t, C) (Eq. 1) over every cached row, with no
 // importance scores and no eviction.  bf16, head_dim 128, G <= 8.
 //

@@ -553,7 +553,7 @@ def kvr_entropy_destroy(h):
 
 class EntropyDetector:
     """Owner of one kvr_entropy handle and the torch buffer it lives in
-    (Sec. 3.3 entropy test; App. Impl. tau 7.0, window 12, guard 24)."""
+    (Sec. 3.2 entropy test; App. C tau 7.0, window 12, guard 24)."""
 
     def __init__(self, rows, vocab, window=12, guard=24, tau=7.0,
                  temperature=1.0, logits_dtype="bf16", device="cuda",

@@ -1,6 +1,6 @@
-"""The analytic model of App. C against the constants the paper prints.
+"""The analytic model of App. D against the constants the paper prints.
 
-Every expected number below is printed in the paper (App. C and Sec. 4.3);
+Every expected number below is printed in the paper (App. D and Sec. 4.3);
 the model must reproduce them from Table 4 alone.
 """
 import pytest
@@ -11,20 +11,20 @@ M7, M72, M15 = cm.TABLE4["7b"], cm.TABLE4["72b"], cm.TABLE4["1.5b"]
 
 
 def test_kv_bytes_per_token():
-    # App. C, after Eq. 8: 56 KiB (7B), 320 KiB (72B), 28 KiB (1.5B)
+    # App. D, after Eq. 8: 56 KiB (7B), 320 KiB (72B), 28 KiB (1.5B)
     assert cm.m_kv(M7) == 56 * cm.KiB
     assert cm.m_kv(M72) == 320 * cm.KiB
     assert cm.m_kv(M15) == 28 * cm.KiB
 
 
 def test_eviction_saving_ratio():
-    # App. C, Eq. 10: 8192 / 640 = 12.8 at l = 8k, B = 512 (B' = 640)
+    # App. D, Eq. 10: 8192 / 640 = 12.8 at l = 8k, B = 512 (B' = 640)
     assert cm.mem_full(M7, 8192) / cm.mem_evict(M7, 640) == pytest.approx(12.8)
     assert cm.mem_full(M72, 8192) / cm.mem_evict(M72, 640) == pytest.approx(12.8)
 
 
 def test_problem_memory_at_4k():
-    # App. C, after Eq. 11: at l = 4k, B = 512, N = 8:
+    # App. D, after Eq. 11: at l = 4k, B = 512, N = 8:
     # 7B 1.75 / 1.15 GiB, 72B 10.0 / 2.44 GiB
     for base, full, kvr in ((M7, 1.75, 1.15), (M72, 10.0, 2.44)):
         assert cm.mem_full_bon(base, 8, 4096) / cm.GiB == pytest.approx(full, abs=0.005)
@@ -37,7 +37,7 @@ def test_problem_memory_at_4k():
 
 
 def test_decode_compute_constants():
-    # App. C, after Eq. 12: C_dense 15.2 / 145.4 GFLOP per token,
+    # App. D, after Eq. 12: C_dense 15.2 / 145.4 GFLOP per token,
     # C_attn = 0.401M * l and 2.62M * l FLOP
     assert cm.c_dense(M7) / 1e9 == pytest.approx(15.2, abs=0.05)
     assert cm.c_dense(M72) / 1e9 == pytest.approx(145.4, abs=0.05)
@@ -50,7 +50,7 @@ def test_decode_compute_constants():
 
 
 def test_crossover_and_alpha():
-    # App. C, Eq. 14: l* ~ 2500 at B' = 640 corresponds to alpha ~ 2.9
+    # App. D, Eq. 14: l* ~ 2500 at B' = 640 corresponds to alpha ~ 2.9
     alpha = 2500 / 640 - 1
     assert alpha == pytest.approx(2.9, abs=0.01)
     assert cm.crossover(640, alpha) == pytest.approx(2500)
@@ -60,7 +60,7 @@ def test_crossover_and_alpha():
 
 
 def test_helper_ratio():
-    # Sec. 4.1 and App. C, Eq. 15: about 24% (7B) and 2.5% (72B) at l = 4k,
+    # Sec. 4.1 and App. D, Eq. 15: about 24% (7B) and 2.5% (72B) at l = 4k,
     # for alpha in the stated range [1.5, 3]
     for alpha in (1.5, 2.0, 3.0):
         assert cm.helper_ratio(M7, M15, 4096, 640, alpha) == pytest.approx(0.24, abs=0.01)

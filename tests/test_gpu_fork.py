@@ -1,4 +1,4 @@
-"""Candidates (Sec. 2.2 Eq. 2, App. Impl. best-of-(N+N)) against the oracle.
+"""Candidates (Sec. 2.2 Eq. 2, App. C best-of-(N+N)) against the oracle.
 
 The oracle forks by physical copy (what the paper's engine does): each
 candidate is a full copy of the parent that decodes its tokens without
