@@ -239,6 +239,40 @@ class OracleCache:
                                _p(self.V), _p(self.score), _p(self.pos),
                                _p(self.len), _p(keep))
 
+    def copy_sequences(self, src: "OracleCache", src_seqs, dst_seqs):
+        """App. C "Best-of-(N+N)": a candidate is forked by physically copying
+        the live (post-eviction) KV slots of the accepted sequence, and the
+        chosen candidate becomes the persistent sequence.  Sequence
+        dst_seqs[i] of this cache takes the whole state (rows, scores,
+        positions, length, position counter) of sequence src_seqs[i] of
+        `src`, every layer and KV head.  Data movement only."""
+        if (src.L, src.H, src.d) != (self.L, self.H, self.d):
+            raise ValueError("geometry differs")
+        moved = [(int(a), int(b)) for a, b in zip(src_seqs, dst_seqs)]
+        for a, b in moved:
+            n = int(src.len[a].max(initial=0))
+            if n > self.cap:
+                raise ValueError("a live length exceeds the capacity")
+        snap = {a: (src.K[a, :, :, :min(src.cap, self.cap)].copy(),
+                    src.V[a, :, :, :min(src.cap, self.cap)].copy(),
+                    src.score[a, :, :, :min(src.cap, self.cap)].copy(),
+                    src.pos[a, :, :, :min(src.cap, self.cap)].copy(),
+                    src.len[a].copy(), src.next_pos[a].copy())
+                for a, _ in moved}
+        for a, b in moved:
+            K, V, sc, ps, ln, nx = snap[a]
+            k = K.shape[2]
+            self.K[b] = 0.0
+            self.V[b] = 0.0
+            self.score[b] = 0.0
+            self.pos[b] = 0
+            self.K[b, :, :, :k] = K
+            self.V[b, :, :, :k] = V
+            self.score[b, :, :, :k] = sc
+            self.pos[b, :, :, :k] = ps
+            self.len[b] = ln
+            self.next_pos[b] = nx
+
     def fork(self, n_cand):
         """App. C "Best-of-(N+N)": N physical copies of the live state."""
         return [self.copy() for _ in range(n_cand)]

@@ -485,3 +485,41 @@ def test_absorb_then_evict_keeps_the_brute_force_set():
             want = {int(ps[i]) for i in _brute_keep(list(sc), list(ps), B, W)}
             got = set(o.pos[0, 0, h, :o.len[0, 0, h]].tolist())
             assert got == want
+
+
+def test_copied_sequence_steps_like_its_source():
+    """A candidate forked by copy (App. C) and driven with the parent's own
+    inputs evolves exactly as the parent does, eviction every token
+    included; a copy into a larger capacity changes nothing either."""
+    w = inputs.WORKLOADS["tiny"]
+    seed, S = 3, 2
+    par = orc.OracleCache(S, w.n_layers, w.n_kv_heads, w.group, w.head_dim,
+                          cap=w.budget + w.window + 1)
+    for s in range(S):
+        k, v = inputs.prompt(w, seed, s, 20)
+        par.load(s, k, v)
+    for t in range(6):
+        q, kn, vn = inputs.step_inputs(w, seed, t, S)
+        par.step(q, kn, vn, B=w.budget, W=w.window)
+    kids = orc.OracleCache(2 * S, w.n_layers, w.n_kv_heads, w.group,
+                           w.head_dim, cap=w.budget + w.window + 9)
+    kids.copy_sequences(par, [0, 0, 1, 1], [0, 1, 2, 3])
+    for t in range(6, 16):
+        q, kn, vn = inputs.step_inputs(w, seed, t, S)
+        ref = par.step(q, kn, vn, B=w.budget, W=w.window)
+        rep = np.repeat(np.arange(S), 2)
+        out = kids.step(q[rep], kn[rep], vn[rep], B=w.budget, W=w.window)
+        assert np.array_equal(out, ref[rep])
+        for c in range(2 * S):
+            a = rep[c]
+            for l in range(w.n_layers):
+                for h in range(w.n_kv_heads):
+                    pp, ps, pk, pv = par.unit_rows(a, l, h)
+                    cp, cs, ck, cv = kids.unit_rows(c, l, h)
+                    assert np.array_equal(pp, cp) and np.array_equal(ps, cs)
+                    assert np.array_equal(pk, ck) and np.array_equal(pv, cv)
+    # commit: the parent takes a candidate's state back
+    par2 = par.copy()
+    par2.copy_sequences(kids, [1, 2], [0, 1])
+    assert np.array_equal(par2.len, par.len)
+    assert np.array_equal(par2.next_pos, par.next_pos)
