@@ -271,6 +271,28 @@ kvr_status kvr_absorb_chunk(kvr_cache *cache, int layer_begin, int layer_end,
                             const void *v_new, void *out, int budget,
                             int window, int evict, void *stream);
 
+/* ---- candidates by copy (the paper's own fork) -------------------------- */
+
+/* App. C ("Best-of-(N+N)"): each reasoning step forks N base candidates by
+ * physically copying the accepted sequence's live (post-eviction) KV slots,
+ * the candidates decode with eviction on every token like any sequence
+ * (kvr_decode_step on a cache that holds them), and the chosen candidate
+ * becomes the persistent sequence.  This call does both copies: sequence
+ * dst_seqs[i] of dst takes the whole state of sequence src_seqs[i] of src
+ * (every layer and KV head: live K/V rows, scores, positions, live length,
+ * position counter), i < n.  dst_seqs and src_seqs are host arrays.
+ *  - The caches must agree in layers, KV heads, head_dim and kv_dtype
+ *    (KVR_EINVAL); capacities may differ, but every copied unit's live
+ *    length must fit dst's capacity (KVR_ECAPACITY).
+ *  - A dst sequence appears at most once; when dst == src, no sequence is
+ *    both read and written (KVR_EINVAL).
+ *  - Neither cache may have a live kvr_fork (KVR_ESTATE).
+ *  - Stream-ordered; nothing is enqueued on an error. */
+kvr_status kvr_cache_copy_sequences(kvr_cache *dst, const int32_t *dst_seqs,
+                                    const kvr_cache *src,
+                                    const int32_t *src_seqs, int n,
+                                    void *stream);
+
 /* ---- degeneration detector: the entropy test ---------------------------- */
 
 /* Sec. 3.2 ("Incoherent generation") and App. C ("Online degeneration

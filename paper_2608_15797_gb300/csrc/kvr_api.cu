@@ -609,6 +609,61 @@ kvr_status kvr_decode_attend_score(kvr_cache *c, int lb, int le, const void *q,
   return KVR_OK;
 }
 
+kvr_status kvr_cache_copy_sequences(kvr_cache *dst, const int32_t *dst_seqs,
+                                    const kvr_cache *src,
+                                    const int32_t *src_seqs, int n,
+                                    void *stream) {
+  if (!dst || !src) return fail(KVR_EINVAL, "null cache");
+  if (n < 0) return fail(KVR_EINVAL, "negative count %d", n);
+  if (n == 0) return KVR_OK;
+  if (!dst_seqs || !src_seqs) return fail(KVR_EINVAL, "null sequence list");
+  if (dst->forks || src->forks) return fail(KVR_ESTATE, "a cache has a live fork");
+  const kvr_cache_desc &a = src->desc, &b = dst->desc;
+  if (a.n_layers != b.n_layers || a.n_kv_heads != b.n_kv_heads ||
+      a.head_dim != b.head_dim || a.kv_dtype != b.kv_dtype)
+    return fail(KVR_EINVAL, "the caches' layers, KV heads, head_dim or "
+                "kv_dtype differ");
+  const int L = a.n_layers;
+  std::vector<char> taken(b.n_seq, 0), read(a.n_seq, 0);
+  for (int i = 0; i < n; ++i) {
+    const int s = src_seqs[i], d = dst_seqs[i];
+    if (s < 0 || s >= a.n_seq || d < 0 || d >= b.n_seq)
+      return fail(KVR_EINVAL, "pair %d (%d -> %d) outside the caches", i, s, d);
+    if (taken[d]) return fail(KVR_EINVAL, "sequence %d is written twice", d);
+    taken[d] = 1;
+    read[s] = 1;
+    for (int l = 0; l < L; ++l)
+      if (src->len[(size_t)s * L + l] > b.capacity)
+        return fail(KVR_ECAPACITY, "sequence %d holds %d rows > capacity %d",
+                    s, src->len[(size_t)s * L + l], b.capacity);
+  }
+  if (dst == src)
+    for (int i = 0; i < n; ++i)
+      if (read[dst_seqs[i]])
+        return fail(KVR_EINVAL, "sequence %d is both read and written",
+                    dst_seqs[i]);
+  const int row_bytes = a.head_dim * esize(a.kv_dtype);
+  kvr::SeqPairs pairs;
+  for (int i0 = 0; i0 < n; i0 += kvr::kMaxSeqPairs) {
+    const int m = std::min(kvr::kMaxSeqPairs, n - i0);
+    for (int i = 0; i < m; ++i) {
+      pairs.src[i] = src_seqs[i0 + i];
+      pairs.dst[i] = dst_seqs[i0 + i];
+    }
+    cudaError_t e = kvr::launch_copy_seqs(dst->view, src->view, pairs, m,
+                                          row_bytes, as_stream(stream));
+    if (e != cudaSuccess) return cuda_fail("kvr_cache_copy_sequences", e);
+    dst->launches += 1;
+  }
+  for (int i = 0; i < n; ++i)
+    for (int l = 0; l < L; ++l) {
+      dst->len[(size_t)dst_seqs[i] * L + l] = src->len[(size_t)src_seqs[i] * L + l];
+      dst->next_pos[(size_t)dst_seqs[i] * L + l] =
+          src->next_pos[(size_t)src_seqs[i] * L + l];
+    }
+  return KVR_OK;
+}
+
 kvr_status kvr_cache_set_fused(kvr_cache *c, int enable) {
   if (!c) return fail(KVR_EINVAL, "null cache");
   c->fused = enable != 0;

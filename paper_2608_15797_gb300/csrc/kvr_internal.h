@@ -93,6 +93,18 @@ cudaError_t launch_load(const CacheView &c, int seq, const void *k,
                         cudaStream_t st);
 cudaError_t launch_init(const CacheView &c, cudaStream_t st);
 
+// Sequence pairs of one kvr_cache_copy_sequences launch (passed by value).
+constexpr int kMaxSeqPairs = 1024;
+struct SeqPairs {
+  int32_t src[kMaxSeqPairs];
+  int32_t dst[kMaxSeqPairs];
+};
+// Copy the whole state of sequence p.src[i] of `src` into sequence p.dst[i]
+// of `dst`, i < n_pairs <= kMaxSeqPairs; row_bytes = d * element size.
+cudaError_t launch_copy_seqs(const CacheView &dst, const CacheView &src,
+                             const SeqPairs &p, int n_pairs, int row_bytes,
+                             cudaStream_t st);
+
 // Fused steady-state step (kvr_fused.cu): bf16, d = 128, G <= 8, at most 128
 // live rows per unit after the append, at most one eviction per unit.
 struct FusedParams {

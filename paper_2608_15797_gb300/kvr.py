@@ -63,6 +63,7 @@ _SIGS = {
     "kvr_evict_compact": (_S, [_P, _I, _I, _I, _I, _P]),
     "kvr_decode_step": (_S, [_P, _I, _I, _P, _P, _P, _P, _I, _I, _P]),
     "kvr_absorb_chunk": (_S, [_P, _I, _I, _I, _P, _P, _P, _P, _I, _I, _I, _P]),
+    "kvr_cache_copy_sequences": (_S, [_P, _P, _P, _P, _I, _P]),
     "kvr_cache_export": (_S, [_P, _I, _P, _P, _P, _P, _P, _P, _P]),
     "kvr_cache_lengths": (_S, [_P, _P]),
     "kvr_cache_launch_count": (_S, [_P, _P]),
@@ -173,6 +174,16 @@ def kvr_absorb_chunk(h, layer_begin, layer_end, chunk, q, k_new, v_new, out,
                                 _ptr(k_new), _ptr(v_new), _ptr(out), budget,
                                 window, 1 if evict else 0, _stream(stream)),
            "kvr_absorb_chunk")
+
+
+def kvr_cache_copy_sequences(dst, dst_seqs, src, src_seqs, stream=None):
+    d = np.ascontiguousarray(dst_seqs, dtype=np.int32)
+    s = np.ascontiguousarray(src_seqs, dtype=np.int32)
+    if d.shape != s.shape or d.ndim != 1:
+        raise ValueError("dst_seqs and src_seqs must be 1-D of one length")
+    _check(lib.kvr_cache_copy_sequences(dst, _ptr(d), src, _ptr(s), len(d),
+                                        _stream(stream)),
+           "kvr_cache_copy_sequences")
 
 
 def kvr_cache_export(h, seq, host_k, host_v, host_score, host_pos, host_len,
@@ -291,6 +302,13 @@ class Cache:
         kvr_absorb_chunk(self.handle, lb, le, c, q, k_new, v_new, out, budget,
                          window, evict, stream)
         return out
+
+    def copy_from(self, src: "Cache", src_seqs, dst_seqs, stream=None):
+        """Sequence dst_seqs[i] takes the whole state of src's sequence
+        src_seqs[i] (App. C: forking a candidate by copy, or committing the
+        chosen one)."""
+        kvr_cache_copy_sequences(self.handle, dst_seqs, src.handle, src_seqs,
+                                 stream)
 
     def lengths(self):
         a = np.zeros((self.S, self.L), np.int32)
