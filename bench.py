@@ -65,8 +65,8 @@ def parse():
                    help="units computed at once per SM by the fused kernel "
                         "(0: the library's choice)")
     p.add_argument("--mode", default="step",
-                   choices=["step", "helper", "fork", "crossover", "absorb",
-                            "entropy"],
+                   choices=["step", "helper", "fork", "fork-copy", "crossover",
+                            "absorb", "entropy"],
                    help="step: the evicted decode step (the headline); "
                         "helper: full-context decode of the 1.5B helper at "
                         "16k context; fork: 72B best-of-8 candidate step")
@@ -807,6 +807,91 @@ def run_fork(args):
                 kernel="kvr_fork_decode_attend_score")
 
 
+def run_fork_copy(args):
+    """The paper's own candidate mode at 72B geometry (App. C): each
+    reasoning step copies the evicted parent (B+W rows) into 8 candidate
+    sequences, every candidate token is a kvr_decode_step over all of them
+    with eviction back to B+W (64 tokens a step), and the chosen candidate is
+    copied back.  One timed step is one candidate token for all 8 candidates,
+    all layers, all sequences; the fork and commit copies are timed apart."""
+    import torch
+    from paper_2608_15797_gb300 import kvr
+    w = inputs.WORKLOADS["72b_bon8"]
+    S = args.seqs or 4
+    L, H, G, d, N = w.n_layers, w.n_kv_heads, w.group, w.head_dim, w.n_cand
+    B, Wn, T = w.budget, w.window, w.cand_step
+    dev = torch.device("cuda", 0)
+    cap = B + Wn + 1
+    parent = kvr.Cache(S, L, H, G, d, cap, "bf16", "bf16", device=dev)
+    kids = kvr.Cache(S * N, L, H, G, d, cap, "bf16", "bf16", device=dev)
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(args.seed + 29)
+    for s in range(S):
+        k = (torch.randn(L, H, B + Wn, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+        v = (torch.randn(L, H, B + Wn, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+        parent.load(s, k, v)
+    q = (torch.randn(S * N, L, H * G, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+    kn = (torch.randn(S * N, L, H, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+    vn = (torch.randn(S * N, L, H, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+    out = torch.empty(S * N, L, H * G, d, dtype=torch.bfloat16, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    src = np.repeat(np.arange(S), N).astype(np.int32)
+    dst = np.arange(S * N, dtype=np.int32)
+    chosen = (np.arange(S) * N).astype(np.int32)
+    K = max(1, min(args.steps, T * 50))
+    tok_ms, fork_ms, commit_ms = [], [], []
+    n0 = parent.launch_count() + kids.launch_count()
+    done, warm = 0, True
+
+    def copy_timed(fn):
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1)
+
+    while done < K:
+        fms = copy_timed(lambda: kids.copy_from(parent, src, dst, stream))
+
+        def step(i):
+            kvr.kvr_decode_step(kids.handle, 0, L, q, kn, vn, out, B, Wn,
+                                stream)
+        tot, per = _timed(step, T, stream)
+        cms = copy_timed(lambda: parent.copy_from(kids, chosen, np.arange(
+            S, dtype=np.int32), stream))
+        if warm:
+            warm = False
+            n0 = parent.launch_count() + kids.launch_count()
+            continue
+        tok_ms.append(per)
+        fork_ms.append(fms)
+        commit_ms.append(cms)
+        done += T
+    parent.sync_status()
+    kids.sync_status()
+    launches = parent.launch_count() + kids.launch_count() - n0
+    per_unit = cost_model.step_unit_bytes(B + Wn, d, G, 2, 2, B, Wn)
+    copy_unit = 2 * (2 * (B + Wn) * d * 2 + 8 * (B + Wn) + 16)
+    tms = float(np.mean(tok_ms))
+    return dict(metric=f"72B best-of-{N} candidate tokens/s with eviction every "
+                       f"token (B={B}, W={Wn}, {S} sequences x {L} layers x {N} "
+                       f"candidates per token, candidates by copy)",
+                total_ms=tms * done, per_ms=tms, K=done, launches=launches,
+                launch_bytes=per_unit * S * N * L * H,
+                fork_ms=float(np.mean(fork_ms)),
+                commit_ms=float(np.mean(commit_ms)),
+                fork_bytes=copy_unit * S * N * L * H,
+                amortized_steps_per_s=T / ((tms * T + float(np.mean(fork_ms))
+                                            + float(np.mean(commit_ms))) / 1e3),
+                config={"workload": "72b_bon8", "n_seq": S, "layers": L,
+                        "kv_heads": H, "group": G, "head_dim": d, "n_cand": N,
+                        "budget": B, "window": Wn, "cand_step": T,
+                        "candidates": "copies, eviction every token"},
+                kernel="kvr_decode_step over the candidate sequences")
+
+
 def print_row_line(args, r):
     peaks, peak_kind = measured_peaks()
     peak = float(peaks["hbm_gbs"])
@@ -823,8 +908,11 @@ def print_row_line(args, r):
                          "algorithmic_bytes_per_launch": r["launch_bytes"],
                          "launch_ms": r["per_ms"], "kernel": r["kernel"]},
             "gpu_launches": r["launches"]}
-    if "commit_ms" in r:
-        line["commit_ms"] = r["commit_ms"]
+    for key in ("commit_ms", "fork_ms", "amortized_steps_per_s"):
+        if key in r:
+            line[key] = r[key]
+    if "fork_bytes" in r:
+        line["fork_copy_gbs"] = r["fork_bytes"] / (r["fork_ms"] / 1e3) / 1e9
     print(json.dumps(line))
 
 
@@ -970,7 +1058,9 @@ def main():
         return 0
     if args.mode != "step":
         if rank == 0:
-            r = run_helper(args) if args.mode == "helper" else run_fork(args)
+            r = (run_helper(args) if args.mode == "helper" else
+                 run_fork_copy(args) if args.mode == "fork-copy" else
+                 run_fork(args))
             print_row_line(args, r)
         return 0
     if world > 1:
