@@ -120,6 +120,24 @@ kvr_status kvr_decode_attend_score(kvr_cache *cache, int layer_begin,
 kvr_status kvr_evict_compact(kvr_cache *cache, int layer_begin, int layer_end,
                              int budget, int window, void *stream);
 
+/* Step 4 with the redundancy-aware score of R-KV, the eviction policy of
+ * the paper's base model (App. C: cached tokens scored by a mix of
+ * query-attention importance and key redundancy by cosine similarity, mix
+ * weight lambda = 0.1, keeping the top B plus a recent window).  The paper
+ * prints no formula; this library reads it, per unit with n live rows,
+ * window rows W (the most recent) and candidates C (the rest), as
+ *   r_i = mean over live j != i of cos(k_i, k_j)   (0 for a zero key)
+ *   R_i = softmax over C of r,   I_i = s_i / sum over C of s   (0 if 0)
+ *   z_i = lambda * I_i - (1 - lambda) * R_i
+ * keeping the window and the B candidates first by (z descending, position
+ * ascending).  s is the accumulated attention score the decode calls keep,
+ * so a step with this policy is kvr_decode_attend_score followed by this
+ * call.  lambda = 1 gives kvr_evict_compact's result.  Arguments as
+ * kvr_evict_compact, plus 0 <= lambda <= 1 (KVR_EINVAL otherwise). */
+kvr_status kvr_evict_compact_rkv(kvr_cache *cache, int layer_begin,
+                                 int layer_end, int budget, int window,
+                                 float lambda, void *stream);
+
 /* Steps 1-4 fused in one pass: equivalent to kvr_decode_attend_score
  * followed by kvr_evict_compact, with the appended row written straight into
  * the slot the eviction frees. */

@@ -141,3 +141,77 @@ def check_and_adopt(o: orc.OracleCache, exports, B, W, evict=True,
                 keep_sets[s][l][h] = got
     o.keep_positions(keep_sets)
     return st
+
+
+# R-KV eviction (oracle/rkv.py): z differs from the oracle's by the fp32
+# rounding of the normalised score (the scores carry up to 1e-4 relative)
+# and of the mean cosines (about 1e-6 absolute); swaps within this bound
+# are near-ties.
+RKV_SWAP_ATOL = 2e-5
+
+
+def check_and_adopt_rkv(o: orc.OracleCache, exports, B, W, lam,
+                        layers=None) -> Stats:
+    """As check_and_adopt, for one R-KV eviction after the step: every
+    unit's CUDA retained set must be a TopB set of the oracle's z (window
+    kept, every kept candidate ranked before every evicted one, up to
+    near-ties of z), and the retained scores must match."""
+    from . import rkv
+    lb, le = (0, o.L) if layers is None else layers
+    st = Stats(steps=1)
+    sets = [[[None] * o.H for _ in range(o.L)] for _ in range(o.S)]
+    for s in range(o.S):
+        ex = exports[s]
+        for l in range(o.L):
+            for h in range(o.H):
+                n = o.len[s, l, h]
+                pos = o.pos[s, l, h, :n]
+                if not (lb <= l < le):
+                    sets[s][l][h] = pos.tolist()
+                    continue
+                where = f"seq {s} layer {l} head {h}"
+                g_n = ex["len"][l, h]
+                g_pos = ex["pos"][l, h, :g_n]
+                g_score = ex["score"][l, h, :g_n].astype(np.float64)
+                got = set(g_pos.tolist())
+                target = min(n, B + W)
+                if g_n != target or len(got) != target:
+                    raise ParityError(f"{where}: retained {g_n} rows, "
+                                      f"expected {target}")
+                if not got <= set(pos.tolist()):
+                    raise ParityError(f"{where}: unknown positions")
+                adopted = False
+                if n > B + W:
+                    want = rkv.rkv_keep(o.K[s, l, h, :n], o.score[s, l, h, :n],
+                                        pos, B, W, lam)
+                    if got != want:
+                        cand, z = rkv.rkv_scores(o.K[s, l, h, :n],
+                                                 o.score[s, l, h, :n], pos, W,
+                                                 lam)
+                        if not set(pos[~cand].tolist()) <= got:
+                            raise ParityError(f"{where}: window evicted")
+                        zc = z[cand]
+                        tol = RKV_SWAP_ATOL * float(np.abs(zc).max()) + 1e-9
+                        kept = [z[i] for i in np.nonzero(cand)[0]
+                                if pos[i] in got]
+                        lo = min(kept) if kept else np.inf
+                        for i in np.nonzero(cand)[0]:
+                            if pos[i] not in got and z[i] > lo + tol:
+                                raise ParityError(
+                                    f"{where}: evicted pos {pos[i]} (z "
+                                    f"{z[i]:.9g}) while keeping z {lo:.9g}: "
+                                    "not a near-tie")
+                        adopted = True
+                ref = dict(zip(pos.tolist(), o.score[s, l, h, :n].tolist()))
+                s_ref = np.array([ref[p] for p in g_pos.tolist()])
+                rel = np.abs(g_score - s_ref) / np.maximum(np.abs(s_ref),
+                                                           SCORE_FLOOR)
+                worst = float(rel.max()) if rel.size else 0.0
+                if worst > SCORE_RTOL:
+                    raise ParityError(f"{where}: score rel error {worst:.3g}")
+                st.units += 1
+                st.adoptions += int(adopted)
+                st.max_score_rel = max(st.max_score_rel, worst)
+                sets[s][l][h] = got
+    o.keep_positions(sets)
+    return st

@@ -748,6 +748,26 @@ kvr_status kvr_evict_compact(kvr_cache *c, int lb, int le, int budget,
   return KVR_OK;
 }
 
+kvr_status kvr_evict_compact_rkv(kvr_cache *c, int lb, int le, int budget,
+                                 int window, float lambda, void *stream) {
+  if (!c) return fail(KVR_EINVAL, "null cache");
+  if (c->forks) return fail(KVR_ESTATE, "the cache has a live fork");
+  kvr_status st = check_layers(c, lb, le);
+  if (st != KVR_OK) return st;
+  st = check_evict(budget, window);
+  if (st != KVR_OK) return st;
+  if (!(lambda >= 0.f && lambda <= 1.f))
+    return fail(KVR_EINVAL, "mix weight %g outside [0, 1]", (double)lambda);
+  const int m = max_len(c, lb, le);
+  if (m <= budget + window) return KVR_OK;
+  cudaError_t e = kvr::launch_evict_rkv(c->view, lb, le - lb, m, budget,
+                                        window, lambda, as_stream(stream));
+  if (e != cudaSuccess) return cuda_fail("kvr_evict_compact_rkv", e);
+  c->launches += 1;
+  mirror_evict(c, lb, le, budget, window);
+  return KVR_OK;
+}
+
 kvr_status kvr_absorb_chunk(kvr_cache *c, int lb, int le, int chunk,
                             const void *q, const void *k_new,
                             const void *v_new, void *out, int budget,

@@ -85,6 +85,11 @@ cudaError_t launch_attend_score_generic(const CacheView &c, const StepArgs &a,
 cudaError_t launch_attend_score_ext_scratch(const CacheView &c,
                                             const StepArgs &a, float *ext,
                                             cudaStream_t st);
+// Eviction with the R-KV score (mix weight lam in [0, 1]); the z of each
+// unit's rows is kept in its logit scratch.
+cudaError_t launch_evict_rkv(const CacheView &c, int lb, int nl, int max_rows,
+                             int budget, int window, float lam,
+                             cudaStream_t st);
 cudaError_t launch_evict_generic(const CacheView &c, int lb, int nl,
                                  int max_rows, int budget, int window,
                                  cudaStream_t st);

@@ -64,6 +64,7 @@ _SIGS = {
     "kvr_decode_step": (_S, [_P, _I, _I, _P, _P, _P, _P, _I, _I, _P]),
     "kvr_absorb_chunk": (_S, [_P, _I, _I, _I, _P, _P, _P, _P, _I, _I, _I, _P]),
     "kvr_cache_copy_sequences": (_S, [_P, _P, _P, _P, _I, _P]),
+    "kvr_evict_compact_rkv": (_S, [_P, _I, _I, _I, _I, ctypes.c_float, _P]),
     "kvr_cache_export": (_S, [_P, _I, _P, _P, _P, _P, _P, _P, _P]),
     "kvr_cache_lengths": (_S, [_P, _P]),
     "kvr_cache_launch_count": (_S, [_P, _P]),
@@ -174,6 +175,13 @@ def kvr_absorb_chunk(h, layer_begin, layer_end, chunk, q, k_new, v_new, out,
                                 _ptr(k_new), _ptr(v_new), _ptr(out), budget,
                                 window, 1 if evict else 0, _stream(stream)),
            "kvr_absorb_chunk")
+
+
+def kvr_evict_compact_rkv(h, layer_begin, layer_end, budget, window, lam,
+                          stream=None):
+    _check(lib.kvr_evict_compact_rkv(h, layer_begin, layer_end, budget, window,
+                                     float(lam), _stream(stream)),
+           "kvr_evict_compact_rkv")
 
 
 def kvr_cache_copy_sequences(dst, dst_seqs, src, src_seqs, stream=None):
@@ -302,6 +310,11 @@ class Cache:
         kvr_absorb_chunk(self.handle, lb, le, c, q, k_new, v_new, out, budget,
                          window, evict, stream)
         return out
+
+    def evict_rkv(self, budget, window, lam=0.1, layers=None, stream=None):
+        """Eviction with the R-KV score (App. C), mix weight lam."""
+        lb, le = self._layers(layers)
+        kvr_evict_compact_rkv(self.handle, lb, le, budget, window, lam, stream)
 
     def copy_from(self, src: "Cache", src_seqs, dst_seqs, stream=None):
         """Sequence dst_seqs[i] takes the whole state of src's sequence

@@ -1,0 +1,103 @@
+"""R-KV eviction (kvr_evict_compact_rkv) against the oracle's reading of it
+(oracle/rkv.py), in lock-step: every step is kvr_decode_attend_score then
+the R-KV eviction on the CUDA side, and the oracle's step without eviction
+then its R-KV eviction on the CPU side.  Outputs, retained scores and the
+retained sets are checked after every step (parity.check_and_adopt_rkv)."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import oracle as orc
+from oracle import parity, rkv
+from paper_2608_15797_gb300 import inputs, kvr
+from tests import harness
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(autouse=True)
+def _cuda():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA device")
+    torch.cuda.set_device(0)
+
+
+def rkv_lockstep(c, o, w, seed, steps, B, W, lam, step0=0):
+    stats = parity.Stats()
+    for t in range(step0, step0 + steps):
+        q, kn, vn = inputs.step_inputs(w, seed, t, c.S)
+        out = c.attend_score(*(harness.dev(a, w.dtype) for a in (q, kn, vn)))
+        c.evict_rkv(B, W, lam)
+        ref = o.step(q, kn, vn, evict=False)
+        torch.cuda.synchronize()
+        parity.check_out(out.float().cpu().numpy(), ref, what=f"out {t}")
+        exports = [c.export(s, kv=False) for s in range(c.S)]
+        stats.merge(parity.check_and_adopt_rkv(o, exports, B, W, lam))
+    c.sync_status()
+    return stats
+
+
+@pytest.mark.parametrize("lam", [0.0, 0.1, 0.5, 1.0])
+def test_rkv_tiny(lam):
+    w = inputs.WORKLOADS["tiny"]
+    c, o = harness.make_pair(w, 41, 2, cap=w.prompt + 1)
+    st = rkv_lockstep(c, o, w, 41, 30, w.budget, w.window, lam)
+    assert st.units > 0
+
+
+@pytest.mark.parametrize("lam", [0.1, 1.0])
+def test_rkv_7b(lam):
+    """7B, B = 64, W = 8: the first step evicts a 200-row prompt, then one
+    row a step."""
+    w = inputs.WORKLOADS["7b_b64"]
+    c, o = harness.make_pair(w, 42, 1, cap=201, prompt_lens=[200])
+    rkv_lockstep(c, o, w, 42, 12, w.budget, w.window, lam)
+
+
+def test_rkv_unscaled_keys_and_ragged_lengths():
+    """Peaked attention (unscaled keys), sequences of different lengths, a
+    budget of 0 and of 1."""
+    w2 = inputs.Workload("u", 3, 2, 4, 128, "bf16", 1, 3, 0, 0, sigma=1.0)
+    for wk, B in ((w2, 1), (w2, 0)):
+        c, o = harness.make_pair(wk, 43, 3, cap=40, prompt_lens=[30, 4, 0])
+        rkv_lockstep(c, o, wk, 43, 8, B, wk.window, 0.1)
+
+
+def test_rkv_duplicate_and_zero_keys():
+    """Keys that repeat, and a zero key: with lambda = 0 the duplicates are
+    the most redundant rows and go first; a zero key has cosine 0."""
+    d, n = 64, 24
+    rng = np.random.default_rng(44)
+    K = rng.standard_normal((n, d)).astype(np.float32)
+    K[5] = K[2]
+    K[9] = K[2]
+    K[14] = 0.0
+    V = rng.standard_normal((n, d)).astype(np.float32)
+    w = inputs.Workload("z", 1, 1, 2, d, "f32", 10, 2, n, 0, sigma=1.0)
+    c = kvr.Cache(1, 1, 1, 2, d, n + 1, kv_dtype="f32", out_dtype="f32")
+    o = orc.OracleCache(1, 1, 1, 2, d, n + 1)
+    c.load(0, harness.dev(K[None, None], "f32"), harness.dev(V[None, None], "f32"))
+    o.load(0, K[None, None], V[None, None])
+    q, kn, vn = inputs.step_inputs(w, 44, 0, 1)
+    c.attend_score(*(harness.dev(a, "f32") for a in (q, kn, vn)))
+    o.step(q, kn, vn, evict=False)
+    c.evict_rkv(10, 2, 0.0)
+    got = set(c.export(0, kv=False)["pos"][0, 0, :12].tolist())
+    want = rkv.rkv_keep(o.K[0, 0, 0, :n + 1], o.score[0, 0, 0, :n + 1],
+                        o.pos[0, 0, 0, :n + 1], 10, 2, 0.0)
+    assert got == want
+    assert not {2, 5, 9} <= got
+
+
+def test_rkv_errors():
+    w = inputs.WORKLOADS["tiny"]
+    c, _ = harness.make_pair(w, 45, 1, cap=w.prompt + 1)
+    for lam in (-0.1, 1.5, float("nan")):
+        with pytest.raises(kvr.KvrError) as e:
+            c.evict_rkv(w.budget, w.window, lam)
+        assert e.value.status == kvr.KVR_EINVAL
+    f = kvr.Fork(c, 2, 4)
+    with pytest.raises(kvr.KvrError) as e:
+        c.evict_rkv(w.budget, w.window, 0.1)
+    assert e.value.status == kvr.KVR_ESTATE
+    del f
