@@ -65,8 +65,8 @@ def parse():
                    help="units computed at once per SM by the fused kernel "
                         "(0: the library's choice)")
     p.add_argument("--mode", default="step",
-                   choices=["step", "helper", "fork", "fork-copy", "crossover",
-                            "absorb", "entropy"],
+                   choices=["step", "helper", "fork", "fork-copy", "rkv",
+                            "crossover", "absorb", "entropy"],
                    help="step: the evicted decode step (the headline); "
                         "helper: full-context decode of the 1.5B helper at "
                         "16k context; fork: 72B best-of-8 candidate step")
@@ -807,6 +807,83 @@ def run_fork(args):
                 kernel="kvr_fork_decode_attend_score")
 
 
+def run_rkv(args):
+    """The evicted 7B step with the paper's R-KV eviction (App. C, lambda =
+    0.1, in the library's reading): 64 sequences x 28 layers at B+W = 72
+    rows; one timed step is kvr_decode_attend_score (append, attend,
+    accumulate) and kvr_evict_compact_rkv (redundancy-aware TopB) over all
+    layers, two launches.  The accumulated-attention step (one fused
+    kvr_decode_step) is timed on the same state for comparison."""
+    import torch
+    from paper_2608_15797_gb300 import kvr
+    w = inputs.WORKLOADS["7b_b64"]
+    S = args.seqs or 64
+    L, H, G, d, B, Wn = (w.n_layers, w.n_kv_heads, w.group, w.head_dim,
+                         w.budget, w.window)
+    lam = 0.1
+    dev = torch.device("cuda", 0)
+    cache = kvr.Cache(S, L, H, G, d, B + Wn + 1, "bf16", "bf16", device=dev)
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(args.seed + 43)
+    for s in range(S):
+        k = (torch.randn(L, H, B + Wn, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+        v = (torch.randn(L, H, B + Wn, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+        cache.load(s, k, v)
+    pool = []
+    for _ in range(8):
+        q = (torch.randn(S, L, H * G, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+        kn = (torch.randn(S, L, H, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+        vn = (torch.randn(S, L, H, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+        pool.append((q, kn, vn))
+    out = torch.empty(S, L, H * G, d, dtype=torch.bfloat16, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def rkv_step(i):
+        q, kn, vn = pool[i % 8]
+        kvr.kvr_decode_attend_score(cache.handle, 0, L, q, kn, vn, out, stream)
+        kvr.kvr_evict_compact_rkv(cache.handle, 0, L, B, Wn, lam, stream)
+
+    def score_step(i):
+        q, kn, vn = pool[i % 8]
+        kvr.kvr_decode_step(cache.handle, 0, L, q, kn, vn, out, B, Wn, stream)
+
+    def timed(fn, K):
+        for i in range(max(3, args.warmup)):
+            fn(i)
+        torch.cuda.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(K):
+            fn(i)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1)
+
+    K = args.steps
+    n0 = cache.launch_count()
+    rkv_ms = timed(rkv_step, K)
+    launches = cache.launch_count() - n0 - 2 * max(3, args.warmup)
+    score_ms = timed(score_step, K)
+    cache.sync_status()
+    n = B + Wn + 1
+    attend = cost_model.step_unit_bytes(B + Wn, d, G, 2, 2, B, Wn)
+    # R-KV eviction: every key once, scores and positions, one row moved
+    evict = n * d * 2 + 8 * n + 2 * 2 * d * 2 + 8 + 16
+    units = S * L * H
+    return dict(total_ms=rkv_ms, per_ms=rkv_ms / K, K=K, launches=launches,
+                launch_bytes=(attend + evict) * units,
+                score_ms=score_ms / K,
+                metric=f"evicted decode steps/s with R-KV eviction at 7B "
+                       f"geometry, B={B}, W={Wn}, lambda={lam} ({S} sequences"
+                       f" x {L} layers per step)",
+                config={"workload": "7b_s64_b64 R-KV", "n_seq": S, "layers": L,
+                        "kv_heads": H, "group": G, "head_dim": d, "budget": B,
+                        "window": Wn, "lambda": lam},
+                kernel="kvr_decode_attend_score + kvr_evict_compact_rkv "
+                       "(bytes: the step's and one more read of every key)")
+
+
 def run_fork_copy(args):
     """The paper's own candidate mode at 72B geometry (App. C): each
     reasoning step copies the evicted parent (B+W rows) into 8 candidate
@@ -908,7 +985,7 @@ def print_row_line(args, r):
                          "algorithmic_bytes_per_launch": r["launch_bytes"],
                          "launch_ms": r["per_ms"], "kernel": r["kernel"]},
             "gpu_launches": r["launches"]}
-    for key in ("commit_ms", "fork_ms", "amortized_steps_per_s"):
+    for key in ("commit_ms", "fork_ms", "amortized_steps_per_s", "score_ms"):
         if key in r:
             line[key] = r[key]
     if "fork_bytes" in r:
@@ -1060,6 +1137,7 @@ def main():
         if rank == 0:
             r = (run_helper(args) if args.mode == "helper" else
                  run_fork_copy(args) if args.mode == "fork-copy" else
+                 run_rkv(args) if args.mode == "rkv" else
                  run_fork(args))
             print_row_line(args, r)
         return 0

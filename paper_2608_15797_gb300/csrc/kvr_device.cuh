@@ -116,5 +116,30 @@ __device__ unsigned long long block_select(int n, int need, Cand cand, Key key,
   return prefix;
 }
 
+// TopB by rank for units of at most kThreads rows, one row per thread: row
+// i is kept iff it is not a candidate, or fewer than `need` candidates have
+// a larger key (keys of candidates are distinct and nonzero).  Every thread
+// must call it; s_keep[i] holds the answer for i < n afterwards.
+template <typename Cand, typename Key>
+__device__ void block_rank_keep(int n, int need, Cand cand, Key key,
+                                unsigned long long *s_key,
+                                unsigned char *s_keep) {
+  const int i = threadIdx.x;
+  const bool ci = i < n && cand(i);
+  if (i < n) s_key[i] = ci ? key(i) : 0ull;
+  __syncthreads();
+  if (i < n) {
+    bool k = true;
+    if (ci) {
+      const unsigned long long ki = s_key[i];
+      int above = 0;
+      for (int j = 0; j < n; ++j) above += s_key[j] > ki ? 1 : 0;
+      k = above < need;
+    }
+    s_keep[i] = k ? 1 : 0;
+  }
+  __syncthreads();
+}
+
 }  // namespace dev
 }  // namespace kvr

@@ -213,14 +213,23 @@ __global__ void __launch_bounds__(kThreads)
   // position is at most newest - W.
   const int wlo = c.state[4 * x.u + 1] - 1 - W;
 
-  // Radix select of the B-th largest candidate key.
+  // TopB: by rank when every row has its own thread, else by a radix
+  // select of the B-th largest candidate key.
+  __shared__ unsigned long long s_key[kThreads];
+  __shared__ unsigned char s_keep[kThreads];
+  const bool by_rank = n <= kThreads;
   unsigned long long thr = ~0ull;
-  if (B > 0)
+  if (by_rank)
+    block_rank_keep(
+        n, B, [&](int i) { return pu[i] <= wlo; },
+        [&](int i) { return rank_key(su[i], pu[i]); }, s_key, s_keep);
+  else if (B > 0)
     thr = block_select(
         n, B, [&](int i) { return pu[i] <= wlo; },
         [&](int i) { return rank_key(su[i], pu[i]); }, hist, &s_prefix,
         &s_need);
   auto keep = [&](int i) {
+    if (by_rank) return s_keep[i] != 0;
     const int32_t p = pu[i];
     return p > wlo || (B > 0 && rank_key(su[i], p) >= thr);
   };

@@ -153,14 +153,23 @@ __global__ void __launch_bounds__(kThreads)
       z[i] = lam * (su[i] * inv_s) - (1.f - lam) * (expf(z[i] - mr) * inv_e);
   __syncthreads();
 
-  // TopB on (z, position), then compaction as in the score eviction.
+  // TopB on (z, position): by rank when every row has its own thread,
+  // else by block radix select; then compaction as in the score eviction.
+  __shared__ unsigned long long s_key[kThreads];
+  __shared__ unsigned char s_keep[kThreads];
+  const bool by_rank = n <= kThreads;
   unsigned long long thr = ~0ull;
-  if (B > 0)
+  if (by_rank)
+    block_rank_keep(
+        n, B, [&](int i) { return pu[i] <= wlo; },
+        [&](int i) { return rkv_key(z[i], pu[i]); }, s_key, s_keep);
+  else if (B > 0)
     thr = block_select(
         n, B, [&](int i) { return pu[i] <= wlo; },
         [&](int i) { return rkv_key(z[i], pu[i]); }, hist, &s_prefix,
         &s_need);
   auto keep = [&](int i) {
+    if (by_rank) return s_keep[i] != 0;
     const int32_t p = pu[i];
     return p > wlo || (B > 0 && rkv_key(z[i], p) >= thr);
   };
