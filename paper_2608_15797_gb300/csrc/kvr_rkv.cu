@@ -16,7 +16,10 @@
 // that sum), reduces the softmax and importance normalisers, and then selects
 // and compacts like the accumulated-attention eviction (block radix select
 // on (z, position), survivors above the new length moved into freed slots).
-// z is kept in the unit's logit scratch.
+// A unit of at most 256 rows whose keys fit in 96 KB is first staged in
+// shared memory (keys, scores, positions and z), with 16-byte loads; each
+// lane then reads a contiguous slice of every key.  Longer units read their
+// keys from global memory and keep z in the unit's logit scratch.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -62,18 +65,41 @@ __device__ float block_reduce(float v, Op op, float *s_red) {
   return r;
 }
 
+constexpr int kStageRows = kThreads;
+constexpr size_t kStageKeyBytes = 96 * 1024;
+
 template <typename T, int D>
+constexpr bool stageable() {
+  return (size_t)kStageRows * D * sizeof(T) <= kStageKeyBytes;
+}
+
+// Shared-memory layout of a staged unit of up to `rows` rows (a multiple of
+// 4): keys [rows][D], then z, scores and positions [rows], then the
+// holes | movers lists.
+template <typename T, int D>
+struct Staged {
+  size_t keys, z, score, pos, lists;
+  __host__ __device__ explicit Staged(int rows)
+      : keys(0),
+        z((size_t)rows * D * sizeof(T)),
+        score(z + (size_t)rows * sizeof(float)),
+        pos(score + (size_t)rows * sizeof(float)),
+        lists(pos + (size_t)rows * sizeof(int32_t)) {}
+};
+
+template <typename T, int D, bool kStaged>
 __global__ void __launch_bounds__(kThreads)
-    rkv_evict_kernel(CacheView c, int lb, int nl, int B, int W, float lam) {
+    rkv_evict_kernel(CacheView c, int lb, int nl, int B, int W, float lam,
+                     int srows) {
   pdl_begin();
-  constexpr int kPer = D / 32;  // key elements per lane
+  constexpr int kPer = D / 32;  // key elements per lane: a contiguous slice
   __shared__ unsigned hist[256];
   __shared__ unsigned long long s_prefix;
   __shared__ int s_need, s_base, s_count;
   __shared__ int s_wsum[kWarps];
   __shared__ float s_red[kWarps];
   __shared__ float s_S[kWarps][D];
-  extern __shared__ int lists[];  // holes | movers
+  extern __shared__ __align__(16) unsigned char dyn[];
 
   const struct { size_t u; } x = {unit_index(c, lb, nl)};
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -81,21 +107,42 @@ __global__ void __launch_bounds__(kThreads)
   if (n <= B + W) return;
   T *Ku = reinterpret_cast<T *>(c.K) + x.u * (size_t)c.cap * D;
   T *Vu = reinterpret_cast<T *>(c.V) + x.u * (size_t)c.cap * D;
-  float *su = c.score + x.u * (size_t)c.sstride;
-  int32_t *pu = c.pos + x.u * (size_t)c.sstride;
-  float *z = c.logits + x.u * (size_t)c.G * c.cap;
+  float *su_g = c.score + x.u * (size_t)c.sstride;
+  int32_t *pu_g = c.pos + x.u * (size_t)c.sstride;
   const int wlo = c.state[4 * x.u + 1] - 1 - W;
+  // Where the pass reads keys, scores, positions and z.
+  const T *Kr = Ku;
+  float *su = su_g, *z = c.logits + x.u * (size_t)c.G * c.cap;
+  int32_t *pu = pu_g;
+  int *lists = reinterpret_cast<int *>(dyn);
+  if constexpr (kStaged) {
+    const Staged<T, D> L(srows);
+    T *ks = reinterpret_cast<T *>(dyn + L.keys);
+    const int n16 = n * D * (int)sizeof(T) / 16;
+    for (int q = tid; q < n16; q += kThreads)
+      reinterpret_cast<int4 *>(ks)[q] = reinterpret_cast<const int4 *>(Ku)[q];
+    su = reinterpret_cast<float *>(dyn + L.score);
+    pu = reinterpret_cast<int32_t *>(dyn + L.pos);
+    z = reinterpret_cast<float *>(dyn + L.z);
+    for (int i = tid; i < n; i += kThreads) {
+      su[i] = su_g[i];
+      pu[i] = pu_g[i];
+    }
+    lists = reinterpret_cast<int *>(dyn + L.lists);
+    Kr = ks;
+    __syncthreads();
+  }
 
   // Pass 1: S = sum of the normalised keys of every live row (warp per row).
   float acc[kPer];
 #pragma unroll
   for (int j = 0; j < kPer; ++j) acc[j] = 0.f;
   for (int i = warp; i < n; i += kWarps) {
-    const T *kr = Ku + (size_t)i * D;
+    const T *kr = Kr + (size_t)i * D + lane * kPer;
     float v[kPer], ss = 0.f;
 #pragma unroll
     for (int j = 0; j < kPer; ++j) {
-      v[j] = to_f(kr[lane + 32 * j]);
+      v[j] = to_f(kr[j]);
       ss = fmaf(v[j], v[j], ss);
     }
     ss = warp_sum(ss);
@@ -104,7 +151,7 @@ __global__ void __launch_bounds__(kThreads)
     for (int j = 0; j < kPer; ++j) acc[j] = fmaf(v[j], inv, acc[j]);
   }
 #pragma unroll
-  for (int j = 0; j < kPer; ++j) s_S[warp][lane + 32 * j] = acc[j];
+  for (int j = 0; j < kPer; ++j) s_S[warp][lane * kPer + j] = acc[j];
   __syncthreads();
   for (int dd = tid; dd < D; dd += kThreads) {
     float t = 0.f;
@@ -117,13 +164,13 @@ __global__ void __launch_bounds__(kThreads)
   const float inv_n1 = 1.f / static_cast<float>(n - 1);
   for (int i = warp; i < n; i += kWarps) {
     if (pu[i] > wlo) continue;  // window rows are not ranked
-    const T *kr = Ku + (size_t)i * D;
+    const T *kr = Kr + (size_t)i * D + lane * kPer;
     float ss = 0.f, dot = 0.f;
 #pragma unroll
     for (int j = 0; j < kPer; ++j) {
-      const float v = to_f(kr[lane + 32 * j]);
+      const float v = to_f(kr[j]);
       ss = fmaf(v, v, ss);
-      dot = fmaf(v, s_S[0][lane + 32 * j], dot);
+      dot = fmaf(v, s_S[0][lane * kPer + j], dot);
     }
     ss = warp_sum(ss);
     dot = warp_sum(dot);
@@ -205,8 +252,8 @@ __global__ void __launch_bounds__(kThreads)
       vd[q] = vs[q];
     }
     if (lane == 0) {
-      su[dst] = su[src];
-      pu[dst] = pu[src];
+      su_g[dst] = su[src];
+      pu_g[dst] = pu[src];
     }
   }
   if (tid == 0) c.state[4 * x.u] = nk;
@@ -217,13 +264,18 @@ cudaError_t rkv_dispatch(const CacheView &c, int lb, int nl, int max_rows,
                          int B, int W, float lam, cudaStream_t st) {
   const int nk = B + W;
   const int max_list = max(1, min(nk, max_rows - nk));
-  const size_t bytes = 2 * (size_t)max_list * sizeof(int);
-  auto kern = rkv_evict_kernel<T, D>;
+  const size_t list_bytes = 2 * (size_t)max_list * sizeof(int);
+  const bool staged = stageable<T, D>() && max_rows <= kStageRows;
+  const int srows = (max_rows + 3) & ~3;
+  const size_t bytes =
+      staged ? Staged<T, D>(srows).lists + list_bytes : list_bytes;
+  auto kern = staged ? rkv_evict_kernel<T, D, stageable<T, D>()>
+                     : rkv_evict_kernel<T, D, false>;
   cudaError_t e = cudaFuncSetAttribute(
       kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
   if (e != cudaSuccess) return e;
   return launch_pdl(kern, dim3(c.S * nl * c.H), dim3(kThreads), bytes, st, c,
-                    lb, nl, B, W, lam);
+                    lb, nl, B, W, lam, srows);
 }
 
 }  // namespace
