@@ -72,6 +72,9 @@ def parse():
                         "16k context; fork: 72B best-of-8 candidate step")
     p.add_argument("--entropy-dtype", default="bf16", choices=["bf16", "f32"],
                    help="logit element type for --mode entropy")
+    p.add_argument("--absorb-kernel", type=int, default=0, choices=[0, 1],
+                   help="--mode absorb kernel: 0 tcgen05 (tensor memory), "
+                        "1 mma.sync")
     p.add_argument("--entropy-kernel", type=int, default=0, choices=[0, 1, 2],
                    help="--mode entropy kernel: 0 library's choice, "
                         "1 persistent streaming, 2 one CTA per piece")
@@ -604,6 +607,7 @@ def run_absorb(args):
     L, H, G, d, B, Wn, C = w.n_layers, w.n_kv_heads, w.group, w.head_dim, w.budget, w.window, 64
     dev = torch.device("cuda", 0)
     cache = kvr.Cache(S, L, H, G, d, B + Wn + C, "bf16", "bf16", device=dev)
+    cache.set_absorb_kernel(args.absorb_kernel)
     gen = torch.Generator(device=dev)
     gen.manual_seed(args.seed + 37)
     for s in range(S):
@@ -646,9 +650,14 @@ def run_absorb(args):
     # positions read and written, state
     per_unit = (2 * m * d * 2 + 2 * C * d * 2 + 2 * min(C, m) * d * 2 +
                 2 * C * G * d * 2 + 8 * m + 8 * m + 16)
-    # flops: QK^T twice (statistics pass, probability pass) and PV (hi + lo
-    # terms) over the causal triangle's mean width m + C/2
-    flops = C * G * (m + C / 2.0) * d * 2 * (2 + 2)
+    # flops over the causal triangle's mean width m + C/2: the mma.sync
+    # kernel runs QK^T twice and PV with hi + lo terms; the tcgen05 kernel
+    # runs QK^T once, PV with hi + lo, and the score column sums (hi + lo)
+    # as a 128-row tensor product over the same width
+    if args.absorb_kernel == 1:
+        flops = C * G * (m + C / 2.0) * d * 2 * (2 + 2)
+    else:
+        flops = C * G * (m + C / 2.0) * d * 2 * (1 + 2 + 2)
     return dict(total_ms=total, per_ms=total / max(1, launches), K=K,
                 launches=launches, launch_bytes=per_unit * units,
                 launch_flops=flops * units, S=S, C=C)
@@ -1074,12 +1083,14 @@ def main():
                              "peak_kind": peak_kind, "traffic": None,
                              "algorithmic_bytes_per_launch": r["launch_bytes"],
                              "launch_ms": r["per_ms"],
-                             "kernel": "kvr_absorb_chunk"},
+                             "kernel": "absorb_tc_kernel (tcgen05)"
+                             if args.absorb_kernel == 0 else
+                             "absorb_kernel (mma.sync)"},
                 "tensor": {"achieved_tflops": tfs,
                            "peak_tflops": float(peaks.get("bf16_tflops", 0)),
                            "frac": tfs / float(peaks.get("bf16_tflops", 1)),
-                           "note": "mma.sync flops incl. the second QK pass "
-                                   "and the lo term of P"},
+                           "note": "issued tensor flops over the causal "
+                                   "width, lo terms of P included"},
                 "gpu_launches": r["launches"]}))
         return 0
     if args.mode == "entropy":

@@ -394,6 +394,12 @@ kvr_status kvr_entropy_launch_count(const kvr_entropy *det, uint64_t *count);
 
 void kvr_entropy_destroy(kvr_entropy *det);
 
+/* Kernel of kvr_absorb_chunk's one-launch path (results agree within
+ * rounding): 0 = 5th-generation tensor cores with the logits, outputs and
+ * score column sums in tensor memory (the default), 1 = mma.sync with
+ * register accumulators. */
+kvr_status kvr_cache_set_absorb_kernel(kvr_cache *cache, int kernel);
+
 /* ---- the same step for callers that cannot allocate -------------------- */
 
 /* The paper has no counterpart to this call: it is a deployment variant.

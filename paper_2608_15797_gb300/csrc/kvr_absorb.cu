@@ -64,45 +64,59 @@ struct AbsorbSmem {
   static constexpr int bytes = kept + 4 * kMaxRows;
 };
 
-template <bool kOutBf16>
-__global__ void __launch_bounds__(kThreads)
-    absorb_kernel(const AbsorbParams p) {
-  pdl_begin();
-  extern __shared__ __align__(1024) unsigned char smem[];
-  __shared__ int s_base, s_count;
-  __shared__ int s_wsum[kWarps];
-  const CacheView &c = p.c;
-  const int G = c.G, C = p.chunk;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int idx = blockIdx.x;
-  const int h = idx % c.H, lr = (idx / c.H) % p.nl, sq = idx / (c.H * p.nl);
-  const size_t ug = ((size_t)sq * c.L + p.lb + lr) * c.H + h;
-  const size_t row0 = ((size_t)sq * p.nl + lr) * C;  // token 0 of this row group
-  const int n0 = c.state[4 * ug], t0 = c.state[4 * ug + 1];
-  const int n = n0 + C;
-  if (n0 < 0 || n > kMaxRows || n > c.cap) {
-    if (tid == 0) atomicOr(c.err, n > c.cap ? ERR_CAPACITY : ERR_LENGTH);
-    return;
-  }
-  __nv_bfloat16 *Ku = reinterpret_cast<__nv_bfloat16 *>(c.K) + ug * (size_t)c.cap * 128;
-  __nv_bfloat16 *Vu = reinterpret_cast<__nv_bfloat16 *>(c.V) + ug * (size_t)c.cap * 128;
-  float *su = c.score + ug * c.sstride;
-  int32_t *pu = c.pos + ug * c.sstride;
-  float *SC = reinterpret_cast<float *>(smem + AbsorbSmem::sc);
-  int32_t *PS = reinterpret_cast<int32_t *>(smem + AbsorbSmem::ps);
-  float *ACC = reinterpret_cast<float *>(smem + AbsorbSmem::acc);
-  const uint32_t sK = smem_u32(smem + AbsorbSmem::k);
-  const uint32_t sV = smem_u32(smem + AbsorbSmem::v);
+// The unit a CTA absorbs into, and where its arrays live in shared memory.
+struct Unit {
+  size_t ug, row0;
+  int h, n0, t0, n;
+  __nv_bfloat16 *Ku, *Vu;
+  float *su;
+  int32_t *pu;
+};
+struct UnitSmem {
+  unsigned char *k, *v;
+  float *sc, *acc;
+  int32_t *ps;
+  int *lists;
+  unsigned long long *key;
+  int *kept;
+};
 
-  // Rows [0, n0) from the slab, rows n0 + j from the chunk's new k/v.
+__device__ __forceinline__ bool unit_begin(const AbsorbParams &p, Unit &u) {
+  const CacheView &c = p.c;
+  const int idx = blockIdx.x;
+  u.h = idx % c.H;
+  const int lr = (idx / c.H) % p.nl, sq = idx / (c.H * p.nl);
+  u.ug = ((size_t)sq * c.L + p.lb + lr) * c.H + u.h;
+  u.row0 = ((size_t)sq * p.nl + lr) * p.chunk;  // token 0 of this row group
+  u.n0 = c.state[4 * u.ug];
+  u.t0 = c.state[4 * u.ug + 1];
+  u.n = u.n0 + p.chunk;
+  if (u.n0 < 0 || u.n > kMaxRows || u.n > c.cap) {
+    if (threadIdx.x == 0) atomicOr(c.err, u.n > c.cap ? ERR_CAPACITY : ERR_LENGTH);
+    return false;
+  }
+  u.Ku = reinterpret_cast<__nv_bfloat16 *>(c.K) + u.ug * (size_t)c.cap * 128;
+  u.Vu = reinterpret_cast<__nv_bfloat16 *>(c.V) + u.ug * (size_t)c.cap * 128;
+  u.su = c.score + u.ug * c.sstride;
+  u.pu = c.pos + u.ug * c.sstride;
+  return true;
+}
+
+// Rows [0, n0) from the slab, rows n0 + j from the chunk's new k/v; scores,
+// positions and zeroed increments.  Ends with the CTA synchronised.
+__device__ void load_unit(const AbsorbParams &p, const Unit &u,
+                          const UnitSmem &m) {
+  const CacheView &c = p.c;
+  const int tid = threadIdx.x, n = u.n, n0 = u.n0;
+  const uint32_t sK = smem_u32(m.k), sV = smem_u32(m.v);
   for (int i = tid; i < n * 16; i += kThreads) {
     const int r = i >> 4, ch = i & 15;
     const __nv_bfloat16 *ks, *vs;
     if (r < n0) {
-      ks = Ku + (size_t)r * 128;
-      vs = Vu + (size_t)r * 128;
+      ks = u.Ku + (size_t)r * 128;
+      vs = u.Vu + (size_t)r * 128;
     } else {
-      const size_t kr = (row0 + (r - n0)) * c.H + h;
+      const size_t kr = (u.row0 + (r - n0)) * c.H + u.h;
       ks = p.k_new + kr * 128;
       vs = p.v_new + kr * 128;
     }
@@ -113,17 +127,127 @@ __global__ void __launch_bounds__(kThreads)
   // zero probability; zero them so stale bits (NaN) cannot leak in.
   for (int i = tid; i < (((n + 15) & ~15) - n) * 16; i += kThreads) {
     const int r = n + (i >> 4), ch = i & 15;
-    *reinterpret_cast<int4 *>(smem + AbsorbSmem::v + swz(r, ch)) =
-        make_int4(0, 0, 0, 0);
+    *reinterpret_cast<int4 *>(m.v + swz(r, ch)) = make_int4(0, 0, 0, 0);
   }
   for (int r = tid; r < n; r += kThreads) {
-    SC[r] = r < n0 ? su[r] : 0.f;
-    PS[r] = r < n0 ? pu[r] : t0 + (r - n0);
-    ACC[r] = 0.f;
+    m.sc[r] = r < n0 ? u.su[r] : 0.f;
+    m.ps[r] = r < n0 ? u.pu[r] : u.t0 + (r - n0);
+    m.acc[r] = 0.f;
   }
   cp_async_commit_wait_all();
   __syncthreads();
+}
 
+// Scores, the TopB cut and compaction, then the unit's state.
+__device__ void finish_unit(const AbsorbParams &p, const Unit &u,
+                            const UnitSmem &m, int *s_base, int *s_count,
+                            int *s_wsum) {
+  const CacheView &c = p.c;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int n = u.n, n0 = u.n0, C = p.chunk;
+  float *SC = m.sc;
+  int32_t *PS = m.ps;
+  for (int r = tid; r < n; r += kThreads) SC[r] += m.acc[r];
+  __syncthreads();
+  const int B = p.budget, W = p.window;
+  const bool cut = p.evict && n > B + W;
+  const int wlo = u.t0 + C - 1 - W;  // a row is a candidate iff pos <= wlo
+  // TopB by rank (n <= kMaxRows <= kThreads rows, one per thread): a
+  // candidate stays iff fewer than B candidates have a larger key (keys are
+  // distinct: positions are).  Rows outside the window-free set always stay.
+  unsigned long long *KEY = m.key;
+  int *KEPT = m.kept;
+  for (int r = tid; r < n; r += kThreads)
+    KEY[r] = PS[r] <= wlo ? dev::rank_key(SC[r], PS[r]) : 0ull;
+  __syncthreads();
+  for (int r = tid; r < n; r += kThreads) {
+    int k = 1;
+    if (cut && PS[r] <= wlo) {
+      const unsigned long long mine_key = KEY[r];
+      int above = 0;
+      for (int j = 0; j < n; ++j) above += KEY[j] > mine_key ? 1 : 0;
+      k = above < B ? 1 : 0;
+    }
+    KEPT[r] = k;
+  }
+  __syncthreads();
+  auto keep = [&](int i) { return KEPT[i] != 0; };
+  if (tid == 0) *s_count = 0;
+  __syncthreads();
+  int mine = 0;
+  for (int i = tid; i < n; i += kThreads) mine += keep(i) ? 1 : 0;
+  atomicAdd(s_count, mine);
+  __syncthreads();
+  const int nk = *s_count;
+  if (cut && nk != B + W) {
+    if (tid == 0) atomicOr(c.err, ERR_LENGTH);
+    return;
+  }
+  int *holes = m.lists, *movers = m.lists + kMaxRows;
+  const int nh = dev::block_collect(0, nk, [&](int i) { return !keep(i); }, holes,
+                                    s_wsum, s_base);
+  const int nm = dev::block_collect(nk, n, keep, movers, s_wsum, s_base);
+  if (nh != nm) {
+    if (tid == 0) atomicOr(c.err, ERR_LENGTH);
+    return;
+  }
+  // Final slot of every kept row: its own below nk, a hole for a mover.
+  // Rows whose bytes must be written: new rows (r >= n0) that stay below nk,
+  // and every mover (all rows are in shared memory).
+  const uint32_t sK = smem_u32(m.k), sV = smem_u32(m.v);
+  auto write_row = [&](int src, int dst, int ln) {  // one warp-lane share
+    const int ch = ln & 15;
+    const uint32_t from = (ln < 16 ? sK : sV) + swz(src, ch);
+    int4 val;
+    asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(val.x), "=r"(val.y), "=r"(val.z), "=r"(val.w)
+                 : "r"(from));
+    __nv_bfloat16 *base = ln < 16 ? u.Ku : u.Vu;
+    reinterpret_cast<int4 *>(base + (size_t)dst * 128)[ch] = val;
+  };
+  for (int r = n0 + warp; r < nk; r += kWarps)  // new rows kept in place
+    if (keep(r)) write_row(r, r, lane);
+  for (int k = warp; k < nh; k += kWarps) write_row(movers[k], holes[k], lane);
+  for (int r = tid; r < nk; r += kThreads)
+    if (keep(r)) {
+      u.su[r] = SC[r];
+      u.pu[r] = PS[r];
+    }
+  for (int k = tid; k < nh; k += kThreads) {
+    u.su[holes[k]] = SC[movers[k]];
+    u.pu[holes[k]] = PS[movers[k]];
+  }
+  if (tid == 0) {
+    c.state[4 * u.ug] = nk;
+    c.state[4 * u.ug + 1] = u.t0 + C;
+  }
+}
+
+template <bool kOutBf16>
+__global__ void __launch_bounds__(kThreads)
+    absorb_kernel(const AbsorbParams p) {
+  pdl_begin();
+  extern __shared__ __align__(1024) unsigned char smem[];
+  __shared__ int s_base, s_count;
+  __shared__ int s_wsum[kWarps];
+  const CacheView &c = p.c;
+  const int G = c.G, C = p.chunk;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  Unit u;
+  if (!unit_begin(p, u)) return;
+  const UnitSmem m{smem + AbsorbSmem::k,
+                   smem + AbsorbSmem::v,
+                   reinterpret_cast<float *>(smem + AbsorbSmem::sc),
+                   reinterpret_cast<float *>(smem + AbsorbSmem::acc),
+                   reinterpret_cast<int32_t *>(smem + AbsorbSmem::ps),
+                   reinterpret_cast<int *>(smem + AbsorbSmem::lists),
+                   reinterpret_cast<unsigned long long *>(smem + AbsorbSmem::key),
+                   reinterpret_cast<int *>(smem + AbsorbSmem::kept)};
+  load_unit(p, u, m);
+  const int n = u.n, n0 = u.n0, h = u.h;
+  const size_t row0 = u.row0;
+  float *ACC = m.acc;
+  const uint32_t sK = smem_u32(m.k), sV = smem_u32(m.v);
   // ---- attention: 16 query rows (token-major: row = j * G + g) per task ----
   const int MQ = C * G, n_tiles = (MQ + 15) / 16;
   const int r0l = lane >> 2, c2 = (lane & 3) * 2;
@@ -287,81 +411,295 @@ __global__ void __launch_bounds__(kThreads)
   }
   __syncthreads();
 
-  // ---- scores, selection, compaction ----
-  for (int r = tid; r < n; r += kThreads) SC[r] += ACC[r];
-  __syncthreads();
-  const int B = p.budget, W = p.window;
-  const bool cut = p.evict && n > B + W;
-  const int wlo = t0 + C - 1 - W;  // a row is a candidate iff pos <= wlo
-  // TopB by rank (n <= kMaxRows <= kThreads rows, one per thread): a
-  // candidate stays iff fewer than B candidates have a larger key (keys are
-  // distinct: positions are).  Rows outside the window-free set always stay.
-  unsigned long long *KEY = reinterpret_cast<unsigned long long *>(smem + AbsorbSmem::key);
-  int *KEPT = reinterpret_cast<int *>(smem + AbsorbSmem::kept);
-  for (int r = tid; r < n; r += kThreads)
-    KEY[r] = PS[r] <= wlo ? dev::rank_key(SC[r], PS[r]) : 0ull;
-  __syncthreads();
-  for (int r = tid; r < n; r += kThreads) {
-    int k = 1;
-    if (cut && PS[r] <= wlo) {
-      const unsigned long long mine_key = KEY[r];
-      int above = 0;
-      for (int j = 0; j < n; ++j) above += KEY[j] > mine_key ? 1 : 0;
-      k = above < B ? 1 : 0;
+  finish_unit(p, u, m, &s_base, &s_count, s_wsum);
+}
+
+// ---- the same absorb on 5th-generation tensor cores ------------------------
+//
+// Query rows go in tiles of 128 (M), with the unit's keys as N (rows
+// rounded up to 16) and K = the head dimension.  Per tile:
+//   1. The tile's q rows land in shared memory (K-major, 128B swizzle) and
+//      one thread issues S = Q K^T into TMEM (fp32, N columns).
+//   2. Every warp reads its rows' logits from TMEM; warps w and w + 4 share
+//      TMEM lanes 32 (w % 4).. and take half the columns each.  They form the
+//      row statistics (an exchange through shared memory), then the exact
+//      probabilities, written as bf16 hi and lo terms into two P buffers
+//      (K-major, 128B swizzle: [64-key block][query row][128 B]).
+//   3. One thread issues O = P_hi V + P_lo V (V read MN-major) and the
+//      score column sums CS = 1 P_hi + 1 P_lo (the same P buffers read as an
+//      MN-major B operand, K = the tile's query rows) into TMEM.
+//   4. The warps write their rows' outputs from TMEM; warp 0 adds the column
+//      sums, times 1/G, to the unit's score increments.
+// Every mbarrier wait is bounded; TMEM is freed before the selection.
+constexpr int kTcRows = 128;                       // query rows per tile
+constexpr int kTcS = 0;                            // TMEM columns: S
+constexpr int kTcO = kMaxRows;                     //               O
+constexpr int kTcCS = kMaxRows + 128;              //               CS
+constexpr int kTcCols = 512;
+static_assert(kTcCS + kMaxRows <= kTcCols, "TMEM columns");
+
+struct TcSmem {  // offsets from a 1024-byte aligned base
+  static constexpr int k = 0;                              // [2][kMaxRows][128 B]
+  static constexpr int v = k + 2 * kMaxRows * 128;
+  static constexpr int ph = v + 2 * kMaxRows * 128;        // [3][128][128 B]
+  static constexpr int pl = ph + 3 * kTcRows * 128;
+  static constexpr int q = ph;                             // [2][128][128 B], aliases P hi
+  static constexpr int ones = pl + 3 * kTcRows * 128;      // [128][128 B] of 1.0
+  static constexpr int sc = ones + kTcRows * 128;
+  static constexpr int ps = sc + 4 * kMaxRows;
+  static constexpr int acc = ps + 4 * kMaxRows;
+  static constexpr int lists = acc + 4 * kMaxRows;
+  static constexpr int key = lists + 8 * kMaxRows;
+  static constexpr int kept = key + 8 * kMaxRows;
+  static constexpr int bytes = kept + 4 * kMaxRows;
+  static constexpr int alloc = bytes + 1024;               // room to align
+};
+static_assert(3 * 64 >= kMaxRows, "P holds kMaxRows keys in 64-key blocks");
+
+template <bool kOutBf16>
+__global__ void __launch_bounds__(kThreads, 1)
+    absorb_tc_kernel(const AbsorbParams p) {
+  pdl_begin();
+  extern __shared__ __align__(1024) unsigned char smem_raw[];
+  __shared__ int s_base, s_count;
+  __shared__ int s_wsum[kWarps];
+  __shared__ uint32_t s_tmem;
+  __shared__ int s_abort;
+  __shared__ __align__(8) uint64_t bar_s, bar_o;
+  __shared__ float2 s_ml[kTcRows];  // (max, sum) of the upper column halves
+  unsigned char *smem = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
+  const CacheView &c = p.c;
+  const int G = c.G, C = p.chunk;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  Unit u;
+  if (!unit_begin(p, u)) return;
+  const UnitSmem m{smem + TcSmem::k,
+                   smem + TcSmem::v,
+                   reinterpret_cast<float *>(smem + TcSmem::sc),
+                   reinterpret_cast<float *>(smem + TcSmem::acc),
+                   reinterpret_cast<int32_t *>(smem + TcSmem::ps),
+                   reinterpret_cast<int *>(smem + TcSmem::lists),
+                   reinterpret_cast<unsigned long long *>(smem + TcSmem::key),
+                   reinterpret_cast<int *>(smem + TcSmem::kept)};
+  if (warp == 0) tmem_alloc(smem_u32(&s_tmem), kTcCols);
+  if (tid == 32) {
+    mbar_init(smem_u32(&bar_s), 1);
+    mbar_init(smem_u32(&bar_o), 1);
+    s_abort = 0;
+    fence_mbar_init();
+  }
+  for (int i = tid; i < kTcRows * 128 / 4; i += kThreads)  // bf16 1.0 pairs
+    reinterpret_cast<uint32_t *>(smem + TcSmem::ones)[i] = 0x3F803F80u;
+  tc_fence_before();
+  load_unit(p, u, m);  // ends with __syncthreads
+  tc_fence_after();
+  const uint32_t tm = s_tmem;
+  const int n = u.n, n0 = u.n0, h = u.h;
+  const int MQ = C * G, n_mt = (MQ + kTcRows - 1) / kTcRows;
+  const int NS = (n + 15) & ~15;
+  const uint32_t id_s = idesc_bf16(kTcRows, NS, false);
+  const uint32_t id_o = idesc_bf16(kTcRows, 128, true);
+  const uint32_t id_c = idesc_bf16(kTcRows, NS, true);
+  const uint32_t aK = smem_u32(m.k), aV = smem_u32(m.v);
+  const uint32_t aPH = smem_u32(smem + TcSmem::ph), aPL = smem_u32(smem + TcSmem::pl);
+  const uint32_t aQ = smem_u32(smem + TcSmem::q), aOnes = smem_u32(smem + TcSmem::ones);
+  const int wq = warp & 3;             // TMEM lane quarter of this warp
+  const bool upper = warp >= 4;        // second half of the columns
+  const int half = ((NS >> 1) + 15) & ~15;
+  const int c_lo = upper ? half : 0, c_hi = upper ? NS : half;
+  const int r = wq * 32 + lane;        // this thread's row of the tile
+  const uint32_t trow = tm + ((uint32_t)(wq * 32) << 16);
+  const float scale = p.scale_log2e, inv_g = p.inv_g;
+  volatile int *abort = &s_abort;
+  bool ok = true;
+  int phase = 0;
+  auto wait_all = [&](uint64_t *bar) {
+    const bool got = mbar_wait(smem_u32(bar), (uint32_t)(phase & 1), abort);
+    const bool all = __syncthreads_and(got) != 0;
+    if (!all && tid == 0) {
+      atomicOr(c.err, ERR_TIMEOUT);
+      *abort = 1;
     }
-    KEPT[r] = k;
-  }
-  __syncthreads();
-  auto keep = [&](int i) { return KEPT[i] != 0; };
-  if (tid == 0) s_count = 0;
-  __syncthreads();
-  int mine = 0;
-  for (int i = tid; i < n; i += kThreads) mine += keep(i) ? 1 : 0;
-  atomicAdd(&s_count, mine);
-  __syncthreads();
-  const int nk = s_count;
-  if (cut && nk != B + W) {
-    if (tid == 0) atomicOr(c.err, ERR_LENGTH);
-    return;
-  }
-  int *lists = reinterpret_cast<int *>(smem + AbsorbSmem::lists);
-  int *holes = lists, *movers = lists + kMaxRows;
-  const int nh = dev::block_collect(0, nk, [&](int i) { return !keep(i); }, holes,
-                                    s_wsum, &s_base);
-  const int nm = dev::block_collect(nk, n, keep, movers, s_wsum, &s_base);
-  if (nh != nm) {
-    if (tid == 0) atomicOr(c.err, ERR_LENGTH);
-    return;
-  }
-  // Final slot of every kept row: its own below nk, a hole for a mover.
-  // Rows whose bytes must be written: new rows (r >= n0) that stay below nk,
-  // and every mover (all rows are in shared memory).
-  auto write_row = [&](int src, int dst, int ln) {  // one warp-lane share
-    const int ch = ln & 15;
-    const uint32_t from = (ln < 16 ? sK : sV) + swz(src, ch);
-    int4 val;
-    asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
-                 : "=r"(val.x), "=r"(val.y), "=r"(val.z), "=r"(val.w)
-                 : "r"(from));
-    __nv_bfloat16 *base = ln < 16 ? Ku : Vu;
-    reinterpret_cast<int4 *>(base + (size_t)dst * 128)[ch] = val;
+    tc_fence_after();
+    return all;
   };
-  for (int r = n0 + warp; r < nk; r += kWarps)  // new rows kept in place
-    if (keep(r)) write_row(r, r, lane);
-  for (int k = warp; k < nh; k += kWarps) write_row(movers[k], holes[k], lane);
-  for (int r = tid; r < nk; r += kThreads)
-    if (keep(r)) {
-      su[r] = SC[r];
-      pu[r] = PS[r];
+  for (int mt = 0; mt < n_mt && ok; ++mt, ++phase) {
+    // 1. The tile's q rows (row R = token j * G + head g); zeros past MQ.
+    for (int i = tid; i < kTcRows * 16; i += kThreads) {
+      const int rr = i >> 4, ch = i & 15, R = mt * kTcRows + rr;
+      const uint32_t dst = aQ + (ch >> 3) * (kTcRows * 128) + rr * 128 +
+                           (((ch & 7) ^ (rr & 7)) << 4);
+      if (R < MQ) {
+        const int j = R / G, g = R % G;
+        cp_async16(dst, p.q + (((u.row0 + j) * c.H + h) * G + g) * 128 + ch * 8);
+      } else {
+        asm volatile("st.shared.v4.b32 [%0], {%1, %1, %1, %1};" ::"r"(dst), "r"(0)
+                     : "memory");
+      }
     }
-  for (int k = tid; k < nh; k += kThreads) {
-    su[holes[k]] = SC[movers[k]];
-    pu[holes[k]] = PS[movers[k]];
+    cp_async_commit_wait_all();
+    fence_proxy_async();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (tid == 0) {
+      for (int k = 0; k < 8; ++k) {  // K = 128 head-dim columns, 16 a step
+        const uint32_t off = (k & 3) * 32;
+        tc_mma(tm + kTcS,
+               sdesc_sw128(aQ + (k >> 2) * (kTcRows * 128) + off, 16, 1024),
+               sdesc_sw128(aK + (k >> 2) * (kMaxRows * 128) + off, 16, 1024),
+               id_s, k > 0);
+      }
+      tc_commit(smem_u32(&bar_s));
+    }
+    if (!(ok = wait_all(&bar_s))) break;
+
+    // 2. Row statistics over this thread's columns, then the whole row.
+    const int R = mt * kTcRows + r;
+    const bool valid = R < MQ;
+    const int lim = valid ? n0 + R / G + 1 : 0;  // keys the row may see
+    float mx = -INFINITY, sm = 0.f;
+    for (int c0 = c_lo; c0 < c_hi; c0 += 16) {
+      uint32_t v[16];
+      tmem_ld16(trow + kTcS + c0, v);
+      float cm = -INFINITY;
+#pragma unroll
+      for (int j = 0; j < 16; ++j)
+        if (c0 + j < lim) cm = fmaxf(cm, __uint_as_float(v[j]) * scale);
+      if (cm > mx) {
+        sm = mx == -INFINITY ? 0.f : sm * ex2(mx - cm);
+        mx = cm;
+      }
+      if (mx > -INFINITY) {
+#pragma unroll
+        for (int j = 0; j < 16; ++j)
+          if (c0 + j < lim) sm += ex2(__uint_as_float(v[j]) * scale - mx);
+      }
+    }
+    if (upper) s_ml[r] = make_float2(mx, sm);
+    __syncthreads();
+    if (!upper) {
+      const float2 o2 = s_ml[r];
+      const float M = fmaxf(mx, o2.x);
+      const float L = (mx == -INFINITY ? 0.f : sm * ex2(mx - M)) +
+                      (o2.x == -INFINITY ? 0.f : o2.y * ex2(o2.x - M));
+      mx = M;
+      sm = L;
+      s_ml[r] = make_float2(M, L);
+    }
+    __syncthreads();
+    if (upper) {
+      const float2 o2 = s_ml[r];
+      mx = o2.x;
+      sm = o2.y;
+    }
+    if (valid && !upper && !(sm >= 1.f && sm < INFINITY)) atomicOr(c.err, ERR_NONFINITE);
+    const float inv = valid && sm > 0.f ? 1.f / sm : 0.f;
+    // Probabilities of this thread's columns as bf16 hi and lo terms.
+    for (int c0 = c_lo; c0 < c_hi; c0 += 16) {
+      uint32_t v[16];
+      tmem_ld16(trow + kTcS + c0, v);
+      uint32_t hi[8], lo[8];
+#pragma unroll
+      for (int j = 0; j < 16; j += 2) {
+        const float p0 = c0 + j < lim ? ex2(__uint_as_float(v[j]) * scale - mx) * inv : 0.f;
+        const float p1 = c0 + j + 1 < lim ? ex2(__uint_as_float(v[j + 1]) * scale - mx) * inv : 0.f;
+        const __nv_bfloat162 b = __floats2bfloat162_rn(p0, p1);
+        hi[j >> 1] = *reinterpret_cast<const uint32_t *>(&b);
+        lo[j >> 1] = pack_bf16(p0 - __low2float(b), p1 - __high2float(b));
+      }
+      const int kb = c0 >> 6, ch = (c0 & 63) >> 3;
+      const uint32_t o0 = kb * (kTcRows * 128) + r * 128 + (((ch) ^ (r & 7)) << 4);
+      const uint32_t o1 = kb * (kTcRows * 128) + r * 128 + (((ch + 1) ^ (r & 7)) << 4);
+      asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(aPH + o0), "r"(hi[0]),
+                   "r"(hi[1]), "r"(hi[2]), "r"(hi[3]) : "memory");
+      asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(aPH + o1), "r"(hi[4]),
+                   "r"(hi[5]), "r"(hi[6]), "r"(hi[7]) : "memory");
+      asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(aPL + o0), "r"(lo[0]),
+                   "r"(lo[1]), "r"(lo[2]), "r"(lo[3]) : "memory");
+      asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(aPL + o1), "r"(lo[4]),
+                   "r"(lo[5]), "r"(lo[6]), "r"(lo[7]) : "memory");
+    }
+    fence_proxy_async();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+
+    // 3. O = P V and the column sums CS = 1 P, hi and lo terms each.
+    if (tid == 0) {
+      for (int k = 0; k < NS / 16; ++k) {  // K = keys, 16 a step
+        const uint32_t pa = (k >> 2) * (kTcRows * 128) + (k & 3) * 32;
+        const uint64_t bv = sdesc_sw128(aV + k * 2048, kMaxRows * 128, 1024);
+        tc_mma(tm + kTcO, sdesc_sw128(aPH + pa, 16, 1024), bv, id_o, k > 0);
+        tc_mma(tm + kTcO, sdesc_sw128(aPL + pa, 16, 1024), bv, id_o, true);
+      }
+      for (int k = 0; k < kTcRows / 16; ++k) {  // K = the tile's query rows
+        const uint64_t ao = sdesc_sw128(aOnes + (k & 3) * 32, 16, 1024);
+        tc_mma(tm + kTcCS, ao, sdesc_sw128(aPH + k * 2048, kTcRows * 128, 1024),
+               id_c, k > 0);
+        tc_mma(tm + kTcCS, ao, sdesc_sw128(aPL + k * 2048, kTcRows * 128, 1024),
+               id_c, true);
+      }
+      tc_commit(smem_u32(&bar_o));
+    }
+    if (!(ok = wait_all(&bar_o))) break;
+
+    // 4. Outputs (this thread's row, half of the head dimension) and the
+    // column sums (every lane holds the same sums: warp 0, lane 0 adds).
+    constexpr int osz = kOutBf16 ? 2 : 4;
+    unsigned char *orow = nullptr;
+    if (valid) {
+      const int j = R / G, g = R % G;
+      orow = reinterpret_cast<unsigned char *>(p.out) +
+             ((((u.row0 + j) * c.H + h) * G + g) * 128) * osz;
+    }
+    for (int c0 = upper ? 64 : 0; c0 < (upper ? 128 : 64); c0 += 16) {
+      uint32_t v[16];
+      tmem_ld16(trow + kTcO + c0, v);
+      if (valid) {
+        if (kOutBf16) {
+          uint32_t w[8];
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            w[j] = pack_bf16(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));
+          reinterpret_cast<int4 *>(orow + c0 * 2)[0] = make_int4(w[0], w[1], w[2], w[3]);
+          reinterpret_cast<int4 *>(orow + c0 * 2)[1] = make_int4(w[4], w[5], w[6], w[7]);
+        } else {
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            reinterpret_cast<int4 *>(orow + c0 * 4)[j] =
+                make_int4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+        }
+      }
+    }
+    if (warp == 0) {
+      for (int c0 = 0; c0 < NS; c0 += 16) {
+        uint32_t v[16];
+        tmem_ld16(tm + kTcCS + c0, v);
+        if (lane == 0) {
+#pragma unroll
+          for (int j = 0; j < 16; ++j)
+            if (c0 + j < n) m.acc[c0 + j] += __uint_as_float(v[j]) * inv_g;
+        }
+      }
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
   }
-  if (tid == 0) {
-    c.state[4 * ug] = nk;
-    c.state[4 * ug + 1] = t0 + C;
+  // After a timeout, wait (bounded) once more for tensor work in flight.
+  if (!ok) {
+    volatile int never = 0;
+    if (tid == 0) {
+      mbar_wait(smem_u32(&bar_s), (uint32_t)(phase & 1), &never);
+      mbar_wait(smem_u32(&bar_o), (uint32_t)(phase & 1), &never);
+    }
   }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tm, kTcCols);
+  if (!ok) return;
+  finish_unit(p, u, m, &s_base, &s_count, s_wsum);
 }
 
 }  // namespace
@@ -369,13 +707,15 @@ __global__ void __launch_bounds__(kThreads)
 int absorb_max_chunk() { return kMaxChunk; }
 int absorb_max_rows() { return kMaxRows; }
 
-cudaError_t launch_absorb(const AbsorbParams &p, cudaStream_t st) {
+cudaError_t launch_absorb(const AbsorbParams &p, int kernel, cudaStream_t st) {
   if (p.chunk < 1 || p.chunk > kMaxChunk || p.c.G > 8 || p.c.d != 128 ||
       !p.c.kv_bf16)
     return cudaErrorInvalidValue;
   const int units = p.c.S * p.nl * p.c.H;
-  const int smem = AbsorbSmem::bytes;
-  auto kern = p.c.out_bf16 ? absorb_kernel<true> : absorb_kernel<false>;
+  const bool tc = kernel != 1;
+  const int smem = tc ? TcSmem::alloc : AbsorbSmem::bytes;
+  auto kern = tc ? (p.c.out_bf16 ? absorb_tc_kernel<true> : absorb_tc_kernel<false>)
+                 : (p.c.out_bf16 ? absorb_kernel<true> : absorb_kernel<false>);
   cudaError_t e = cudaFuncSetAttribute(
       kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;

@@ -101,6 +101,7 @@ struct kvr_cache {
   int fused_group_warps = 0;      // warps per unit (0: auto)
   int chunk_groups = 0;           // chunked kernel: groups (0 auto, -1 off)
   int chunk_stages = 0;           // chunked kernel: stages per group (0 auto)
+  int absorb_kernel = 0;          // 0 tcgen05, 1 mma.sync (kvr_absorb_chunk)
   int forks = 0;                  // live forks: the cache is read-only meanwhile
   int sm_count = 0;               // of the device, queried on first use
   int smem_optin = 0;
@@ -664,6 +665,13 @@ kvr_status kvr_cache_copy_sequences(kvr_cache *dst, const int32_t *dst_seqs,
   return KVR_OK;
 }
 
+kvr_status kvr_cache_set_absorb_kernel(kvr_cache *c, int kernel) {
+  if (!c) return fail(KVR_EINVAL, "null cache");
+  if (kernel < 0 || kernel > 1) return fail(KVR_EINVAL, "kernel must be 0 or 1");
+  c->absorb_kernel = kernel;
+  return KVR_OK;
+}
+
 kvr_status kvr_cache_set_fused(kvr_cache *c, int enable) {
   if (!c) return fail(KVR_EINVAL, "null cache");
   c->fused = enable != 0;
@@ -810,7 +818,7 @@ kvr_status kvr_absorb_chunk(kvr_cache *c, int lb, int le, int chunk,
     p.evict = evict ? 1 : 0;
     p.scale_log2e = v.scale * 1.4426950408889634f;
     p.inv_g = 1.f / (float)v.G;
-    cudaError_t e = kvr::launch_absorb(p, as_stream(stream));
+    cudaError_t e = kvr::launch_absorb(p, c->absorb_kernel, as_stream(stream));
     if (e != cudaSuccess) return cuda_fail("kvr_absorb_chunk", e);
     c->launches += 1;
     for (int j = 0; j < chunk; ++j) mirror_append(c, lb, le);

@@ -245,7 +245,8 @@ struct AbsorbParams {
 };
 int absorb_max_chunk();
 int absorb_max_rows();
-cudaError_t launch_absorb(const AbsorbParams &p, cudaStream_t st);
+// kernel: 0 the tensor-memory (tcgen05) kernel, 1 the mma.sync kernel.
+cudaError_t launch_absorb(const AbsorbParams &p, int kernel, cudaStream_t st);
 
 // Persistent chunked step (kvr_chunked.cu): bf16, d = 128, G <= 8, at most
 // chunk_max_rows() rows per job with the new row.  A job is one unit of the

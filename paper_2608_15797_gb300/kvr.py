@@ -72,6 +72,7 @@ _SIGS = {
     "kvr_cache_set_fused_tuning": (_S, [_P, _I, _I]),
     "kvr_cache_set_chunk_tuning": (_S, [_P, _I, _I]),
     "kvr_fork_set_kernel": (_S, [_P, _I]),
+    "kvr_cache_set_absorb_kernel": (_S, [_P, _I]),
     "kvr_sync_status": (_S, [_P, _P]),
     "kvr_last_error": (ctypes.c_char_p, []),
 }
@@ -345,6 +346,11 @@ class Cache:
             res["K"] = hk.float().numpy()
             res["V"] = hv.float().numpy()
         return res
+
+    def set_absorb_kernel(self, kernel: int):
+        """kvr_absorb_chunk's one-launch kernel: 0 tcgen05, 1 mma.sync."""
+        _check(lib.kvr_cache_set_absorb_kernel(self.handle, kernel),
+               "kvr_cache_set_absorb_kernel")
 
     def set_fused(self, enable: bool):
         kvr_cache_set_fused(self.handle, enable)

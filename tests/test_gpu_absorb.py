@@ -39,40 +39,52 @@ def absorb_lockstep(c, o, w, seed, chunk, B, W, evict=True, step0=20_000):
     return st
 
 
-@pytest.mark.parametrize("fused", [True, False], ids=["fused", "tokenwise"])
+# The absorb paths: the one-launch kernel on tcgen05 (default) or mma.sync,
+# and the token-by-token path (one attend+score launch a token, then one
+# eviction).
+PATHS = {"tc": (True, 0), "mma": (True, 1), "tokenwise": (False, 0)}
+
+
+def _pair(w, seed, S, cap, prompt_lens, path):
+    fused, kernel = PATHS[path]
+    c, o = harness.make_pair(w, seed, S, cap=cap, prompt_lens=prompt_lens,
+                             fused=fused)
+    c.set_absorb_kernel(kernel)
+    return c, o
+
+
+@pytest.mark.parametrize("path", list(PATHS))
 @pytest.mark.parametrize("G,d,dtype", [(7, 128, "bf16"), (1, 128, "bf16"),
                                        (8, 128, "bf16"), (3, 64, "f32")])
 @pytest.mark.parametrize("chunk", [1, 5, 33, 64])
-def test_absorb_shapes(G, d, dtype, chunk, fused):
+def test_absorb_shapes(G, d, dtype, chunk, path):
     """Ragged units (an empty one included), chunks crossing tile ends, then
-    three decode steps.  fused=False runs the token-by-token path."""
+    three decode steps."""
     B, W = 12, 4
     w = inputs.Workload("ab", 2, 2, G, d, dtype, B, W, 20, 0, sigma=1.0)
-    c, o = harness.make_pair(w, 50, 3, cap=20 + chunk + 4,
-                             prompt_lens=[20, 0, 9], fused=fused)
+    c, o = _pair(w, 50, 3, 20 + chunk + 4, [20, 0, 9], path)
     absorb_lockstep(c, o, w, 50, chunk, B, W)
     harness.lockstep(c, o, w, 50, 3, B, W, step0=100)
 
 
-@pytest.mark.parametrize("fused", [True, False], ids=["fused", "tokenwise"])
-def test_absorb_without_eviction_grows_every_unit(fused):
+@pytest.mark.parametrize("path", list(PATHS))
+def test_absorb_without_eviction_grows_every_unit(path):
     w = inputs.Workload("ab", 1, 2, 4, 128, "bf16", 8, 2, 10, 0, sigma=1.0)
-    c, o = harness.make_pair(w, 51, 2, cap=40, prompt_lens=[10, 3], fused=fused)
+    c, o = _pair(w, 51, 2, 40, [10, 3], path)
     absorb_lockstep(c, o, w, 51, 17, 8, 2, evict=False)
     assert c.lengths().tolist() == [[27], [20]]
 
 
-@pytest.mark.parametrize("fused", [True, False], ids=["fused", "tokenwise"])
-def test_absorb_7b_helper_step(fused):
+@pytest.mark.parametrize("path", list(PATHS))
+def test_absorb_7b_helper_step(path):
     """7B geometry (28 layers, G=7), an evicted cache at B+W = 72 rows absorbs
     an accepted 64-token step in one call, evicts back to 72, then decodes."""
     w = inputs.WORKLOADS["7b_unscaled"]
     B, W = w.budget, w.window
-    c, o = harness.make_pair(w, 52, 2, cap=B + W + 64 + 1,
-                             prompt_lens=[B + W, B + W - 30], fused=fused)
+    c, o = _pair(w, 52, 2, B + W + 64 + 1, [B + W, B + W - 30], path)
     n0 = c.launch_count()
     absorb_lockstep(c, o, w, 52, 64, B, W)
-    if fused:
+    if PATHS[path][0]:
         assert c.launch_count() - n0 == 1  # one launch for the whole chunk
     assert (c.lengths() <= B + W).all()
     harness.lockstep(c, o, w, 52, 4, B, W, step0=200)
@@ -104,10 +116,22 @@ def test_absorb_errors():
     assert c.lengths().tolist() == [[8]]
 
 
-def test_absorb_into_a_longer_than_budget_unit():
+@pytest.mark.parametrize("path", list(PATHS))
+def test_absorb_into_a_longer_than_budget_unit(path):
     """Units above B + W before the chunk (a prompt loaded with zero scores):
     the cut moves surviving old rows as well as placing new ones."""
     w = inputs.Workload("lo", 1, 2, 5, 128, "bf16", 16, 4, 60, 0, sigma=1.0)
-    c, o = harness.make_pair(w, 55, 2, cap=100, prompt_lens=[60, 25])
+    c, o = _pair(w, 55, 2, 100, [60, 25], path)
     absorb_lockstep(c, o, w, 55, 40, w.budget, w.window)
     harness.lockstep(c, o, w, 55, 2, w.budget, w.window, step0=300)
+
+
+@pytest.mark.parametrize("path", ["tc", "mma"])
+def test_absorb_full_unit_and_128_row_tiles(path):
+    """The largest unit the one-launch kernels take (128 old rows + a
+    64-token chunk = 192 rows) and G = 8, so the 512 query rows fill four
+    128-row tiles exactly."""
+    w = inputs.Workload("fu", 2, 2, 8, 128, "bf16", 100, 8, 128, 0, sigma=1.0)
+    c, o = _pair(w, 56, 2, 192, [128, 127], path)
+    absorb_lockstep(c, o, w, 56, 64, w.budget, w.window)
+    harness.lockstep(c, o, w, 56, 2, w.budget, w.window, step0=400)
