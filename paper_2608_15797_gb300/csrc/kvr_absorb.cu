@@ -418,8 +418,10 @@ __global__ void __launch_bounds__(kThreads)
 //
 // Query rows go in tiles of 128 (M), with the unit's keys as N (rows
 // rounded up to 16) and K = the head dimension.  Per tile:
-//   1. The tile's q rows land in shared memory (K-major, 128B swizzle) and
-//      one thread issues S = Q K^T into TMEM (fp32, N columns).
+//   1. The tile's q rows are in shared memory (K-major, 128B swizzle, in the
+//      P lo buffer: loaded with the unit for the first tile, during the
+//      previous tile's output phase for the others) and one thread issues
+//      S = Q K^T into TMEM (fp32, N columns).
 //   2. Every warp reads its rows' logits from TMEM; warps w and w + 4 share
 //      TMEM lanes 32 (w % 4).. and take half the columns each.  They form the
 //      row statistics (an exchange through shared memory), then the exact
@@ -443,7 +445,7 @@ struct TcSmem {  // offsets from a 1024-byte aligned base
   static constexpr int v = k + 2 * kMaxRows * 128;
   static constexpr int ph = v + 2 * kMaxRows * 128;        // [3][128][128 B]
   static constexpr int pl = ph + 3 * kTcRows * 128;
-  static constexpr int q = ph;                             // [2][128][128 B], aliases P hi
+  static constexpr int q = pl;                             // [2][128][128 B], aliases P lo
   static constexpr int ones = pl + 3 * kTcRows * 128;      // [128][128 B] of 1.0
   static constexpr int sc = ones + kTcRows * 128;
   static constexpr int ps = sc + 4 * kMaxRows;
@@ -490,19 +492,37 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   for (int i = tid; i < kTcRows * 128 / 4; i += kThreads)  // bf16 1.0 pairs
     reinterpret_cast<uint32_t *>(smem + TcSmem::ones)[i] = 0x3F803F80u;
-  tc_fence_before();
-  load_unit(p, u, m);  // ends with __syncthreads
-  tc_fence_after();
-  const uint32_t tm = s_tmem;
   const int n = u.n, n0 = u.n0, h = u.h;
   const int MQ = C * G, n_mt = (MQ + kTcRows - 1) / kTcRows;
+  const uint32_t aQ = smem_u32(smem + TcSmem::q);
+  // Tile mt's q rows (row R = token j * G + head g), zeros past MQ, into the
+  // Q buffer with cp.async (completed by the next commit-and-wait).
+  auto load_q = [&](int mt) {
+    for (int i = tid; i < kTcRows * 16; i += kThreads) {
+      const int rr = i >> 4, ch = i & 15, R = mt * kTcRows + rr;
+      const uint32_t dst = aQ + (ch >> 3) * (kTcRows * 128) + rr * 128 +
+                           (((ch & 7) ^ (rr & 7)) << 4);
+      if (R < MQ) {
+        const int j = R / G, g = R % G;
+        cp_async16(dst, p.q + (((u.row0 + j) * c.H + h) * G + g) * 128 + ch * 8);
+      } else {
+        asm volatile("st.shared.v4.b32 [%0], {%1, %1, %1, %1};" ::"r"(dst), "r"(0)
+                     : "memory");
+      }
+    }
+  };
+  load_q(0);
+  tc_fence_before();
+  load_unit(p, u, m);  // ends with the copies complete and __syncthreads
+  tc_fence_after();
+  const uint32_t tm = s_tmem;
   const int NS = (n + 15) & ~15;
   const uint32_t id_s = idesc_bf16(kTcRows, NS, false);
   const uint32_t id_o = idesc_bf16(kTcRows, 128, true);
   const uint32_t id_c = idesc_bf16(kTcRows, NS, true);
   const uint32_t aK = smem_u32(m.k), aV = smem_u32(m.v);
   const uint32_t aPH = smem_u32(smem + TcSmem::ph), aPL = smem_u32(smem + TcSmem::pl);
-  const uint32_t aQ = smem_u32(smem + TcSmem::q), aOnes = smem_u32(smem + TcSmem::ones);
+  const uint32_t aOnes = smem_u32(smem + TcSmem::ones);
   const int wq = warp & 3;             // TMEM lane quarter of this warp
   const bool upper = warp >= 4;        // second half of the columns
   const int half = ((NS >> 1) + 15) & ~15;
@@ -524,19 +544,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     return all;
   };
   for (int mt = 0; mt < n_mt && ok; ++mt, ++phase) {
-    // 1. The tile's q rows (row R = token j * G + head g); zeros past MQ.
-    for (int i = tid; i < kTcRows * 16; i += kThreads) {
-      const int rr = i >> 4, ch = i & 15, R = mt * kTcRows + rr;
-      const uint32_t dst = aQ + (ch >> 3) * (kTcRows * 128) + rr * 128 +
-                           (((ch & 7) ^ (rr & 7)) << 4);
-      if (R < MQ) {
-        const int j = R / G, g = R % G;
-        cp_async16(dst, p.q + (((u.row0 + j) * c.H + h) * G + g) * 128 + ch * 8);
-      } else {
-        asm volatile("st.shared.v4.b32 [%0], {%1, %1, %1, %1};" ::"r"(dst), "r"(0)
-                     : "memory");
-      }
-    }
+    // 1. The tile's q rows have landed (issued earlier).
     cp_async_commit_wait_all();
     fence_proxy_async();
     tc_fence_before();
@@ -643,9 +651,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_commit(smem_u32(&bar_o));
     }
     if (!(ok = wait_all(&bar_o))) break;
+    if (mt + 1 < n_mt) load_q(mt + 1);  // P lo is free until the next softmax
 
     // 4. Outputs (this thread's row, half of the head dimension) and the
-    // column sums (every lane holds the same sums: warp 0, lane 0 adds).
+    // column sums (every lane of warp 0 holds the same sums).
     constexpr int osz = kOutBf16 ? 2 : 4;
     unsigned char *orow = nullptr;
     if (valid) {
@@ -672,15 +681,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
-    if (warp == 0) {
-      for (int c0 = 0; c0 < NS; c0 += 16) {
+    // Every TMEM lane holds the same sums: warp w reads 16-column chunk w,
+    // w + 8, ... from its own lane quarter, and lane j adds column c0 + j.
+    {
+      for (int c0 = 16 * warp; c0 < NS; c0 += 16 * kWarps) {
         uint32_t v[16];
-        tmem_ld16(tm + kTcCS + c0, v);
-        if (lane == 0) {
+        tmem_ld16(trow + kTcCS + c0, v);
+        float mine = 0.f;
 #pragma unroll
-          for (int j = 0; j < 16; ++j)
-            if (c0 + j < n) m.acc[c0 + j] += __uint_as_float(v[j]) * inv_g;
-        }
+        for (int j = 0; j < 16; ++j)
+          if (lane == j) mine = __uint_as_float(v[j]);
+        if (lane < 16 && c0 + lane < n) m.acc[c0 + lane] += mine * inv_g;
       }
     }
     tc_fence_before();
