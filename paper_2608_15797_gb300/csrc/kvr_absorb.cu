@@ -438,6 +438,7 @@ constexpr int kTcS = 0;                            // TMEM columns: S
 constexpr int kTcO = kMaxRows;                     //               O
 constexpr int kTcCS = kMaxRows + 128;              //               CS
 constexpr int kTcCols = 512;
+constexpr int kTcChunks = (kMaxRows / 2 + 15) / 16;  // a thread's column chunks
 static_assert(kTcCS + kMaxRows <= kTcCols, "TMEM columns");
 
 struct TcSmem {  // offsets from a 1024-byte aligned base
@@ -562,71 +563,86 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     if (!(ok = wait_all(&bar_s))) break;
 
-    // 2. Row statistics over this thread's columns, then the whole row.
+    // 2. This thread's logits (at most kTcChunks 16-column chunks) read
+    // from TMEM once, exponentiated once against the thread's own maximum;
+    // the row's maximum and sum come from an exchange with the partner warp,
+    // and the probabilities are the thread's terms rescaled.
     const int R = mt * kTcRows + r;
     const bool valid = R < MQ;
     const int lim = valid ? n0 + R / G + 1 : 0;  // keys the row may see
-    float mx = -INFINITY, sm = 0.f;
-    for (int c0 = c_lo; c0 < c_hi; c0 += 16) {
-      uint32_t v[16];
-      tmem_ld16(trow + kTcS + c0, v);
-      float cm = -INFINITY;
+    const int nch = (c_hi - c_lo) >> 4;
+    float e[kTcChunks][16];
+    float mx = -INFINITY;
 #pragma unroll
-      for (int j = 0; j < 16; ++j)
-        if (c0 + j < lim) cm = fmaxf(cm, __uint_as_float(v[j]) * scale);
-      if (cm > mx) {
-        sm = mx == -INFINITY ? 0.f : sm * ex2(mx - cm);
-        mx = cm;
+    for (int k = 0; k < kTcChunks; ++k)
+      if (k < nch) tmem_ld16f_nowait(trow + kTcS + c_lo + 16 * k, e[k]);
+    tmem_wait_ld();
+#pragma unroll
+    for (int k = 0; k < kTcChunks; ++k) {
+      if (k < nch) {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          const bool in = c_lo + 16 * k + j < lim;
+          e[k][j] = in ? e[k][j] * scale : -INFINITY;
+          mx = fmaxf(mx, e[k][j]);
+        }
       }
-      if (mx > -INFINITY) {
+    }
+    float sm = 0.f;
+    const float ref = mx == -INFINITY ? 0.f : mx;
 #pragma unroll
-        for (int j = 0; j < 16; ++j)
-          if (c0 + j < lim) sm += ex2(__uint_as_float(v[j]) * scale - mx);
+    for (int k = 0; k < kTcChunks; ++k) {
+      if (k < nch) {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          e[k][j] = ex2(e[k][j] - ref);  // exp2(-inf) = 0 for masked keys
+          sm += e[k][j];
+        }
       }
     }
     if (upper) s_ml[r] = make_float2(mx, sm);
     __syncthreads();
+    float M = mx, L = sm;
     if (!upper) {
       const float2 o2 = s_ml[r];
-      const float M = fmaxf(mx, o2.x);
-      const float L = (mx == -INFINITY ? 0.f : sm * ex2(mx - M)) +
-                      (o2.x == -INFINITY ? 0.f : o2.y * ex2(o2.x - M));
-      mx = M;
-      sm = L;
+      M = fmaxf(mx, o2.x);
+      L = (mx == -INFINITY ? 0.f : sm * ex2(mx - M)) +
+          (o2.x == -INFINITY ? 0.f : o2.y * ex2(o2.x - M));
       s_ml[r] = make_float2(M, L);
     }
     __syncthreads();
     if (upper) {
       const float2 o2 = s_ml[r];
-      mx = o2.x;
-      sm = o2.y;
+      M = o2.x;
+      L = o2.y;
     }
-    if (valid && !upper && !(sm >= 1.f && sm < INFINITY)) atomicOr(c.err, ERR_NONFINITE);
-    const float inv = valid && sm > 0.f ? 1.f / sm : 0.f;
-    // Probabilities of this thread's columns as bf16 hi and lo terms.
-    for (int c0 = c_lo; c0 < c_hi; c0 += 16) {
-      uint32_t v[16];
-      tmem_ld16(trow + kTcS + c0, v);
-      uint32_t hi[8], lo[8];
+    if (valid && !upper && !(L >= 1.f && L < INFINITY)) atomicOr(c.err, ERR_NONFINITE);
+    // p = e * exp2(own max - row max) / row sum
+    const float f = valid && L > 0.f && mx > -INFINITY ? ex2(mx - M) / L : 0.f;
 #pragma unroll
-      for (int j = 0; j < 16; j += 2) {
-        const float p0 = c0 + j < lim ? ex2(__uint_as_float(v[j]) * scale - mx) * inv : 0.f;
-        const float p1 = c0 + j + 1 < lim ? ex2(__uint_as_float(v[j + 1]) * scale - mx) * inv : 0.f;
-        const __nv_bfloat162 b = __floats2bfloat162_rn(p0, p1);
-        hi[j >> 1] = *reinterpret_cast<const uint32_t *>(&b);
-        lo[j >> 1] = pack_bf16(p0 - __low2float(b), p1 - __high2float(b));
+    for (int k = 0; k < kTcChunks; ++k) {
+      if (k < nch) {
+        const int c0 = c_lo + 16 * k;
+        uint32_t hi[8], lo[8];
+#pragma unroll
+        for (int j = 0; j < 16; j += 2) {
+          const float p0 = e[k][j] * f, p1 = e[k][j + 1] * f;
+          const __nv_bfloat162 b = __floats2bfloat162_rn(p0, p1);
+          hi[j >> 1] = *reinterpret_cast<const uint32_t *>(&b);
+          lo[j >> 1] = pack_bf16(p0 - __low2float(b), p1 - __high2float(b));
+        }
+        const int kb = c0 >> 6, ch = (c0 & 63) >> 3;
+        const uint32_t o0 = kb * (kTcRows * 128) + r * 128 + (((ch) ^ (r & 7)) << 4);
+        const uint32_t o1 = kb * (kTcRows * 128) + r * 128 + (((ch + 1) ^ (r & 7)) << 4);
+        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(aPH + o0), "r"(hi[0]),
+                     "r"(hi[1]), "r"(hi[2]), "r"(hi[3]) : "memory");
+        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(aPH + o1), "r"(hi[4]),
+                     "r"(hi[5]), "r"(hi[6]), "r"(hi[7]) : "memory");
+        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(aPL + o0), "r"(lo[0]),
+                     "r"(lo[1]), "r"(lo[2]), "r"(lo[3]) : "memory");
+        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(aPL + o1), "r"(lo[4]),
+                     "r"(lo[5]), "r"(lo[6]), "r"(lo[7]) : "memory");
       }
-      const int kb = c0 >> 6, ch = (c0 & 63) >> 3;
-      const uint32_t o0 = kb * (kTcRows * 128) + r * 128 + (((ch) ^ (r & 7)) << 4);
-      const uint32_t o1 = kb * (kTcRows * 128) + r * 128 + (((ch + 1) ^ (r & 7)) << 4);
-      asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(aPH + o0), "r"(hi[0]),
-                   "r"(hi[1]), "r"(hi[2]), "r"(hi[3]) : "memory");
-      asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(aPH + o1), "r"(hi[4]),
-                   "r"(hi[5]), "r"(hi[6]), "r"(hi[7]) : "memory");
-      asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(aPL + o0), "r"(lo[0]),
-                   "r"(lo[1]), "r"(lo[2]), "r"(lo[3]) : "memory");
-      asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(aPL + o1), "r"(lo[4]),
-                   "r"(lo[5]), "r"(lo[6]), "r"(lo[7]) : "memory");
     }
     fence_proxy_async();
     tc_fence_before();
@@ -662,9 +678,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       orow = reinterpret_cast<unsigned char *>(p.out) +
              ((((u.row0 + j) * c.H + h) * G + g) * 128) * osz;
     }
-    for (int c0 = upper ? 64 : 0; c0 < (upper ? 128 : 64); c0 += 16) {
-      uint32_t v[16];
-      tmem_ld16(trow + kTcO + c0, v);
+    uint32_t ov[4][16];
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+      tmem_ld16_nowait(trow + kTcO + (upper ? 64 : 0) + 16 * k, ov[k]);
+    tmem_wait_ld();
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int c0 = (upper ? 64 : 0) + 16 * k;
+      const uint32_t(&v)[16] = ov[k];
       if (valid) {
         if (kOutBf16) {
           uint32_t w[8];
