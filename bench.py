@@ -243,6 +243,35 @@ def committed_traffic(name):
     return d.get("dram_bytes_per_launch")
 
 
+# --------------------------------------------------------------------------
+# ranks: weak scaling, each rank its own sequences, no data-path collective
+# --------------------------------------------------------------------------
+
+def rank_seeds(seed, rank):
+    """Seeds of rank `rank`'s prior lengths and of its inputs: every rank
+    decodes its own sequences (weak scaling)."""
+    return seed + 7919 * rank, 1_000_003 * (seed + 1) + rank
+
+
+def max_over_ranks(x, device=None):
+    """The largest of every rank's x (the job ends with its slowest rank);
+    x itself outside a process group of more than one rank."""
+    import torch
+    dist = torch.distributed
+    if not (dist.is_available() and dist.is_initialized()) or \
+            dist.get_world_size() == 1:
+        return float(x)
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_rate(world, units_per_rank, max_ms):
+    """Whole-job throughput: the units all ranks processed over the slowest
+    rank's time."""
+    return world * units_per_rank / (max_ms / 1e3)
+
+
 def run_kvr(args, rank, world, local_rank):
     import torch
     from paper_2608_15797_gb300 import kvr
@@ -252,8 +281,8 @@ def run_kvr(args, rank, world, local_rank):
     w = inputs.WORKLOADS[args.workload]
     S, L, H, G, d = w.n_seq, w.n_layers, w.n_kv_heads, w.group, w.head_dim
     B, W = w.budget, w.window
-    lens = inputs.prior_lengths(args.seed + 7919 * rank, S, args.prior_min,
-                                args.prior_max)
+    len_seed, in_seed = rank_seeds(args.seed, rank)
+    lens = inputs.prior_lengths(len_seed, S, args.prior_min, args.prior_max)
     cap = int(lens.max()) + 1
     cache = kvr.Cache(S, L, H, G, d, cap, kv_dtype="bf16", out_dtype="bf16",
                       device=dev)
@@ -264,7 +293,7 @@ def run_kvr(args, rank, world, local_rank):
         kvr.kvr_cache_set_chunk_tuning(cache.handle, args.chunk_groups,
                                        args.chunk_stages)
     gen = torch.Generator(device=dev)
-    gen.manual_seed(1_000_003 * (args.seed + 1) + rank)
+    gen.manual_seed(in_seed)
     for s in range(S):
         n = int(lens[s])
         k = (torch.randn(L, H, n, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
@@ -356,10 +385,7 @@ def run_kvr(args, rank, world, local_rank):
     cache.sync_status()
     del lpool, lout
 
-    if world > 1:
-        t = torch.tensor([total_ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(total_ms, dev)
 
     # End to end through the public call: pinned host inputs in, output out.
     hpool = [tuple(x.cpu().pin_memory() for x in p) for p in pool[:4]]
@@ -380,7 +406,7 @@ def run_kvr(args, rank, world, local_rank):
         hout.copy_(out, non_blocking=True)
     e1.record(stream)
     torch.cuda.synchronize()
-    e2e_ms = e0.elapsed_time(e1)
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), dev)
     cache.sync_status()
 
     unit_bytes = cost_model.step_unit_bytes(B + W, d, G, 2, 2, B, W)
@@ -1162,7 +1188,7 @@ def main():
 
     peaks, peak_kind = measured_peaks()
     peak = float(peaks["hbm_gbs"])
-    steps_per_s = world * r["K"] / (r["total_ms"] / 1e3)
+    steps_per_s = job_rate(world, r["K"], r["total_ms"])
     achieved = r["launch_bytes"] / (r["per_launch_ms"] / 1e3) / 1e9
     lat = run_latency_s1(args, local_rank) if world == 1 else None
     cpu = None
@@ -1209,7 +1235,7 @@ def main():
                      "launch_ms": r["per_launch_ms"],
                      "launch_timing": "timed region / launches in it",
                      "kernel": "kvr_decode_step (all layers, one call)"},
-        "e2e": {"value": world * r["Ke"] / (r["e2e_ms"] / 1e3),
+        "e2e": {"value": job_rate(world, r["Ke"], r["e2e_ms"]),
                 "unit": "steps/s", "h2d_bytes_per_step": r["bi"],
                 "d2h_bytes_per_step": r["bo"]},
         "gpu_launches": r["launches"],
