@@ -444,6 +444,19 @@ kvr_status kvr_cache_export(const kvr_cache *cache, int seq, void *host_k,
                             int32_t *host_len, int32_t *host_next_pos,
                             void *stream);
 
+/* The scores half of the step's result, with no copy: device pointers into
+ * the caller's cache buffer, valid for the cache's lifetime.
+ *   score  [S][L][H][row_stride] fp32: the accumulated importance score of
+ *          the row in each slot (Sec. 2.1)
+ *   pos    [S][L][H][row_stride] int32: the row's position (token index)
+ *   state  [S][L][H][4] int32: live length, next position, 0, 0
+ * Slots [0, live length) of a unit hold its rows, in no particular order.
+ * The values are those after the last call enqueued on the cache's stream;
+ * read them stream-ordered.  Any output pointer may be NULL. */
+kvr_status kvr_cache_scores(const kvr_cache *cache, float **score,
+                            int32_t **pos, int32_t **state,
+                            int64_t *row_stride);
+
 /* Host mirror of the live length of every (sequence, layer): host_len
  * [S][L].  Not synchronising (the mirror is exact after every call). */
 kvr_status kvr_cache_lengths(const kvr_cache *cache, int32_t *host_len);

@@ -918,6 +918,17 @@ kvr_status kvr_cache_lengths(const kvr_cache *c, int32_t *host_len) {
   return KVR_OK;
 }
 
+kvr_status kvr_cache_scores(const kvr_cache *c, float **score,
+                            int32_t **pos, int32_t **state,
+                            int64_t *row_stride) {
+  if (!c) return fail(KVR_EINVAL, "null cache");
+  if (score) *score = c->view.score;
+  if (pos) *pos = c->view.pos;
+  if (state) *state = c->view.state;
+  if (row_stride) *row_stride = c->view.sstride;
+  return KVR_OK;
+}
+
 kvr_status kvr_cache_launch_count(const kvr_cache *c, uint64_t *count) {
   if (!c || !count) return fail(KVR_EINVAL, "null argument");
   *count = c->launches;

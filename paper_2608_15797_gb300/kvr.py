@@ -73,6 +73,7 @@ _SIGS = {
     "kvr_cache_set_chunk_tuning": (_S, [_P, _I, _I]),
     "kvr_fork_set_kernel": (_S, [_P, _I]),
     "kvr_cache_set_absorb_kernel": (_S, [_P, _I]),
+    "kvr_cache_scores": (_S, [_P, _P, _P, _P, _P]),
     "kvr_sync_status": (_S, [_P, _P]),
     "kvr_last_error": (ctypes.c_char_p, []),
 }
@@ -346,6 +347,27 @@ class Cache:
             res["K"] = hk.float().numpy()
             res["V"] = hv.float().numpy()
         return res
+
+    def scores_view(self):
+        """(score, pos, state) as device tensors viewing the cache buffer (no
+        copy): score and pos [S][L][H][row_stride], state [S][L][H][4]."""
+        sp, pp, stp = _P(), _P(), _P()
+        stride = ctypes.c_int64()
+        _check(lib.kvr_cache_scores(self.handle, ctypes.byref(sp), ctypes.byref(pp),
+                                    ctypes.byref(stp), ctypes.byref(stride)),
+               "kvr_cache_scores")
+        base = self.buf.data_ptr()
+        rows = self.S * self.L * self.H * stride.value
+
+        def view(ptr, n, dtype):
+            off = ptr.value - base
+            return self.buf[off:off + 4 * n].view(dtype)
+
+        shape = (self.S, self.L, self.H, stride.value)
+        return (view(sp, rows, torch.float32).view(shape),
+                view(pp, rows, torch.int32).view(shape),
+                view(stp, self.S * self.L * self.H * 4, torch.int32).view(
+                    self.S, self.L, self.H, 4))
 
     def set_absorb_kernel(self, kernel: int):
         """kvr_absorb_chunk's one-launch kernel: 0 tcgen05, 1 mma.sync."""

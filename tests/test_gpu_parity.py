@@ -240,3 +240,24 @@ def test_chunked_ring_configurations_agree_bitwise():
                     n = int(ea["len"][l, h])  # rows past len are unset memory
                     for key in ("pos", "score", "K", "V"):
                         assert np.array_equal(ea[key][l, h, :n], eb[key][l, h, :n])
+
+
+def test_scores_view_matches_export():
+    """kvr_cache_scores: the step's scores read in place on the device agree
+    with the synchronising export, slot for slot."""
+    w = inputs.WORKLOADS["tiny"]
+    c, o = harness.make_pair(w, 61, 2, cap=w.prompt + 1)
+    harness.lockstep(c, o, w, 61, 5, w.budget, w.window)
+    score, pos, state = c.scores_view()
+    torch.cuda.synchronize()
+    for s in range(2):
+        e = c.export(s, kv=False)
+        n = e["len"]
+        assert np.array_equal(state[s, :, :, 0].cpu().numpy(), n)
+        for l in range(c.L):
+            for h in range(c.H):
+                k = n[l, h]
+                assert np.array_equal(score[s, l, h, :k].cpu().numpy(),
+                                      e["score"][l, h, :k])
+                assert np.array_equal(pos[s, l, h, :k].cpu().numpy(),
+                                      e["pos"][l, h, :k])
