@@ -9,11 +9,11 @@
 //
 // The work is one read of every logit, so the kernel is an HBM stream.
 // `entropy_stream_kernel` (rows 16-byte aligned) is persistent: a multiple of
-// the SM count of CTAs, each streaming one contiguous, equal span of the
-// [rows][vocab] logits.  In each CTA one producer thread moves 16 KB stages
-// into a six-stage shared-memory ring with cp.async.bulk (completion on an
-// mbarrier) and eight consumer warps reduce them, so HBM reads and the
-// arithmetic overlap.  `entropy_kernel` (any alignment) cuts each row into
+// the SM count of CTAs (three a SM), each streaming one contiguous, equal
+// span of the [rows][vocab] logits.  In each CTA one producer thread moves
+// 16 KB stages into a four-stage shared-memory ring with cp.async.bulk
+// (completion on an mbarrier) and eight consumer warps reduce them, so HBM
+// reads and the arithmetic overlap.  `entropy_kernel` (any alignment) cuts each row into
 // pieces of 2,048 16-byte vectors (16,384 bf16 or 8,192 fp32 logits), one
 // CTA each.  Both keep an online softmax in base 2:
 //   y = x * log2(e) / T,  m = max y,  s = sum 2^(y - m),
@@ -401,7 +401,9 @@ __global__ void __launch_bounds__(kThreads, 4)
 constexpr int kSWarps = 8;                    // consumer warps
 constexpr int kSThreads = (kSWarps + 1) * 32;  // + one producer warp
 constexpr int kStageVecs = 1024;              // 16 KB a stage
-constexpr int kSStages = 6;
+constexpr int kSStages = 4;                   // three CTAs fit an SM
+static_assert(kStageVecs % (kSWarps * 32) == 0,
+              "every consumer thread takes the same number of vectors");
 constexpr size_t kStreamSmem =
     static_cast<size_t>(kSStages) * kStageVecs * 16 + kSStages * 16 +
     2 * kSStages * 8;
@@ -450,7 +452,7 @@ __device__ void segment_done(const EntropyView &v, const StepIO &io, int r,
 // vocab % (16 / element size) logits go with the segment holding its last
 // whole vector.
 template <bool kBf16>
-__global__ void __launch_bounds__(kSThreads, 2)
+__global__ void __launch_bounds__(kSThreads, 3)
     entropy_stream_kernel(const EntropyView v, const StepIO io,
                           const long long span, const int nvf) {
   using namespace kvr::ptx;
