@@ -16,6 +16,7 @@
 // that sum), reduces the softmax and importance normalisers, and then selects
 // and compacts like the accumulated-attention eviction (block radix select
 // on (z, position), survivors above the new length moved into freed slots).
+// Units of at most 128 rows (the steady state) take one warp each (below).
 // A unit of at most 256 rows whose keys fit in 96 KB is first staged in
 // shared memory (keys, scores, positions and z), with 16-byte loads; each
 // lane then reads a contiguous slice of every key.  Longer units read their
@@ -259,12 +260,238 @@ __global__ void __launch_bounds__(kThreads)
   if (tid == 0) c.state[4 * x.u] = nk;
 }
 
+// ---- one warp per unit (units of at most 128 rows: the steady state) -------
+//
+// The same arithmetic with no CTA-wide synchronisation: eight units a CTA,
+// one a warp.  In the key passes each half-warp takes one row (16 lanes x
+// D/16 elements, 16-byte loads for bf16 d = 128), so a warp reads two rows a
+// step and keeps D/16 elements of the normalised-key sum per lane.  For the
+// ranking every lane owns rows lane, lane + 32, ...; the warp's candidates
+// rank by counting larger keys, and ballots build the hole and mover lists.
+constexpr int kWarpRows = 128;
+
+template <typename T, int D>
+__global__ void __launch_bounds__(kThreads)
+    rkv_evict_warp_kernel(CacheView c, int lb, int nl, int B, int W, float lam,
+                          int units) {
+  pdl_begin();
+  constexpr int kE = D / 16;  // elements of a row per half-warp lane
+  constexpr int kR = kWarpRows / 32;
+  __shared__ float s_r[kWarps][kWarpRows];
+  __shared__ unsigned long long s_key[kWarps][kWarpRows];
+  __shared__ int s_list[kWarps][2][kWarpRows];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int ui = blockIdx.x * kWarps + warp;
+  if (ui >= units) return;
+  const int b = ui;
+  const int hh = b % c.H, lr = (b / c.H) % nl, sq = b / (c.H * nl);
+  const size_t u = ((size_t)sq * c.L + lb + lr) * c.H + hh;
+  const int n = c.state[4 * u];
+  if (n <= B + W) return;
+  if (n > kWarpRows) {  // the host sized the launch from its mirror
+    if (lane == 0) atomicOr(c.err, ERR_LENGTH);
+    return;
+  }
+  T *Ku = reinterpret_cast<T *>(c.K) + u * (size_t)c.cap * D;
+  T *Vu = reinterpret_cast<T *>(c.V) + u * (size_t)c.cap * D;
+  float *su = c.score + u * (size_t)c.sstride;
+  int32_t *pu = c.pos + u * (size_t)c.sstride;
+  const int wlo = c.state[4 * u + 1] - 1 - W;
+  const int half = lane >> 4, l16 = lane & 15;
+  float *rs = s_r[warp];
+
+  // kE elements of row i with vector loads (8, 16 or 32 bytes).
+  auto load_row = [&](int i, float (&v)[kE]) {
+    const T *kr = Ku + (size_t)i * D + l16 * kE;
+    if constexpr (sizeof(T) == 2 && kE == 8) {
+      const uint4 w = __ldg(reinterpret_cast<const uint4 *>(kr));
+      const uint32_t x[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        v[2 * j] = __uint_as_float(x[j] << 16);
+        v[2 * j + 1] = __uint_as_float(x[j] & 0xffff0000u);
+      }
+    } else if constexpr (sizeof(T) == 2 && kE == 4) {
+      const uint2 w = __ldg(reinterpret_cast<const uint2 *>(kr));
+      v[0] = __uint_as_float(w.x << 16);
+      v[1] = __uint_as_float(w.x & 0xffff0000u);
+      v[2] = __uint_as_float(w.y << 16);
+      v[3] = __uint_as_float(w.y & 0xffff0000u);
+    } else {
+#pragma unroll
+      for (int j = 0; j < kE; j += 4) {
+        const float4 w = __ldg(reinterpret_cast<const float4 *>(kr + j));
+        v[j] = w.x, v[j + 1] = w.y, v[j + 2] = w.z, v[j + 3] = w.w;
+      }
+    }
+  };
+  auto half_sum = [](float x) {
+#pragma unroll
+    for (int o = 8; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+    return x;
+  };
+  // Rows go kU pairs a step, all their loads issued before any is used.
+  constexpr int kU = 4;
+  auto load_rows = [&](int i0, float (&v)[kU][kE]) {
+#pragma unroll
+    for (int q = 0; q < kU; ++q) {
+      const int i = i0 + 2 * q + half;
+      if (i < n) load_row(i, v[q]);
+      else {
+#pragma unroll
+        for (int j = 0; j < kE; ++j) v[q][j] = 0.f;
+      }
+    }
+  };
+  // Pass 1: S = sum of the normalised keys (this lane's kE dimensions).
+  float S[kE];
+#pragma unroll
+  for (int j = 0; j < kE; ++j) S[j] = 0.f;
+  for (int i0 = 0; i0 < n; i0 += 2 * kU) {
+    float v[kU][kE];
+    load_rows(i0, v);
+#pragma unroll
+    for (int q = 0; q < kU; ++q) {
+      float ss = 0.f;
+#pragma unroll
+      for (int j = 0; j < kE; ++j) ss = fmaf(v[q][j], v[q][j], ss);
+      ss = half_sum(ss);
+      const float inv = ss > 0.f ? 1.f / sqrtf(ss) : 0.f;
+#pragma unroll
+      for (int j = 0; j < kE; ++j) S[j] = fmaf(v[q][j], inv, S[j]);
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < kE; ++j) S[j] += __shfl_xor_sync(0xffffffffu, S[j], 16);
+  // Pass 2: each row's mean cosine with the other live rows.
+  const float inv_n1 = 1.f / (float)(n - 1);
+  for (int i0 = 0; i0 < n; i0 += 2 * kU) {
+    float v[kU][kE];
+    load_rows(i0, v);
+#pragma unroll
+    for (int q = 0; q < kU; ++q) {
+      const int i = i0 + 2 * q + half;
+      float ss = 0.f, dot = 0.f;
+#pragma unroll
+      for (int j = 0; j < kE; ++j) {
+        ss = fmaf(v[q][j], v[q][j], ss);
+        dot = fmaf(v[q][j], S[j], dot);
+      }
+      ss = half_sum(ss);
+      dot = half_sum(dot);
+      if (l16 == 0 && i < n) {
+        const float inv = ss > 0.f ? 1.f / sqrtf(ss) : 0.f;
+        rs[i] = (dot * inv - (ss > 0.f ? 1.f : 0.f)) * inv_n1;
+      }
+    }
+  }
+  __syncwarp();
+  // This lane's rows: positions, scores, candidacy; normalisers over C.
+  int ps[kR];
+  float sc[kR], r[kR];
+  bool cd[kR];
+  float mr = -INFINITY, ssum = 0.f;
+#pragma unroll
+  for (int k = 0; k < kR; ++k) {
+    const int i = lane + 32 * k;
+    const bool in = i < n;
+    ps[k] = in ? pu[i] : 0;
+    sc[k] = in ? su[i] : 0.f;
+    r[k] = in ? rs[i] : 0.f;
+    cd[k] = in && ps[k] <= wlo;
+    if (cd[k]) {
+      mr = fmaxf(mr, r[k]);
+      ssum += sc[k];
+    }
+  }
+  mr = dev::warp_max(mr);
+  ssum = dev::warp_sum(ssum);
+  float esum = 0.f;
+#pragma unroll
+  for (int k = 0; k < kR; ++k)
+    if (cd[k]) esum += expf(r[k] - mr);
+  esum = dev::warp_sum(esum);
+  const float inv_e = 1.f / esum, inv_s = ssum > 0.f ? 1.f / ssum : 0.f;
+  unsigned long long key[kR];
+#pragma unroll
+  for (int k = 0; k < kR; ++k) {
+    const float z = lam * (sc[k] * inv_s) - (1.f - lam) * (expf(r[k] - mr) * inv_e);
+    key[k] = cd[k] ? rkv_key(z, ps[k]) : 0ull;
+    if (lane + 32 * k < n) s_key[warp][lane + 32 * k] = key[k];
+  }
+  __syncwarp();
+  // Rank: a candidate stays iff fewer than B candidates have a larger key.
+  bool kp[kR];
+#pragma unroll
+  for (int k = 0; k < kR; ++k) {
+    const int i = lane + 32 * k;
+    bool keepi = i < n;
+    if (cd[k]) {
+      int above = 0;
+      for (int j = 0; j < n; ++j) above += s_key[warp][j] > key[k] ? 1 : 0;
+      keepi = above < B;
+    }
+    kp[k] = keepi;
+  }
+  int nk = 0;
+#pragma unroll
+  for (int k = 0; k < kR; ++k) nk += __popc(__ballot_sync(0xffffffffu, kp[k]));
+  if (nk != B + W) {
+    if (lane == 0) atomicOr(c.err, ERR_LENGTH);
+    return;
+  }
+  // Holes (dropped rows below nk) and movers (kept rows at nk or above), in
+  // row order; the j-th mover fills the j-th hole.
+  int nh = 0, nm = 0;
+#pragma unroll
+  for (int k = 0; k < kR; ++k) {
+    const int i = lane + 32 * k;
+    const bool hole = i < nk && !kp[k];
+    const bool mover = i >= nk && i < n && kp[k];
+    const unsigned bh = __ballot_sync(0xffffffffu, hole);
+    const unsigned bm = __ballot_sync(0xffffffffu, mover);
+    const unsigned below = (1u << lane) - 1u;
+    if (hole) s_list[warp][0][nh + __popc(bh & below)] = i;
+    if (mover) s_list[warp][1][nm + __popc(bm & below)] = i;
+    nh += __popc(bh);
+    nm += __popc(bm);
+  }
+  __syncwarp();
+  if (nh != nm) {
+    if (lane == 0) atomicOr(c.err, ERR_LENGTH);
+    return;
+  }
+  constexpr int kChunks = D * (int)sizeof(T) / 16;
+  for (int j = 0; j < nh; ++j) {
+    const int dst = s_list[warp][0][j], src = s_list[warp][1][j];
+    const int4 *ks = reinterpret_cast<const int4 *>(Ku + (size_t)src * D);
+    const int4 *vs = reinterpret_cast<const int4 *>(Vu + (size_t)src * D);
+    int4 *kd = reinterpret_cast<int4 *>(Ku + (size_t)dst * D);
+    int4 *vd = reinterpret_cast<int4 *>(Vu + (size_t)dst * D);
+    for (int q = lane; q < kChunks; q += 32) {
+      kd[q] = ks[q];
+      vd[q] = vs[q];
+    }
+    if (lane == 0) {
+      su[dst] = su[src];
+      pu[dst] = pu[src];
+    }
+  }
+  if (lane == 0) c.state[4 * u] = nk;
+}
+
 template <typename T, int D>
 cudaError_t rkv_dispatch(const CacheView &c, int lb, int nl, int max_rows,
                          int B, int W, float lam, cudaStream_t st) {
   const int nk = B + W;
   const int max_list = max(1, min(nk, max_rows - nk));
   const size_t list_bytes = 2 * (size_t)max_list * sizeof(int);
+  if (max_rows <= kWarpRows) {
+    const int units = c.S * nl * c.H;
+    return launch_pdl(rkv_evict_warp_kernel<T, D>,
+                      dim3((units + kWarps - 1) / kWarps), dim3(kThreads), 0,
+                      st, c, lb, nl, B, W, lam, units);
+  }
   const bool staged = stageable<T, D>() && max_rows <= kStageRows;
   const int srows = (max_rows + 3) & ~3;
   const size_t bytes =
