@@ -498,18 +498,25 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t aQ = smem_u32(smem + TcSmem::q);
   // Tile mt's q rows (row R = token j * G + head g), zeros past MQ, into the
   // Q buffer with cp.async (completed by the next commit-and-wait).
+  // Two threads a row, eight 16-byte pieces each.
+  static_assert(kThreads == 2 * kTcRows, "two threads a q row");
   auto load_q = [&](int mt) {
-    for (int i = tid; i < kTcRows * 16; i += kThreads) {
-      const int rr = i >> 4, ch = i & 15, R = mt * kTcRows + rr;
+    const int rr = tid >> 1, ch0 = (tid & 1) * 8, R = mt * kTcRows + rr;
+    const __nv_bfloat16 *src = nullptr;
+    if (R < MQ) {
+      const int j = R / G, g = R % G;
+      src = p.q + (((u.row0 + j) * c.H + h) * G + g) * 128;
+    }
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const int ch = ch0 + k;
       const uint32_t dst = aQ + (ch >> 3) * (kTcRows * 128) + rr * 128 +
                            (((ch & 7) ^ (rr & 7)) << 4);
-      if (R < MQ) {
-        const int j = R / G, g = R % G;
-        cp_async16(dst, p.q + (((u.row0 + j) * c.H + h) * G + g) * 128 + ch * 8);
-      } else {
+      if (src)
+        cp_async16(dst, src + ch * 8);
+      else
         asm volatile("st.shared.v4.b32 [%0], {%1, %1, %1, %1};" ::"r"(dst), "r"(0)
                      : "memory");
-      }
     }
   };
   load_q(0);
