@@ -85,3 +85,27 @@ def test_missing_library_fails_loudly(tmp_path, monkeypatch):
     mod = importlib.util.module_from_spec(spec)
     with pytest.raises(ImportError, match="libkvr.so not found"):
         spec.loader.exec_module(mod)
+
+
+def test_entropy_descriptor_and_buffer_checks_on_host():
+    """kvr_entropy_*: descriptors and buffers are validated on the host,
+    before any device call."""
+    good = kvr.kvr_entropy_desc(512, 152064, 12, 24, 7.0, 1.0, kvr.KVR_BF16)
+    need = kvr.kvr_entropy_required_bytes(good)
+    assert need >= 512 * 12 * 4  # the entropy ring at least
+    for bad in (kvr.kvr_entropy_desc(0, 100, 12, 24, 7.0, 1.0, 0),
+                kvr.kvr_entropy_desc(70000, 100, 12, 24, 7.0, 1.0, 0),
+                kvr.kvr_entropy_desc(4, 100, 65, 24, 7.0, 1.0, 0),
+                kvr.kvr_entropy_desc(4, 100, 12, 24, float("nan"), 1.0, 0),
+                kvr.kvr_entropy_desc(4, 100, 12, 24, 7.0, 1.0, 3)):
+        assert kvr.kvr_entropy_required_bytes(bad) == 0
+    h = ctypes.c_void_p()
+    st = kvr.lib.kvr_entropy_create(ctypes.byref(good), None, need, None,
+                                    ctypes.byref(h))
+    assert st == kvr.KVR_EINVAL and not h.value
+    st = kvr.lib.kvr_entropy_create(ctypes.byref(good), ctypes.c_void_p(0x1000 + 8),
+                                    need, None, ctypes.byref(h))
+    assert st == kvr.KVR_EINVAL and "aligned" in kvr.kvr_last_error()
+    st = kvr.lib.kvr_entropy_create(ctypes.byref(good), ctypes.c_void_p(0x1000),
+                                    need - 1, None, ctypes.byref(h))
+    assert st == kvr.KVR_ENOMEM
