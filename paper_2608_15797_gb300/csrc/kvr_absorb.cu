@@ -428,18 +428,23 @@ __global__ void __launch_bounds__(kThreads)
 //      probabilities, written as bf16 hi and lo terms into two P buffers
 //      (K-major, 128B swizzle: [64-key block][query row][128 B]).
 //   3. One thread issues O = P_hi V + P_lo V (V read MN-major) and the
-//      score column sums CS = 1 P_hi + 1 P_lo (the same P buffers read as an
-//      MN-major B operand, K = the tile's query rows) into TMEM.
-//   4. The warps write their rows' outputs from TMEM; warp 0 adds the column
-//      sums, times 1/G, to the unit's score increments.
+//      score column sums CS = P_hi^T 1 + P_lo^T 1 (the same P buffers read as
+//      an MN-major A operand, M = keys in 128-key tiles, K = the tile's query
+//      rows, N = 16 columns of ones) into TMEM.
+//      CS accumulates over the unit's tiles.
+//   4. The warps write their rows' outputs from TMEM.
+// After the last tile thread t adds the sum of key t (TMEM lane t % 128 of
+// key tile t / 128), times 1/G, to the unit's score increments.
 // Every mbarrier wait is bounded; TMEM is freed before the selection.
 constexpr int kTcRows = 128;                       // query rows per tile
 constexpr int kTcS = 0;                            // TMEM columns: S
 constexpr int kTcO = kMaxRows;                     //               O
 constexpr int kTcCS = kMaxRows + 128;              //               CS
+constexpr int kTcCsTiles = (kMaxRows + 127) / 128;  // 128-key tiles of CS
 constexpr int kTcCols = 512;
 constexpr int kTcChunks = (kMaxRows / 2 + 15) / 16;  // a thread's column chunks
-static_assert(kTcCS + kMaxRows <= kTcCols, "TMEM columns");
+static_assert(kTcCS + 16 * kTcCsTiles <= kTcCols, "TMEM columns");
+static_assert(kTcCsTiles * 128 <= 2 * kTcRows, "one key of CS a thread");
 
 struct TcSmem {  // offsets from a 1024-byte aligned base
   static constexpr int k = 0;                              // [2][kMaxRows][128 B]
@@ -447,17 +452,24 @@ struct TcSmem {  // offsets from a 1024-byte aligned base
   static constexpr int ph = v + 2 * kMaxRows * 128;        // [3][128][128 B]
   static constexpr int pl = ph + 3 * kTcRows * 128;
   static constexpr int q = pl;                             // [2][128][128 B], aliases P lo
-  static constexpr int ones = pl + 3 * kTcRows * 128;      // [128][128 B] of 1.0
-  static constexpr int sc = ones + kTcRows * 128;
+  static constexpr int ones = pl + 3 * kTcRows * 128;      // [16][128 B] of 1.0
+  static constexpr int sc = ones + 16 * 128;
   static constexpr int ps = sc + 4 * kMaxRows;
   static constexpr int acc = ps + 4 * kMaxRows;
   static constexpr int lists = acc + 4 * kMaxRows;
   static constexpr int key = lists + 8 * kMaxRows;
   static constexpr int kept = key + 8 * kMaxRows;
-  static constexpr int bytes = kept + 4 * kMaxRows;
+  static constexpr int end = kept + 4 * kMaxRows;
+  // The last CS key tile reads P blocks up to 2 kTcCsTiles - 1: past the
+  // three P hi blocks lies P lo, past P lo the ones and the lists (rows of
+  // keys >= NS, never read back), so the buffer reaches that far.
+  static constexpr int cs_end = pl + 2 * kTcCsTiles * kTcRows * 128;
+  static constexpr int bytes = end > cs_end ? end : cs_end;
   static constexpr int alloc = bytes + 1024;               // room to align
 };
+static_assert(TcSmem::alloc <= 227 * 1024, "shared memory per CTA");
 static_assert(3 * 64 >= kMaxRows, "P holds kMaxRows keys in 64-key blocks");
+static_assert(TcSmem::cs_end <= TcSmem::bytes, "CS key tiles stay in the buffer");
 
 template <bool kOutBf16>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -491,7 +503,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     s_abort = 0;
     fence_mbar_init();
   }
-  for (int i = tid; i < kTcRows * 128 / 4; i += kThreads)  // bf16 1.0 pairs
+  for (int i = tid; i < 16 * 128 / 4; i += kThreads)  // bf16 1.0 pairs
     reinterpret_cast<uint32_t *>(smem + TcSmem::ones)[i] = 0x3F803F80u;
   const int n = u.n, n0 = u.n0, h = u.h;
   const int MQ = C * G, n_mt = (MQ + kTcRows - 1) / kTcRows;
@@ -527,7 +539,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int NS = (n + 15) & ~15;
   const uint32_t id_s = idesc_bf16(kTcRows, NS, false);
   const uint32_t id_o = idesc_bf16(kTcRows, 128, true);
-  const uint32_t id_c = idesc_bf16(kTcRows, NS, true);
+  const uint32_t id_c = idesc_bf16(128, 16, false, true);
+  const int n_ct = (NS + 127) >> 7;  // 128-key tiles of CS
   const uint32_t aK = smem_u32(m.k), aV = smem_u32(m.v);
   const uint32_t aPH = smem_u32(smem + TcSmem::ph), aPL = smem_u32(smem + TcSmem::pl);
   const uint32_t aOnes = smem_u32(smem + TcSmem::ones);
@@ -656,7 +669,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc_fence_after();
 
-    // 3. O = P V and the column sums CS = 1 P, hi and lo terms each.
+    // 3. O = P V and the column sums CS = P^T 1, hi and lo terms each.
     if (tid == 0) {
       for (int k = 0; k < NS / 16; ++k) {  // K = keys, 16 a step
         const uint32_t pa = (k >> 2) * (kTcRows * 128) + (k & 3) * 32;
@@ -664,12 +677,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_mma(tm + kTcO, sdesc_sw128(aPH + pa, 16, 1024), bv, id_o, k > 0);
         tc_mma(tm + kTcO, sdesc_sw128(aPL + pa, 16, 1024), bv, id_o, true);
       }
-      for (int k = 0; k < kTcRows / 16; ++k) {  // K = the tile's query rows
-        const uint64_t ao = sdesc_sw128(aOnes + (k & 3) * 32, 16, 1024);
-        tc_mma(tm + kTcCS, ao, sdesc_sw128(aPH + k * 2048, kTcRows * 128, 1024),
-               id_c, k > 0);
-        tc_mma(tm + kTcCS, ao, sdesc_sw128(aPL + k * 2048, kTcRows * 128, 1024),
-               id_c, true);
+      for (int t = 0; t < n_ct; ++t) {  // M = 128 keys (two 64-key P blocks)
+        const uint32_t pb = t * 2 * (kTcRows * 128);
+        for (int k = 0; k < kTcRows / 16; ++k) {  // K = the tile's query rows
+          const uint64_t bo = sdesc_sw128(aOnes + (k & 3) * 32, 16, 1024);
+          tc_mma(tm + kTcCS + 16 * t,
+                 sdesc_sw128(aPH + pb + k * 2048, kTcRows * 128, 1024), bo, id_c,
+                 mt > 0 || k > 0);
+          tc_mma(tm + kTcCS + 16 * t,
+                 sdesc_sw128(aPL + pb + k * 2048, kTcRows * 128, 1024), bo, id_c,
+                 true);
+        }
       }
       tc_commit(smem_u32(&bar_o));
     }
@@ -710,22 +728,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
-    // Every TMEM lane holds the same sums: warp w reads 16-column chunk w,
-    // w + 8, ... from its own lane quarter, and lane j adds column c0 + j.
-    {
-      for (int c0 = 16 * warp; c0 < NS; c0 += 16 * kWarps) {
-        uint32_t v[16];
-        tmem_ld16(trow + kTcCS + c0, v);
-        float mine = 0.f;
-#pragma unroll
-        for (int j = 0; j < 16; ++j)
-          if (lane == j) mine = __uint_as_float(v[j]);
-        if (lane < 16 && c0 + lane < n) m.acc[c0 + lane] += mine * inv_g;
-      }
-    }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
+  }
+  // Key tid's sum over the unit's query rows: TMEM lane tid % 128 of CS
+  // tile tid / 128 (all 16 columns of a lane hold the same sum).
+  if (ok && n_mt > 0 && (!upper || n_ct > 1)) {
+    uint32_t v[16];
+    tmem_ld16(trow + kTcCS + (upper ? 16 : 0), v);
+    if (tid < n) m.acc[tid] += __uint_as_float(v[0]) * inv_g;
   }
   // After a timeout, wait (bounded) once more for tensor work in flight.
   if (!ok) {

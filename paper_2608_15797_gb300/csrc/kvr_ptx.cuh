@@ -167,11 +167,13 @@ __device__ __forceinline__ uint64_t sdesc_sw128(uint32_t addr, uint32_t lbo,
   d |= (uint64_t)2 << 61;  // 128-byte swizzle
   return d;
 }
-// Instruction descriptor of kind::f16 with bf16 A and B, fp32 D; A K-major,
-// B K-major or MN-major.
-__device__ __forceinline__ uint32_t idesc_bf16(int M, int N, bool b_mn_major) {
-  return (1u << 4) | (1u << 7) | (1u << 10) | (b_mn_major ? 1u << 16 : 0u) |
-         ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+// Instruction descriptor of kind::f16 with bf16 A and B, fp32 D; A and B
+// each K-major or MN-major.
+__device__ __forceinline__ uint32_t idesc_bf16(int M, int N, bool b_mn_major,
+                                               bool a_mn_major = false) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | (a_mn_major ? 1u << 15 : 0u) |
+         (b_mn_major ? 1u << 16 : 0u) | ((uint32_t)(N >> 3) << 17) |
+         ((uint32_t)(M >> 4) << 24);
 }
 // One warp: allocate `cols` TMEM columns (a power of two >= 32); the base
 // address lands in shared memory at dst.
