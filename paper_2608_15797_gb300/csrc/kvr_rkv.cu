@@ -265,9 +265,12 @@ __global__ void __launch_bounds__(kThreads)
 // The same arithmetic with no CTA-wide synchronisation: eight units a CTA,
 // one a warp.  In the key passes each half-warp takes one row (16 lanes x
 // D/16 elements, 16-byte loads for bf16 d = 128), so a warp reads two rows a
-// step and keeps D/16 elements of the normalised-key sum per lane.  For the
-// ranking every lane owns rows lane, lane + 32, ...; the warp's candidates
-// rank by counting larger keys, and ballots build the hole and mover lists.
+// step and keeps D/16 elements of the normalised-key sum per lane; pass 1
+// leaves each row's inverse norm in the row's scratch slot for pass 2.  For
+// the selection every lane owns rows lane, lane + 32, ...; the e = (number
+// of candidates) - B smallest keys are dropped by e warp-wide minimum
+// searches (keys are unique: they end in the position), which is one search
+// in the steady state, and ballots build the hole and mover lists.
 constexpr int kWarpRows = 128;
 
 template <typename T, int D>
@@ -278,7 +281,6 @@ __global__ void __launch_bounds__(kThreads)
   constexpr int kE = D / 16;  // elements of a row per half-warp lane
   constexpr int kR = kWarpRows / 32;
   __shared__ float s_r[kWarps][kWarpRows];
-  __shared__ unsigned long long s_key[kWarps][kWarpRows];
   __shared__ int s_list[kWarps][2][kWarpRows];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int ui = blockIdx.x * kWarps + warp;
@@ -343,7 +345,8 @@ __global__ void __launch_bounds__(kThreads)
       }
     }
   };
-  // Pass 1: S = sum of the normalised keys (this lane's kE dimensions).
+  // Pass 1: S = sum of the normalised keys (this lane's kE dimensions);
+  // rs[i] = 1 / |k_i| (0 for a zero key).
   float S[kE];
 #pragma unroll
   for (int j = 0; j < kE; ++j) S[j] = 0.f;
@@ -359,11 +362,14 @@ __global__ void __launch_bounds__(kThreads)
       const float inv = ss > 0.f ? 1.f / sqrtf(ss) : 0.f;
 #pragma unroll
       for (int j = 0; j < kE; ++j) S[j] = fmaf(v[q][j], inv, S[j]);
+      const int i = i0 + 2 * q + half;
+      if (l16 == 0 && i < n) rs[i] = inv;
     }
   }
 #pragma unroll
   for (int j = 0; j < kE; ++j) S[j] += __shfl_xor_sync(0xffffffffu, S[j], 16);
-  // Pass 2: each row's mean cosine with the other live rows.
+  // Pass 2: each row's mean cosine with the other live rows (the lane that
+  // wrote rs[i] in pass 1 reads and replaces it).
   const float inv_n1 = 1.f / (float)(n - 1);
   for (int i0 = 0; i0 < n; i0 += 2 * kU) {
     float v[kU][kE];
@@ -371,17 +377,13 @@ __global__ void __launch_bounds__(kThreads)
 #pragma unroll
     for (int q = 0; q < kU; ++q) {
       const int i = i0 + 2 * q + half;
-      float ss = 0.f, dot = 0.f;
+      float dot = 0.f;
 #pragma unroll
-      for (int j = 0; j < kE; ++j) {
-        ss = fmaf(v[q][j], v[q][j], ss);
-        dot = fmaf(v[q][j], S[j], dot);
-      }
-      ss = half_sum(ss);
+      for (int j = 0; j < kE; ++j) dot = fmaf(v[q][j], S[j], dot);
       dot = half_sum(dot);
       if (l16 == 0 && i < n) {
-        const float inv = ss > 0.f ? 1.f / sqrtf(ss) : 0.f;
-        rs[i] = (dot * inv - (ss > 0.f ? 1.f : 0.f)) * inv_n1;
+        const float inv = rs[i];
+        rs[i] = (dot * inv - (inv > 0.f ? 1.f : 0.f)) * inv_n1;
       }
     }
   }
@@ -413,25 +415,34 @@ __global__ void __launch_bounds__(kThreads)
   esum = dev::warp_sum(esum);
   const float inv_e = 1.f / esum, inv_s = ssum > 0.f ? 1.f / ssum : 0.f;
   unsigned long long key[kR];
+  int ncand = 0;
 #pragma unroll
   for (int k = 0; k < kR; ++k) {
     const float z = lam * (sc[k] * inv_s) - (1.f - lam) * (expf(r[k] - mr) * inv_e);
-    key[k] = cd[k] ? rkv_key(z, ps[k]) : 0ull;
-    if (lane + 32 * k < n) s_key[warp][lane + 32 * k] = key[k];
+    key[k] = rkv_key(z, ps[k]);
+    ncand += __popc(__ballot_sync(0xffffffffu, cd[k]));
   }
-  __syncwarp();
-  // Rank: a candidate stays iff fewer than B candidates have a larger key.
-  bool kp[kR];
+  // Drop the ncand - B smallest candidate keys, one warp-wide minimum at a
+  // time; the rest of the candidates are the B largest.
+  bool kp[kR], live[kR];
 #pragma unroll
   for (int k = 0; k < kR; ++k) {
-    const int i = lane + 32 * k;
-    bool keepi = i < n;
-    if (cd[k]) {
-      int above = 0;
-      for (int j = 0; j < n; ++j) above += s_key[warp][j] > key[k] ? 1 : 0;
-      keepi = above < B;
+    kp[k] = lane + 32 * k < n;
+    live[k] = cd[k];
+  }
+  for (int d = 0; d < ncand - B; ++d) {
+    unsigned long long m = ~0ull;
+#pragma unroll
+    for (int k = 0; k < kR; ++k)
+      if (live[k] && key[k] < m) m = key[k];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const unsigned long long x = __shfl_xor_sync(0xffffffffu, m, o);
+      m = x < m ? x : m;
     }
-    kp[k] = keepi;
+#pragma unroll
+    for (int k = 0; k < kR; ++k)
+      if (live[k] && key[k] == m) live[k] = kp[k] = false;
   }
   int nk = 0;
 #pragma unroll
