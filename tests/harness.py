@@ -23,29 +23,47 @@ def dev(x: np.ndarray, dtype: str) -> torch.Tensor:
 
 def make_pair(w: inputs.Workload, seed: int, S: int, cap: int,
               prompt_lens=None, out_dtype="f32", first_pos=None, fused=True,
-              chunk=(0, 0)):
+              chunk=(0, 0), sample=None):
     """A CUDA cache and an oracle cache loaded with the same prompts.
     fused=False restricts the CUDA cache to the generic kernels; chunk is
-    the chunked kernel's (groups, stages) tuning, groups -1 turning it off."""
+    the chunked kernel's (groups, stages) tuning, groups -1 turning it off.
+    With `sample` (a list of sequence indices) the oracle holds only those
+    sequences, in that order; the others get device-drawn prompts of the
+    same lengths, which no check reads (sequences are independent)."""
     c = kvr.Cache(S, w.n_layers, w.n_kv_heads, w.group, w.head_dim, cap,
                   kv_dtype=w.dtype, out_dtype=out_dtype)
     c.set_fused(fused)
     c.set_chunk_tuning(*chunk)
-    o = orc.OracleCache(S, w.n_layers, w.n_kv_heads, w.group, w.head_dim, cap)
+    samp = list(range(S)) if sample is None else list(sample)
+    o = orc.OracleCache(len(samp), w.n_layers, w.n_kv_heads, w.group,
+                        w.head_dim, cap)
     lens = [w.prompt] * S if prompt_lens is None else list(prompt_lens)
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(seed + 1_000_003)
     for s in range(S):
-        k, v = inputs.prompt(w, seed, s, int(lens[s]))
+        n = int(lens[s])
         fp = 0 if first_pos is None else int(first_pos[s])
-        c.load(s, dev(k, w.dtype), dev(v, w.dtype), first_pos=fp)
-        o.load(s, k, v, first_pos=fp)
+        if s in samp:
+            k, v = inputs.prompt(w, seed, s, n)
+            c.load(s, dev(k, w.dtype), dev(v, w.dtype), first_pos=fp)
+            o.load(samp.index(s), k, v, first_pos=fp)
+        else:
+            shape = (w.n_layers, w.n_kv_heads, n, w.head_dim)
+            k, v = (torch.randn(shape, generator=gen, device="cuda")
+                    .mul_(w.sigma).to(kvr.TORCH_DTYPES[w.dtype])
+                    for _ in range(2))
+            c.load(s, k, v, first_pos=fp)
     return c, o
 
 
 def lockstep(c: kvr.Cache, o: orc.OracleCache, w: inputs.Workload, seed: int,
              steps: int, budget: int, window: int, fused: bool = True,
-             step0: int = 0, layers=None, evict: bool = True) -> parity.Stats:
-    """Run `steps` decode steps on both sides, checking after every step."""
+             step0: int = 0, layers=None, evict: bool = True,
+             sample=None) -> parity.Stats:
+    """Run `steps` decode steps on both sides, checking after every step
+    (the sequences `sample` only, when the oracle holds just those)."""
     S = c.S
+    samp = list(range(S)) if sample is None else list(sample)
     stats = parity.Stats()
     lb, le = (0, c.L) if layers is None else layers
     for t in range(step0, step0 + steps):
@@ -58,11 +76,12 @@ def lockstep(c: kvr.Cache, o: orc.OracleCache, w: inputs.Workload, seed: int,
         else:
             out = c.attend_score(qd, kd, vd, layers=(lb, le))
             c.evict(budget, window, layers=(lb, le))
-        ref = o.step(q, kn, vn, evict=False, layer_begin=lb, layer_end=le)
+        ref = o.step(q[samp], kn[samp], vn[samp], evict=False, layer_begin=lb,
+                     layer_end=le)
         torch.cuda.synchronize()
         stats.max_out_excess = max(stats.max_out_excess, parity.check_out(
-            out.float().cpu().numpy(), ref, what=f"out at step {t}"))
-        exports = [c.export(s, kv=False) for s in range(S)]
+            out[samp].float().cpu().numpy(), ref, what=f"out at step {t}"))
+        exports = [c.export(s, kv=False) for s in samp]
         st = parity.check_and_adopt(o, exports, budget, window, evict=evict,
                                     layers=(lb, le))
         stats.merge(st)

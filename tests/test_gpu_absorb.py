@@ -20,20 +20,23 @@ def _cuda():
     torch.cuda.set_device(0)
 
 
-def absorb_lockstep(c, o, w, seed, chunk, B, W, evict=True, step0=20_000):
+def absorb_lockstep(c, o, w, seed, chunk, B, W, evict=True, step0=20_000,
+                    sample=None):
     """One absorb call on both sides, checking every token's output, then the
-    retained rows and scores of every unit."""
+    retained rows and scores of every unit (of the sequences `sample` only,
+    when the oracle holds just those)."""
     S = c.S
+    samp = list(range(S)) if sample is None else list(sample)
     toks = [inputs.step_inputs(w, seed, step0 + j, S) for j in range(chunk)]
     q, kn, vn = (np.stack([t[i] for t in toks], axis=2) for i in range(3))
     out = c.absorb(harness.dev(q, w.dtype), harness.dev(kn, w.dtype),
                    harness.dev(vn, w.dtype), B, W, evict=evict)
-    ref = o.absorb(q, kn, vn, B=B, W=W, evict=False)
+    ref = o.absorb(q[samp], kn[samp], vn[samp], B=B, W=W, evict=False)
     torch.cuda.synchronize()
-    got = out.float().cpu().numpy()
+    got = out[samp].float().cpu().numpy()
     for j in range(chunk):
         parity.check_out(got[:, :, j], ref[:, :, j], what=f"token {j} of the chunk")
-    exports = [c.export(s, kv=False) for s in range(S)]
+    exports = [c.export(s, kv=False) for s in samp]
     st = parity.check_and_adopt(o, exports, B, W, evict=evict)
     c.sync_status()
     return st

@@ -1,0 +1,87 @@
+"""Parity at the benchmarked sizes, in the launch configuration bench.py
+times, on sampled sequences.
+
+Sequences are independent, so an oracle that holds a few of them (the
+first, one in the middle and the last, which land on CTAs at both ends of
+the persistent grids' unit order) checks those units of the full-size
+launch exactly as a full oracle would; the other sequences run alongside
+with device-drawn inputs that no check reads.
+
+- decode step (Eq. 1 + TopB eviction, Sec. 2.1): 7B geometry, 64 sequences x
+  28 layers x 4 KV heads = 7,168 units a launch, B = 64, W = 8, bf16 in and
+  out.  The first step evicts every unit from its prior context (80-600
+  rows here: the bench's longer prior contexts change only that untimed
+  first step); the steady-state steps run the fused kernel on 73-row units.
+- R-KV step (App. C, lambda = 0.1): the same 64 x 28 x 4 units at B + W = 72
+  rows, attend+score then the R-KV eviction, as bench.py --mode rkv.
+- chunk absorb (Algorithm 1's single forward pass over an accepted step): 64
+  sequences x 28 layers at B + W = 72 rows taking 64-token chunks, as
+  bench.py --mode absorb.
+- candidate step (Sec. 2.2 Eq. 2): 72B geometry, the bench's 4 sequences x
+  80 layers x 8 KV heads with 8 candidates and a 64-row tail capacity, every
+  sequence checked (the bench's full size), a few candidate tokens, then
+  the commit.
+"""
+import numpy as np
+import pytest
+import torch
+
+from paper_2608_15797_gb300 import inputs
+from tests import harness
+from tests.test_gpu_absorb import absorb_lockstep
+from tests.test_gpu_rkv import rkv_lockstep
+
+pytestmark = pytest.mark.gpu
+
+SAMPLE = [0, 37, 63]
+
+
+@pytest.fixture(autouse=True)
+def _cuda():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA device")
+    torch.cuda.set_device(0)
+
+
+def test_decode_step_7b_s64_b64_sampled():
+    w = inputs.WORKLOADS["7b_s64_b64"]
+    S = w.n_seq
+    lens = inputs.prior_lengths(61, S, 80, 600)
+    c, o = harness.make_pair(w, 61, S, cap=int(lens.max()) + 1,
+                             prompt_lens=lens, out_dtype="bf16", sample=SAMPLE)
+    st = harness.lockstep(c, o, w, 61, 7, w.budget, w.window, sample=SAMPLE)
+    assert st.units == 7 * len(SAMPLE) * w.n_layers * w.n_kv_heads
+    assert (c.lengths() == w.budget + w.window).all()
+
+
+def test_rkv_step_7b_s64_b64_sampled():
+    w = inputs.WORKLOADS["7b_b64"]
+    S, m = 64, w.budget + w.window
+    c, o = harness.make_pair(w, 62, S, cap=m + 1, prompt_lens=[m] * S,
+                             out_dtype="bf16", sample=SAMPLE)
+    st = rkv_lockstep(c, o, w, 62, 6, w.budget, w.window, 0.1, sample=SAMPLE)
+    assert st.units == 6 * len(SAMPLE) * w.n_layers * w.n_kv_heads
+    assert (c.lengths() == m).all()
+
+
+def test_absorb_7b_s64_c64_sampled():
+    w = inputs.WORKLOADS["7b_b64"]
+    S, m, C = 64, w.budget + w.window, 64
+    c, o = harness.make_pair(w, 63, S, cap=m + C, prompt_lens=[m] * S,
+                             out_dtype="bf16", sample=SAMPLE)
+    for k in range(2):
+        absorb_lockstep(c, o, w, 63, C, w.budget, w.window,
+                        step0=20_000 + 100 * k, sample=SAMPLE)
+    assert (c.lengths() == m).all()
+
+
+def test_candidate_step_72b_bon8_full():
+    w = inputs.WORKLOADS["72b_bon8"]
+    S, m = 4, w.budget + w.window
+    c, o = harness.make_pair(w, 64, S, cap=m + w.cand_step + 1,
+                             prompt_lens=[m] * S, out_dtype="bf16")
+    o = o.resized(m + w.cand_step)
+    o2, chosen, st = harness.fork_lockstep(c, o, w, 64, w.n_cand, 4, w.budget,
+                                           w.window, tail_cap=w.cand_step)
+    assert st.steps == 5  # the tokens, then the commit
+    assert (c.lengths() == m).all()
