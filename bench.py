@@ -387,59 +387,48 @@ def run_kvr(args, rank, world, local_rank):
 
     total_ms = max_over_ranks(total_ms, dev)
 
-    # End to end through the public call: every step's inputs copied in from
-    # pinned host memory and its output copied back, inside the timed region.
+    # End to end through the public call with HOST buffers
+    # (kvr_decode_step_host): every step's inputs copied in from pinned host
+    # memory and its output copied back by the library, inside the timed
+    # region.
     hpool = [tuple(x.cpu().pin_memory() for x in p) for p in pool[:4]]
-    hout = [torch.empty(out.shape, dtype=out.dtype).pin_memory() for _ in range(2)]
+    n_str = 3
+    hout = [torch.empty(out.shape, dtype=out.dtype).pin_memory()
+            for _ in range(n_str)]
     bi = sum(x.numel() * x.element_size() for x in hpool[0])
     bo = hout[0].numel() * hout[0].element_size()
     Ke = max(1, min(K, args.e2e_steps))
+    stage = [tuple(torch.empty_like(x) for x in pool[0]) + (torch.empty_like(out),)
+             for _ in range(n_str)]
 
     # Serial: copy in, decode, copy out, one stream.
-    dq, dk, dv = (torch.empty_like(x) for x in pool[0])
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     torch.cuda.synchronize()
     e0.record(stream)
     for i in range(Ke):
-        hq, hk, hv = hpool[i % len(hpool)]
-        dq.copy_(hq, non_blocking=True)
-        dk.copy_(hk, non_blocking=True)
-        dv.copy_(hv, non_blocking=True)
-        kvr.kvr_decode_step(cache.handle, 0, L, dq, dk, dv, out, B, W, stream)
-        hout[0].copy_(out, non_blocking=True)
+        kvr.kvr_decode_step_host(cache.handle, 0, L, *hpool[i % len(hpool)],
+                                 hout[0], *stage[0], B, W, stream)
     e1.record(stream)
     torch.cuda.synchronize()
     e2e_serial_ms = max_over_ranks(e0.elapsed_time(e1), dev)
 
-    # Pipelined (a serving loop): copies on their own streams with two
-    # device buffers each way, so step i + 1's inputs land and step i - 1's
-    # output returns while step i decodes.
-    din = [tuple(torch.empty_like(x) for x in pool[0]) for _ in range(2)]
-    dout = [torch.empty_like(out) for _ in range(2)]
-    h2d, d2h = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
-    ev_in = [torch.cuda.Event() for _ in range(Ke)]
-    ev_done = [torch.cuda.Event() for _ in range(Ke)]
-    ev_out = [torch.cuda.Event() for _ in range(Ke)]
+    # Pipelined (a serving loop): step i on stream i % 3 with staging set
+    # i % 3; the library orders the steps, so step i + 1's copy in and step
+    # i - 1's copy out overlap step i's compute.
+    strs = [torch.cuda.Stream(dev) for _ in range(n_str)]
     torch.cuda.synchronize()
-    e0.record(h2d)
+    e0.record(strs[0])
+    for x in strs[1:]:
+        x.wait_event(e0)
     for i in range(Ke):
-        b = i % 2
-        if i >= 2:
-            h2d.wait_event(ev_done[i - 2])   # din[b] consumed
-        with torch.cuda.stream(h2d):
-            for dst, src in zip(din[b], hpool[i % len(hpool)]):
-                dst.copy_(src, non_blocking=True)
-        ev_in[i].record(h2d)
-        stream.wait_event(ev_in[i])
-        if i >= 2:
-            stream.wait_event(ev_out[i - 2])  # dout[b] copied out
-        kvr.kvr_decode_step(cache.handle, 0, L, *din[b], dout[b], B, W, stream)
-        ev_done[i].record(stream)
-        d2h.wait_event(ev_done[i])
-        with torch.cuda.stream(d2h):
-            hout[b].copy_(dout[b], non_blocking=True)
-        ev_out[i].record(d2h)
-    e1.record(d2h)
+        j = i % n_str
+        kvr.kvr_decode_step_host(cache.handle, 0, L, *hpool[i % len(hpool)],
+                                 hout[j], *stage[j], B, W, strs[j])
+    for x in strs[1:]:
+        ev = torch.cuda.Event()
+        ev.record(x)
+        strs[0].wait_event(ev)
+    e1.record(strs[0])
     torch.cuda.synchronize()
     e2e_ms = max_over_ranks(e0.elapsed_time(e1), dev)
     cache.sync_status()
@@ -1274,12 +1263,16 @@ def main():
         "e2e": {"value": job_rate(world, r["Ke"], r["e2e_ms"]),
                 "unit": "steps/s", "h2d_bytes_per_step": r["bi"],
                 "d2h_bytes_per_step": r["bo"],
+                "call": "kvr_decode_step_host (host q/k/v in, host output "
+                        "out; the library copies)",
                 "copies": "every step's q/k/v in and output out inside the "
-                          "timed region, on their own streams with two "
-                          "device buffers each way (overlapping the decode)"},
+                          "timed region; steps rotate over 3 streams with "
+                          "their own staging buffers, so copies overlap the "
+                          "neighbouring steps' decode"},
         "e2e_serial": {"value": job_rate(world, r["Ke"], r["e2e_serial_ms"]),
                        "unit": "steps/s",
-                       "note": "copy in, decode, copy out on one stream"},
+                       "note": "kvr_decode_step_host on one stream: copy in, "
+                               "decode, copy out"},
         "gpu_launches": r["launches"],
         "per_layer_launches": {
             "launches_per_step": w.n_layers,

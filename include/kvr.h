@@ -145,6 +145,28 @@ kvr_status kvr_decode_step(kvr_cache *cache, int layer_begin, int layer_end,
                            const void *q, const void *k_new, const void *v_new,
                            void *out, int budget, int window, void *stream);
 
+/* kvr_decode_step with the step's inputs and output in HOST memory, as a
+ * serving loop feeds it (Sec. 2.1 Eq. 1, one decode step of every sequence).
+ * Enqueued on stream, in order: the copies of q_host, k_new_host and
+ * v_new_host (shapes and element types of kvr_decode_step's q, k_new,
+ * v_new) into the caller's device staging buffers q_dev, k_new_dev,
+ * v_new_dev; the step, which writes out_dev (kvr_decode_step's out); the
+ * copy of out_dev into out_host.  The step waits for the handle's previous
+ * kvr_decode_step_host step, on whatever stream that ran, so a caller may
+ * alternate two streams, each with its own staging buffers, and have one
+ * step's copies overlap the other's compute.  A staging set may be reused on
+ * the stream that last used it (stream order covers it).  Host buffers are
+ * caller-owned, must stay valid until the stream passes the copy out, and
+ * should be page-locked (cudaHostAlloc / cudaHostRegister) for the copies
+ * to be asynchronous.  Errors: as kvr_decode_step, KVR_EINVAL for a null
+ * host or staging pointer, KVR_ECUDA when a copy or event call fails. */
+kvr_status kvr_decode_step_host(kvr_cache *cache, int layer_begin,
+                                int layer_end, const void *q_host,
+                                const void *k_new_host, const void *v_new_host,
+                                void *out_host, void *q_dev, void *k_new_dev,
+                                void *v_new_dev, void *out_dev, int budget,
+                                int window, void *stream);
+
 /* ---- full-context decode (the helper's cache: no scores, no eviction) -- */
 
 /* The full-context helper of KV-Rescue keeps its whole cache (Sec. 3.1;

@@ -106,6 +106,8 @@ struct kvr_cache {
   int sm_count = 0;               // of the device, queried on first use
   int smem_optin = 0;
   std::map<int, std::pair<CUtensorMap, CUtensorMap>> tmaps;  // by box rows
+  cudaEvent_t host_step_done = nullptr;  // last kvr_decode_step_host step
+  bool host_step_recorded = false;
 };
 
 namespace {
@@ -564,7 +566,10 @@ kvr_status kvr_cache_create(const kvr_cache_desc *desc, void *dev_buf,
   return KVR_OK;
 }
 
-void kvr_cache_destroy(kvr_cache *cache) { delete cache; }
+void kvr_cache_destroy(kvr_cache *cache) {
+  if (cache && cache->host_step_done) cudaEventDestroy(cache->host_step_done);
+  delete cache;
+}
 
 kvr_status kvr_cache_load(kvr_cache *c, int seq, const void *k, const void *v,
                           int n_rows, int first_pos, void *stream) {
@@ -860,6 +865,46 @@ kvr_status kvr_decode_step(kvr_cache *c, int lb, int le, const void *q,
   st = kvr_decode_attend_score(c, lb, le, q, k_new, v_new, out, stream);
   if (st != KVR_OK) return st;
   return kvr_evict_compact(c, lb, le, budget, window, stream);
+}
+
+kvr_status kvr_decode_step_host(kvr_cache *c, int lb, int le,
+                                const void *q_host, const void *k_new_host,
+                                const void *v_new_host, void *out_host,
+                                void *q_dev, void *k_new_dev, void *v_new_dev,
+                                void *out_dev, int budget, int window,
+                                void *stream) {
+  if (!q_host || !k_new_host || !v_new_host || !out_host)
+    return fail(KVR_EINVAL, "null host q, k_new, v_new or out");
+  kvr_status st = check_step(c, lb, le, q_dev, k_new_dev, v_new_dev, out_dev);
+  if (st != KVR_OK) return st;
+  st = check_evict(budget, window);
+  if (st != KVR_OK) return st;
+  const kvr_cache_desc &d = c->desc;
+  const size_t rows = (size_t)d.n_seq * (le - lb) * d.n_kv_heads;
+  const size_t row_kv = (size_t)d.head_dim * esize(d.kv_dtype);
+  const size_t qb = rows * d.group * row_kv, kb = rows * row_kv;
+  const size_t ob = rows * d.group * d.head_dim * esize(d.out_dtype);
+  cudaStream_t s = as_stream(stream);
+  cudaError_t e = cudaMemcpyAsync(q_dev, q_host, qb, cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(k_new_dev, k_new_host, kb, cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(v_new_dev, v_new_host, kb, cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess && !c->host_step_done)
+    e = cudaEventCreateWithFlags(&c->host_step_done, cudaEventDisableTiming);
+  if (e == cudaSuccess && c->host_step_recorded)
+    e = cudaStreamWaitEvent(s, c->host_step_done, 0);
+  if (e != cudaSuccess) return cuda_fail("kvr_decode_step_host: copy in", e);
+  st = kvr_decode_step(c, lb, le, q_dev, k_new_dev, v_new_dev, out_dev, budget,
+                       window, stream);
+  if (st != KVR_OK) return st;
+  e = cudaEventRecord(c->host_step_done, s);
+  if (e == cudaSuccess) {
+    c->host_step_recorded = true;
+    e = cudaMemcpyAsync(out_host, out_dev, ob, cudaMemcpyDeviceToHost, s);
+  }
+  if (e != cudaSuccess) return cuda_fail("kvr_decode_step_host: copy out", e);
+  return KVR_OK;
 }
 
 kvr_status kvr_cache_export(const kvr_cache *c, int seq, void *host_k,

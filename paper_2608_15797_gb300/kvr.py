@@ -62,6 +62,8 @@ _SIGS = {
     "kvr_decode_attend_score_noalloc": (_S, [_P, _I, _I, _P, _P, _P, _P, _P]),
     "kvr_evict_compact": (_S, [_P, _I, _I, _I, _I, _P]),
     "kvr_decode_step": (_S, [_P, _I, _I, _P, _P, _P, _P, _I, _I, _P]),
+    "kvr_decode_step_host": (_S, [_P, _I, _I, _P, _P, _P, _P, _P, _P, _P, _P,
+                                  _I, _I, _P]),
     "kvr_absorb_chunk": (_S, [_P, _I, _I, _I, _P, _P, _P, _P, _I, _I, _I, _P]),
     "kvr_cache_copy_sequences": (_S, [_P, _P, _P, _P, _I, _P]),
     "kvr_evict_compact_rkv": (_S, [_P, _I, _I, _I, _I, ctypes.c_float, _P]),
@@ -169,6 +171,16 @@ def kvr_decode_step(h, layer_begin, layer_end, q, k_new, v_new, out, budget,
     _check(lib.kvr_decode_step(h, layer_begin, layer_end, _ptr(q), _ptr(k_new),
                                _ptr(v_new), _ptr(out), budget, window,
                                _stream(stream)), "kvr_decode_step")
+
+
+def kvr_decode_step_host(h, layer_begin, layer_end, q_host, k_new_host,
+                         v_new_host, out_host, q_dev, k_new_dev, v_new_dev,
+                         out_dev, budget, window, stream=None):
+    _check(lib.kvr_decode_step_host(
+        h, layer_begin, layer_end, _ptr(q_host), _ptr(k_new_host),
+        _ptr(v_new_host), _ptr(out_host), _ptr(q_dev), _ptr(k_new_dev),
+        _ptr(v_new_dev), _ptr(out_dev), budget, window, _stream(stream)),
+        "kvr_decode_step_host")
 
 
 def kvr_absorb_chunk(h, layer_begin, layer_end, chunk, q, k_new, v_new, out,

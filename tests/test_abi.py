@@ -109,3 +109,15 @@ def test_entropy_descriptor_and_buffer_checks_on_host():
     st = kvr.lib.kvr_entropy_create(ctypes.byref(good), ctypes.c_void_p(0x1000),
                                     need - 1, None, ctypes.byref(h))
     assert st == kvr.KVR_ENOMEM
+
+
+def test_host_step_rejects_null_buffers_on_host():
+    """kvr_decode_step_host checks its host and staging pointers (and the
+    handle) before it enqueues anything."""
+    one = ctypes.c_void_p(16)
+    st = kvr.lib.kvr_decode_step_host(None, 0, 1, None, one, one, one, one,
+                                      one, one, one, 4, 1, None)
+    assert st == kvr.KVR_EINVAL and "null host" in kvr.kvr_last_error()
+    st = kvr.lib.kvr_decode_step_host(None, 0, 1, one, one, one, one, one,
+                                      one, one, one, 4, 1, None)
+    assert st == kvr.KVR_EINVAL and "null cache" in kvr.kvr_last_error()

@@ -261,3 +261,50 @@ def test_scores_view_matches_export():
                                       e["score"][l, h, :k])
                 assert np.array_equal(pos[s, l, h, :k].cpu().numpy(),
                                       e["pos"][l, h, :k])
+
+
+def test_host_buffer_step_equals_device_step():
+    """kvr_decode_step_host (host q/k/v in, host output out, the library
+    copying) gives the device call's result bit for bit, with the steps
+    alternating over two streams and two staging sets (the library orders
+    them), first evictions included."""
+    w = inputs.Workload("h", 3, 2, 7, 128, "bf16", 10, 3, 0, 0, sigma=1.0)
+    lens = [40, 13, 27]
+    c1, _ = harness.make_pair(w, 71, 3, cap=41, prompt_lens=lens, out_dtype="bf16")
+    c2, _ = harness.make_pair(w, 71, 3, cap=41, prompt_lens=lens, out_dtype="bf16")
+    streams = [torch.cuda.Stream(), torch.cuda.Stream()]
+    stage = [None, None]
+    hout = [None, None]
+    outs = []
+    hold = []  # pinned inputs stay alive until the library's copies are done
+    for t in range(8):
+        q, kn, vn = (harness.dev(a, w.dtype) for a in inputs.step_inputs(w, 71, t, 3))
+        outs.append(c1.step(q, kn, vn, w.budget, w.window).cpu())
+        j = t % 2
+        torch.cuda.synchronize()
+        if stage[j] is None:
+            stage[j] = tuple(torch.empty_like(x) for x in (q, kn, vn)) + \
+                (torch.empty_like(outs[-1], device="cuda"),)
+            hout[j] = torch.empty_like(outs[-1]).pin_memory()
+        else:
+            streams[j].synchronize()  # host buffers of step t - 2 read back
+            assert torch.equal(hout[j], outs[t - 2]), f"step {t - 2}"
+        hq, hk, hv = (x.cpu().pin_memory() for x in (q, kn, vn))
+        hold.append((hq, hk, hv))
+        kvr.kvr_decode_step_host(c2.handle, 0, w.n_layers, hq, hk, hv, hout[j],
+                                 *stage[j], w.budget, w.window, streams[j])
+    torch.cuda.synchronize()
+    for t in (6, 7):
+        assert torch.equal(hout[t % 2], outs[t]), f"step {t}"
+    c1.sync_status()
+    c2.sync_status()
+    for s in range(3):
+        a, b = c1.export(s), c2.export(s)
+        assert np.array_equal(a["len"], b["len"]), s
+        assert np.array_equal(a["next_pos"], b["next_pos"]), s
+        for l in range(w.n_layers):
+            for h in range(w.n_kv_heads):
+                n = a["len"][l, h]  # slots past the live rows are never read
+                for key in ("pos", "score", "K", "V"):
+                    assert np.array_equal(a[key][l, h, :n], b[key][l, h, :n]), \
+                        (s, l, h, key)
