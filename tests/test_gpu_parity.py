@@ -198,6 +198,23 @@ def test_long_unit_fused_step(B, G, out, chunk):
     assert c.launch_count() - n0 == 5
 
 
+@pytest.mark.parametrize("rows", [128, 129, 1024, 1025, 2048, 2049])
+def test_kernel_row_limits(rows):
+    """Units at each one-launch kernel's row limit and one row past it (rows
+    counted with the appended one): staged fused <= 128, chunked <= 1024,
+    streaming <= 2048, then the generic attend + evict pair.  Steady state,
+    one eviction a step, ragged units, in lock-step with the oracle."""
+    W = 8
+    B = rows - 1 - W
+    w = inputs.Workload("lim", 2, 2, 7, 128, "bf16", B, W, B + W, 4, sigma=1.0)
+    c, o = harness.make_pair(w, 16, 2, cap=rows, prompt_lens=[B + W, B + W - 37],
+                             out_dtype="bf16")
+    n0 = c.launch_count()
+    harness.lockstep(c, o, w, 16, 4, B, W)
+    launches = c.launch_count() - n0
+    assert launches == 4 if rows <= 2048 else launches == 8
+
+
 @pytest.mark.parametrize("chunk", [(0, 0), (-1, 0)], ids=["chunked", "stream"])
 def test_long_unit_growth_without_eviction(chunk):
     """Units growing from 100 to 300 rows with no eviction: the staged kernel
