@@ -59,30 +59,31 @@ def test_rkv_7b(lam):
 
 def test_rkv_unscaled_keys_and_ragged_lengths():
     """Peaked attention (unscaled keys), sequences of different lengths, a
-    budget of 0 and of 1."""
+    budget of 0 and of 1 (first evictions dropping up to 26 rows)."""
     w2 = inputs.Workload("u", 3, 2, 4, 128, "bf16", 1, 3, 0, 0, sigma=1.0)
     for wk, B in ((w2, 1), (w2, 0)):
         c, o = harness.make_pair(wk, 43, 3, cap=40, prompt_lens=[30, 4, 0])
         rkv_lockstep(c, o, wk, 43, 8, B, wk.window, 0.1)
 
 
-def test_rkv_duplicate_and_zero_keys():
+@pytest.mark.parametrize("d,dtype", [(64, "f32"), (128, "bf16")])
+def test_rkv_duplicate_and_zero_keys(d, dtype):
     """Keys that repeat, and a zero key: with lambda = 0 the duplicates are
     the most redundant rows and go first; a zero key has cosine 0."""
-    d, n = 64, 24
+    n = 24
     rng = np.random.default_rng(44)
-    K = rng.standard_normal((n, d)).astype(np.float32)
+    K = inputs.round_to(rng.standard_normal((n, d)).astype(np.float32), dtype)
     K[5] = K[2]
     K[9] = K[2]
     K[14] = 0.0
-    V = rng.standard_normal((n, d)).astype(np.float32)
-    w = inputs.Workload("z", 1, 1, 2, d, "f32", 10, 2, n, 0, sigma=1.0)
-    c = kvr.Cache(1, 1, 1, 2, d, n + 1, kv_dtype="f32", out_dtype="f32")
+    V = inputs.round_to(rng.standard_normal((n, d)).astype(np.float32), dtype)
+    w = inputs.Workload("z", 1, 1, 2, d, dtype, 10, 2, n, 0, sigma=1.0)
+    c = kvr.Cache(1, 1, 1, 2, d, n + 1, kv_dtype=dtype, out_dtype="f32")
     o = orc.OracleCache(1, 1, 1, 2, d, n + 1)
-    c.load(0, harness.dev(K[None, None], "f32"), harness.dev(V[None, None], "f32"))
+    c.load(0, harness.dev(K[None, None], dtype), harness.dev(V[None, None], dtype))
     o.load(0, K[None, None], V[None, None])
     q, kn, vn = inputs.step_inputs(w, 44, 0, 1)
-    c.attend_score(*(harness.dev(a, "f32") for a in (q, kn, vn)))
+    c.attend_score(*(harness.dev(a, dtype) for a in (q, kn, vn)))
     o.step(q, kn, vn, evict=False)
     c.evict_rkv(10, 2, 0.0)
     got = set(c.export(0, kv=False)["pos"][0, 0, :12].tolist())
