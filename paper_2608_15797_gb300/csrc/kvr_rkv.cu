@@ -333,7 +333,7 @@ __global__ void __launch_bounds__(kThreads)
     return x;
   };
   // Rows go kU pairs a step, all their loads issued before any is used.
-  constexpr int kU = 4;
+  constexpr int kU = 5;
   auto load_rows = [&](int i0, float (&v)[kU][kE]) {
 #pragma unroll
     for (int q = 0; q < kU; ++q) {
