@@ -72,6 +72,10 @@ def parse():
                         "16k context; fork: 72B best-of-8 candidate step")
     p.add_argument("--entropy-dtype", default="bf16", choices=["bf16", "f32"],
                    help="logit element type for --mode entropy")
+    p.add_argument("--fork-kernel", type=int, default=0, choices=[0, 1, 2, 3, 4],
+                   help="--mode fork candidate kernel (kvr_fork_set_kernel): "
+                        "0 library's choice, 1 batched, 2 chunked, 3 one CTA "
+                        "a unit, 4 generic")
     p.add_argument("--absorb-kernel", type=int, default=0, choices=[0, 1],
                    help="--mode absorb kernel: 0 tcgen05 (tensor memory), "
                         "1 mma.sync")
@@ -833,7 +837,7 @@ def run_fork(args):
     done = 0
     warm = True
     while done < K:
-        f = kvr.Fork(cache, N, T)
+        f = kvr.Fork(cache, N, T, kernel=args.fork_kernel)
         steps_here = T
         def step(i):
             kvr.kvr_fork_decode_attend_score(f.handle, 0, L, q, kn, vn, out, stream)
