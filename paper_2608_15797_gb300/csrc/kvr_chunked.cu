@@ -49,6 +49,7 @@ using namespace ptx;
 constexpr int kCR = 32;       // rows per chunk
 constexpr int kBox = 16;      // rows per TMA box (and per MMA tile)
 constexpr int kU = 2;         // consumer warps per group, one tile each
+static_assert(kU == 2, "the partial-output exchange pairs two warps");
 constexpr int kMaxGroups = 4;
 constexpr int kMaxStages = 4; // per group
 constexpr int kQPitch = 272;  // bytes per staged query row (256 + 16 padding)
@@ -84,8 +85,9 @@ struct ChunkGroup {
   __host__ __device__ explicit ChunkGroup(int n_max) {
     const int n = round_up16(n_max);
     xs = 0;                      // [kU][5] 16-byte slots
-    ox = 256;                    // [kU][8][32] float4 partial outputs
-    lg = ox + kU * 8 * 32 * 16;  // [n][8] scaled logits
+    ox = 256;                    // [kU][4][32] float4 partial outputs: the
+                                 // 4 head-dim tiles the other warp owns
+    lg = ox + kU * 4 * 32 * 16;  // [n][8] scaled logits
     sc = lg + n * 8 * 4;         // [n] old scores
     ps = sc + n * 4;             // [n] positions
     ns = ps + n * 4;             // [n] new scores
@@ -475,10 +477,13 @@ __global__ void __launch_bounds__(kMaxGroups * (kU + 1) * 32, 1)
         l1 += __shfl_xor_sync(0xffffffffu, l1, off);
       }
       if (lane < 4) XS4[w * 5 + lane] = make_float4(m0, m1, l0, l1);
+      // The partials of the head-dim tiles the other warp owns (mt of the
+      // other parity); each warp keeps its own tiles' partials in registers.
 #pragma unroll
       for (int mt = 0; mt < 8; ++mt)
-        OX[(w * 8 + mt) * 32 + lane] =
-            make_float4(o[mt][0], o[mt][1], o[mt][2], o[mt][3]);
+        if ((mt & 1) != w)
+          OX[(w * 4 + (mt >> 1)) * 32 + lane] =
+              make_float4(o[mt][0], o[mt][1], o[mt][2], o[mt][3]);
       group_bar(bar_id, 32 * kU);
       // Per head: the merged maximum and 1 / sum, for all 8 heads (the
       // scores need every head) and the warps' rescale factors for this
@@ -518,18 +523,21 @@ __global__ void __launch_bounds__(kMaxGroups * (kU + 1) * 32, 1)
           atomicOr(c.err, ERR_NONFINITE);
       }
       const Job jb = job_of(p, idx);
-      // Output: warp w owns head-dim tiles w, w + kU, ...
+      // Output: warp w owns head-dim tiles of parity w; the two warps'
+      // terms are added in warp order.
       {
         constexpr int osz = kOutBf16 ? 2 : 4;
         unsigned char *gout = reinterpret_cast<unsigned char *>(p.out) +
                               jb.orow * G * 128 * osz;
 #pragma unroll
-        for (int i = 0; i < 8 / kU; ++i) {
-          const int mt = w + i * kU;
+        for (int mt = 0; mt < 8; ++mt) {
+          if ((mt & 1) != w) continue;
+          const float4 mine = make_float4(o[mt][0], o[mt][1], o[mt][2], o[mt][3]);
+          const float4 other = OX[((1 - w) * 4 + (mt >> 1)) * 32 + lane];
           float e0 = 0.f, e1 = 0.f, e2 = 0.f, e3 = 0.f;
 #pragma unroll
           for (int v = 0; v < kU; ++v) {
-            const float4 x = OX[(v * 8 + mt) * 32 + lane];
+            const float4 x = v == w ? mine : other;
             e0 += x.x * fv0[v];
             e1 += x.y * fv1[v];
             e2 += x.z * fv0[v];
