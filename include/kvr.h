@@ -456,6 +456,23 @@ kvr_status kvr_decode_attend_score_noalloc(kvr_cache *cache, int layer_begin,
 
 /* ---- inspection -------------------------------------------------------- */
 
+/* Synchronising: wait for stream, then replace sequence seq's state with a
+ * host copy in the layout kvr_cache_export writes (resuming a decode, or a
+ * state built outside the library): host_k, host_v [L][H][capacity][d]
+ * (kv_dtype); host_score [L][H][capacity] fp32; host_pos [L][H][capacity]
+ * int32; host_len and host_next_pos [L][H] int32.  Rows [0, len) of a unit
+ * are live; the rest are copied but never read.  Checked on the host before
+ * anything is copied (KVR_EINVAL): no pointer is NULL; 0 <= len <=
+ * capacity; the KV heads of a layer share len and next_pos (every decode
+ * call keeps them equal); 0 <= next_pos < INT32_MAX; live positions are
+ * distinct and below next_pos.  KVR_ESTATE while the cache has a live fork.
+ * Importing what kvr_cache_export returned and decoding on gives the same
+ * results bit for bit. */
+kvr_status kvr_cache_import(kvr_cache *cache, int seq, const void *host_k,
+                            const void *host_v, const float *host_score,
+                            const int32_t *host_pos, const int32_t *host_len,
+                            const int32_t *host_next_pos, void *stream);
+
 /* Synchronising: wait for stream, then copy sequence seq's state to host.
  * host_k, host_v [L][H][capacity][d] (kv_dtype); host_score [L][H][capacity]
  * fp32; host_pos [L][H][capacity] int32; host_len and host_next_pos [L][H]

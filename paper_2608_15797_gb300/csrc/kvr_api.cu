@@ -957,6 +957,77 @@ kvr_status kvr_cache_export(const kvr_cache *c, int seq, void *host_k,
   return KVR_OK;
 }
 
+kvr_status kvr_cache_import(kvr_cache *c, int seq, const void *host_k,
+                            const void *host_v, const float *host_score,
+                            const int32_t *host_pos, const int32_t *host_len,
+                            const int32_t *host_next_pos, void *stream) {
+  if (!c) return fail(KVR_EINVAL, "null cache");
+  if (c->forks) return fail(KVR_ESTATE, "the cache has a live fork");
+  if (seq < 0 || seq >= c->desc.n_seq)
+    return fail(KVR_EINVAL, "sequence %d outside [0, %d)", seq, c->desc.n_seq);
+  if (!host_k || !host_v || !host_score || !host_pos || !host_len ||
+      !host_next_pos)
+    return fail(KVR_EINVAL, "null host buffer");
+  const CacheView &v = c->view;
+  const int L = v.L, H = v.H, cap = v.cap;
+  std::vector<int32_t> live;
+  for (int l = 0; l < L; ++l)
+    for (int h = 0; h < H; ++h) {
+      const size_t u = (size_t)l * H + h;
+      const int n = host_len[u], np = host_next_pos[u];
+      if (n < 0 || n > cap)
+        return fail(KVR_EINVAL, "layer %d head %d: length %d outside [0, %d]",
+                    l, h, n, cap);
+      if (np < 0 || np == INT32_MAX)
+        return fail(KVR_EINVAL, "layer %d head %d: next position %d", l, h, np);
+      if (n != host_len[(size_t)l * H] || np != host_next_pos[(size_t)l * H])
+        return fail(KVR_EINVAL,
+                    "layer %d: KV heads differ in length or next position", l);
+      live.assign(host_pos + u * cap, host_pos + u * cap + n);
+      std::sort(live.begin(), live.end());
+      for (int i = 0; i < n; ++i)
+        if (live[i] < 0 || live[i] >= np || (i > 0 && live[i] == live[i - 1]))
+          return fail(KVR_EINVAL,
+                      "layer %d head %d: live positions must be distinct and "
+                      "in [0, %d)", l, h, np);
+    }
+  cudaError_t e = cudaStreamSynchronize(as_stream(stream));
+  if (e != cudaSuccess) return cuda_fail("kvr_cache_import: sync", e);
+  const size_t units = (size_t)L * H, rows = units * cap;
+  const size_t ebytes = (size_t)v.d * esize(c->desc.kv_dtype);
+  e = cudaMemcpy(static_cast<char *>(v.K) + seq * rows * ebytes, host_k,
+                 rows * ebytes, cudaMemcpyHostToDevice);
+  if (e == cudaSuccess)
+    e = cudaMemcpy(static_cast<char *>(v.V) + seq * rows * ebytes, host_v,
+                   rows * ebytes, cudaMemcpyHostToDevice);
+  if (e == cudaSuccess)
+    e = cudaMemcpy2D(v.score + seq * units * v.sstride, (size_t)v.sstride * 4,
+                     host_score, (size_t)cap * 4, (size_t)cap * 4, units,
+                     cudaMemcpyHostToDevice);
+  if (e == cudaSuccess)
+    e = cudaMemcpy2D(v.pos + seq * units * v.sstride, (size_t)v.sstride * 4,
+                     host_pos, (size_t)cap * 4, (size_t)cap * 4, units,
+                     cudaMemcpyHostToDevice);
+  std::vector<int32_t> st(units * 4);
+  if (e == cudaSuccess)
+    e = cudaMemcpy(st.data(), v.state + seq * units * 4,
+                   st.size() * sizeof(int32_t), cudaMemcpyDeviceToHost);
+  if (e == cudaSuccess) {
+    for (size_t i = 0; i < units; ++i) {
+      st[4 * i] = host_len[i];
+      st[4 * i + 1] = host_next_pos[i];
+    }
+    e = cudaMemcpy(v.state + seq * units * 4, st.data(),
+                   st.size() * sizeof(int32_t), cudaMemcpyHostToDevice);
+  }
+  if (e != cudaSuccess) return cuda_fail("kvr_cache_import", e);
+  for (int l = 0; l < L; ++l) {
+    c->len[(size_t)seq * L + l] = host_len[(size_t)l * H];
+    c->next_pos[(size_t)seq * L + l] = host_next_pos[(size_t)l * H];
+  }
+  return KVR_OK;
+}
+
 kvr_status kvr_cache_lengths(const kvr_cache *c, int32_t *host_len) {
   if (!c || !host_len) return fail(KVR_EINVAL, "null argument");
   std::memcpy(host_len, c->len.data(), c->len.size() * sizeof(int32_t));

@@ -68,6 +68,7 @@ _SIGS = {
     "kvr_cache_copy_sequences": (_S, [_P, _P, _P, _P, _I, _P]),
     "kvr_evict_compact_rkv": (_S, [_P, _I, _I, _I, _I, ctypes.c_float, _P]),
     "kvr_cache_export": (_S, [_P, _I, _P, _P, _P, _P, _P, _P, _P]),
+    "kvr_cache_import": (_S, [_P, _I, _P, _P, _P, _P, _P, _P, _P]),
     "kvr_cache_lengths": (_S, [_P, _P]),
     "kvr_cache_launch_count": (_S, [_P, _P]),
     "kvr_cache_set_fused": (_S, [_P, _I]),
@@ -206,6 +207,14 @@ def kvr_cache_copy_sequences(dst, dst_seqs, src, src_seqs, stream=None):
     _check(lib.kvr_cache_copy_sequences(dst, _ptr(d), src, _ptr(s), len(d),
                                         _stream(stream)),
            "kvr_cache_copy_sequences")
+
+
+def kvr_cache_import(h, seq, host_k, host_v, host_score, host_pos, host_len,
+                     host_next_pos, stream=None):
+    _check(lib.kvr_cache_import(h, seq, _ptr(host_k), _ptr(host_v),
+                                _ptr(host_score), _ptr(host_pos),
+                                _ptr(host_len), _ptr(host_next_pos),
+                                _stream(stream)), "kvr_cache_import")
 
 
 def kvr_cache_export(h, seq, host_k, host_v, host_score, host_pos, host_len,
@@ -359,6 +368,17 @@ class Cache:
             res["K"] = hk.float().numpy()
             res["V"] = hv.float().numpy()
         return res
+
+    def import_state(self, seq, state, stream=None):
+        """Replace sequence seq with a state dict in the form export(seq,
+        kv=True) returns (kvr_cache_import); K/V are cast to kv_dtype."""
+        hk, hv = (torch.from_numpy(np.ascontiguousarray(state[x], np.float32))
+                  .to(self.kv_torch_dtype).contiguous() for x in ("K", "V"))
+        arr = {x: np.ascontiguousarray(state[x], t) for x, t in (
+            ("score", np.float32), ("pos", np.int32), ("len", np.int32),
+            ("next_pos", np.int32))}
+        kvr_cache_import(self.handle, seq, hk, hv, arr["score"], arr["pos"],
+                         arr["len"], arr["next_pos"], stream)
 
     def scores_view(self):
         """(score, pos, state) as device tensors viewing the cache buffer (no

@@ -121,3 +121,9 @@ def test_host_step_rejects_null_buffers_on_host():
     st = kvr.lib.kvr_decode_step_host(None, 0, 1, one, one, one, one, one,
                                       one, one, one, 4, 1, None)
     assert st == kvr.KVR_EINVAL and "null cache" in kvr.kvr_last_error()
+
+
+def test_import_rejects_null_arguments_on_host():
+    one = ctypes.c_void_p(16)
+    st = kvr.lib.kvr_cache_import(None, 0, one, one, one, one, one, one, None)
+    assert st == kvr.KVR_EINVAL and "null cache" in kvr.kvr_last_error()

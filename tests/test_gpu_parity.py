@@ -325,3 +325,49 @@ def test_host_buffer_step_equals_device_step():
                 for key in ("pos", "score", "K", "V"):
                     assert np.array_equal(a[key][l, h, :n], b[key][l, h, :n]), \
                         (s, l, h, key)
+
+
+def test_export_import_resumes_bit_for_bit():
+    """kvr_cache_import of what kvr_cache_export returned, into another cache
+    and into another sequence slot, then decoding on: outputs and live rows
+    equal the uninterrupted cache's bit for bit.  Bad states are refused."""
+    w = inputs.Workload("imp", 2, 2, 7, 128, "bf16", 10, 3, 0, 0, sigma=1.0)
+    c1, _ = harness.make_pair(w, 81, 2, cap=41, prompt_lens=[40, 13],
+                              out_dtype="bf16")
+    for t in range(3):
+        q, kn, vn = (harness.dev(a, w.dtype) for a in inputs.step_inputs(w, 81, t, 2))
+        c1.step(q, kn, vn, w.budget, w.window)
+    saved = [c1.export(s) for s in range(2)]
+    c2, _ = harness.make_pair(w, 82, 2, cap=41, prompt_lens=[5, 7], out_dtype="bf16")
+    c2.import_state(0, saved[0])
+    c2.import_state(1, saved[1])
+    for t in range(3, 8):
+        q, kn, vn = (harness.dev(a, w.dtype) for a in inputs.step_inputs(w, 81, t, 2))
+        o1 = c1.step(q, kn, vn, w.budget, w.window)
+        o2 = c2.step(q, kn, vn, w.budget, w.window)
+        torch.cuda.synchronize()
+        assert torch.equal(o1, o2), f"step {t}"
+    for s in range(2):
+        a, b = c1.export(s), c2.export(s)
+        assert np.array_equal(a["len"], b["len"]) and np.array_equal(a["next_pos"], b["next_pos"])
+        for l in range(w.n_layers):
+            for h in range(w.n_kv_heads):
+                n = a["len"][l, h]
+                for key in ("pos", "score", "K", "V"):
+                    assert np.array_equal(a[key][l, h, :n], b[key][l, h, :n]), (s, l, h, key)
+    # refused states: a length past the capacity, duplicate live positions,
+    # heads of one layer at different lengths
+    bad = []
+    x = {k: v.copy() for k, v in saved[0].items()}
+    x["len"][0, 0] = 42
+    bad.append(x)
+    x = {k: v.copy() for k, v in saved[0].items()}
+    x["pos"][1, 1, 1] = x["pos"][1, 1, 0]
+    bad.append(x)
+    x = {k: v.copy() for k, v in saved[0].items()}
+    x["len"][1, 0] -= 1
+    bad.append(x)
+    for x in bad:
+        with pytest.raises(kvr.KvrError) as e:
+            c2.import_state(0, x)
+        assert e.value.status == kvr.KVR_EINVAL
