@@ -42,6 +42,26 @@ constexpr int kMaxChunk = 64;
 constexpr int kMaxRows = 192;
 static_assert(kMaxRows <= kThreads, "one row per thread in the selection");
 
+// Packed fp32 pairs (round to nearest, no flush: the scalar code's results).
+__device__ __forceinline__ uint64_t pk2(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void upk2(uint64_t v, float &lo, float &hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t add2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ uint64_t mul2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
 __device__ __forceinline__ void cp_async_commit_wait_all() {
   asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
 }
@@ -597,28 +617,47 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int k = 0; k < kTcChunks; ++k)
       if (k < nch) tmem_ld16f_nowait(trow + kTcS + c_lo + 16 * k, e[k]);
     tmem_wait_ld();
+    const uint64_t scale2 = pk2(scale, scale);
 #pragma unroll
     for (int k = 0; k < kTcChunks; ++k) {
       if (k < nch) {
+        if (c_lo + 16 * k + 16 <= lim) {  // the whole chunk is visible
 #pragma unroll
-        for (int j = 0; j < 16; ++j) {
-          const bool in = c_lo + 16 * k + j < lim;
-          e[k][j] = in ? e[k][j] * scale : -INFINITY;
-          mx = fmaxf(mx, e[k][j]);
+          for (int j = 0; j < 16; j += 2) {
+            upk2(mul2(pk2(e[k][j], e[k][j + 1]), scale2), e[k][j], e[k][j + 1]);
+            mx = fmaxf(mx, fmaxf(e[k][j], e[k][j + 1]));
+          }
+        } else {
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            const bool in = c_lo + 16 * k + j < lim;
+            e[k][j] = in ? e[k][j] * scale : -INFINITY;
+            mx = fmaxf(mx, e[k][j]);
+          }
         }
       }
     }
-    float sm = 0.f;
     const float ref = mx == -INFINITY ? 0.f : mx;
+    const uint64_t nref2 = pk2(-ref, -ref);
+    uint64_t sm2 = pk2(0.f, 0.f);  // even and odd terms
 #pragma unroll
     for (int k = 0; k < kTcChunks; ++k) {
       if (k < nch) {
 #pragma unroll
-        for (int j = 0; j < 16; ++j) {
-          e[k][j] = ex2(e[k][j] - ref);  // exp2(-inf) = 0 for masked keys
-          sm += e[k][j];
+        for (int j = 0; j < 16; j += 2) {
+          float d0, d1;
+          upk2(add2(pk2(e[k][j], e[k][j + 1]), nref2), d0, d1);
+          e[k][j] = ex2(d0);  // exp2(-inf) = 0 for masked keys
+          e[k][j + 1] = ex2(d1);
+          sm2 = add2(sm2, pk2(e[k][j], e[k][j + 1]));
         }
       }
+    }
+    float sm;
+    {
+      float s0, s1;
+      upk2(sm2, s0, s1);
+      sm = s0 + s1;
     }
     if (upper) s_ml[r] = make_float2(mx, sm);
     __syncthreads();
@@ -639,6 +678,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (valid && !upper && !(L >= 1.f && L < INFINITY)) atomicOr(c.err, ERR_NONFINITE);
     // p = e * exp2(own max - row max) / row sum
     const float f = valid && L > 0.f && mx > -INFINITY ? ex2(mx - M) / L : 0.f;
+    const uint64_t f2 = pk2(f, f);
 #pragma unroll
     for (int k = 0; k < kTcChunks; ++k) {
       if (k < nch) {
@@ -646,10 +686,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint32_t hi[8], lo[8];
 #pragma unroll
         for (int j = 0; j < 16; j += 2) {
-          const float p0 = e[k][j] * f, p1 = e[k][j + 1] * f;
+          const uint64_t p2 = mul2(pk2(e[k][j], e[k][j + 1]), f2);
+          float p0, p1;
+          upk2(p2, p0, p1);
           const __nv_bfloat162 b = __floats2bfloat162_rn(p0, p1);
           hi[j >> 1] = *reinterpret_cast<const uint32_t *>(&b);
-          lo[j >> 1] = pack_bf16(p0 - __low2float(b), p1 - __high2float(b));
+          float r0, r1;  // p - bf16(p), both terms at once
+          upk2(add2(p2, pk2(-__low2float(b), -__high2float(b))), r0, r1);
+          lo[j >> 1] = pack_bf16(r0, r1);
         }
         const int kb = c0 >> 6, ch = (c0 & 63) >> 3;
         const uint32_t o0 = kb * (kTcRows * 128) + r * 128 + (((ch) ^ (r & 7)) << 4);
