@@ -32,6 +32,21 @@ namespace {
 
 using namespace dev;
 
+// Packed fp32 pairs (round to nearest, no flush).
+__device__ __forceinline__ uint64_t pk2(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void upk2(uint64_t v, float &lo, float &hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+
 // A float's order as an unsigned integer, negative values included.
 __device__ __forceinline__ unsigned ord_bits(float z) {
   const unsigned b = __float_as_uint(z);
@@ -345,29 +360,43 @@ __global__ void __launch_bounds__(kThreads)
       }
     }
   };
-  // Pass 1: S = sum of the normalised keys (this lane's kE dimensions);
-  // rs[i] = 1 / |k_i| (0 for a zero key).
-  float S[kE];
+  // Pass 1: S = sum of the normalised keys (this lane's kE dimensions, as
+  // packed fp32 pairs); rs[i] = 1 / |k_i| (0 for a zero key).
+  static_assert(kE % 2 == 0, "dimension pairs");
+  uint64_t S2[kE / 2];
 #pragma unroll
-  for (int j = 0; j < kE; ++j) S[j] = 0.f;
+  for (int j = 0; j < kE / 2; ++j) S2[j] = pk2(0.f, 0.f);
   for (int i0 = 0; i0 < n; i0 += 2 * kU) {
     float v[kU][kE];
     load_rows(i0, v);
 #pragma unroll
     for (int q = 0; q < kU; ++q) {
-      float ss = 0.f;
+      uint64_t ss2 = pk2(0.f, 0.f);
 #pragma unroll
-      for (int j = 0; j < kE; ++j) ss = fmaf(v[q][j], v[q][j], ss);
-      ss = half_sum(ss);
+      for (int j = 0; j < kE; j += 2) {
+        const uint64_t x = pk2(v[q][j], v[q][j + 1]);
+        ss2 = fma2(x, x, ss2);
+      }
+      float sa, sb;
+      upk2(ss2, sa, sb);
+      const float ss = half_sum(sa + sb);
       const float inv = ss > 0.f ? 1.f / sqrtf(ss) : 0.f;
+      const uint64_t inv2 = pk2(inv, inv);
 #pragma unroll
-      for (int j = 0; j < kE; ++j) S[j] = fmaf(v[q][j], inv, S[j]);
+      for (int j = 0; j < kE; j += 2)
+        S2[j / 2] = fma2(pk2(v[q][j], v[q][j + 1]), inv2, S2[j / 2]);
       const int i = i0 + 2 * q + half;
       if (l16 == 0 && i < n) rs[i] = inv;
     }
   }
 #pragma unroll
-  for (int j = 0; j < kE; ++j) S[j] += __shfl_xor_sync(0xffffffffu, S[j], 16);
+  for (int j = 0; j < kE / 2; ++j) {
+    float a, b;
+    upk2(S2[j], a, b);
+    a += __shfl_xor_sync(0xffffffffu, a, 16);
+    b += __shfl_xor_sync(0xffffffffu, b, 16);
+    S2[j] = pk2(a, b);
+  }
   // Pass 2: each row's mean cosine with the other live rows (the lane that
   // wrote rs[i] in pass 1 reads and replaces it).
   const float inv_n1 = 1.f / (float)(n - 1);
@@ -377,10 +406,13 @@ __global__ void __launch_bounds__(kThreads)
 #pragma unroll
     for (int q = 0; q < kU; ++q) {
       const int i = i0 + 2 * q + half;
-      float dot = 0.f;
+      uint64_t dot2 = pk2(0.f, 0.f);
 #pragma unroll
-      for (int j = 0; j < kE; ++j) dot = fmaf(v[q][j], S[j], dot);
-      dot = half_sum(dot);
+      for (int j = 0; j < kE; j += 2)
+        dot2 = fma2(pk2(v[q][j], v[q][j + 1]), S2[j / 2], dot2);
+      float da, db;
+      upk2(dot2, da, db);
+      const float dot = half_sum(da + db);
       if (l16 == 0 && i < n) {
         const float inv = rs[i];
         rs[i] = (dot * inv - (inv > 0.f ? 1.f : 0.f)) * inv_n1;
