@@ -47,6 +47,21 @@ namespace {
 
 using namespace ptx;
 
+// Packed fp32 pairs (round to nearest, no flush).
+__device__ __forceinline__ uint64_t pk2(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void upk2(uint64_t v, float &lo, float &hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t mul2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
 constexpr int kBox = 16;         // rows per partial-prefix TMA box, per MMA tile
 constexpr int kBlockRows = 128;  // rows of a block
 constexpr int kMaxCand = 8;
@@ -164,12 +179,13 @@ __device__ __forceinline__ void tile_group(const unsigned char *K0,
   m1 = n1;
   l0 *= a0;
   l1 *= a1;
+  {
+    const uint64_t a2 = pk2(a0, a1);  // (head c2, head c2 + 1)
 #pragma unroll
-  for (int mt = 0; mt < 8; ++mt) {
-    o[mt][0] *= a0;
-    o[mt][2] *= a0;
-    o[mt][1] *= a1;
-    o[mt][3] *= a1;
+    for (int mt = 0; mt < 8; ++mt) {
+      upk2(mul2(pk2(o[mt][0], o[mt][1]), a2), o[mt][0], o[mt][1]);
+      upk2(mul2(pk2(o[mt][2], o[mt][3]), a2), o[mt][2], o[mt][3]);
+    }
   }
 #pragma unroll
   for (int t = 0; t < kGroupTiles; ++t) {
