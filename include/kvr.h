@@ -264,6 +264,25 @@ void kvr_fork_destroy(kvr_fork *fork);
  * generic kernel for that call.  Returns KVR_EINVAL outside [0, 4]. */
 kvr_status kvr_fork_set_kernel(kvr_fork *fork, int kernel);
 
+/* Bound, in nanoseconds, of each wait of the step kernels (fused,
+ * chunked and streaming) on an asynchronous copy into shared memory for this
+ * cache.  A wait that runs out sets the timeout bit of the device error
+ * word; the launch then waits (up to the default bound) for the copies it
+ * has in flight, leaves the units it had not finished untouched and
+ * returns, and the next kvr_sync_status reports KVR_EDEVICE.  The cache's
+ * state is then undefined for those units: restore it with
+ * kvr_cache_import.  Not tied to a passage of the paper (failure handling
+ * only).  ns: 1 .. 2e9; 0 restores the default of 2 s.  KVR_EINVAL above
+ * the default or for a null cache. */
+kvr_status kvr_cache_set_wait_limit(kvr_cache *cache, uint64_t ns);
+
+/* Testing hook for the timeout path: while enable != 0, the fused and
+ * chunked step kernels never load the first unit of their first CTA, so
+ * the wait for it runs out after the cache's wait limit (no fault, no
+ * hang; the launch returns with the timeout bit set, as above).  Never
+ * enabled by the library itself.  enable: 0 or 1. */
+kvr_status kvr_cache_set_hold_first_unit(kvr_cache *cache, int enable);
+
 /* Choose whether kvr_decode_attend_score / kvr_decode_step may use the
  * fused single-pass kernel (bf16, head_dim 128, G <= 8, at most 128 live rows
  * per unit, at most one eviction per unit; the default) or must use the

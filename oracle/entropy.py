@@ -27,10 +27,6 @@ Readings where the paper is silent:
   (1 unless stated), before any top-k / top-p truncation: with top-k 20 the
   entropy could never exceed ln 20 < 3, so tau_ent = 7 would never fire.
 
-``decide_fp32`` takes the same decision from float32 entropies in float32
-arithmetic (a sum over the window from oldest to newest, compared with
-tau * |W_e|), the precision in which the kernel decides.
-
 Pins: ``tests/test_entropy_oracle_pins.py`` (scipy's entropy of scipy's softmax,
 closed forms, invariances) and ``tests/golden/entropy_detector_worked.json``
 (hand-derived stop positions).
@@ -90,22 +86,3 @@ class EntropyDetector:
             if e > self.guard and mean[r] > self.tau:
                 self.stop[r] = e
         return mean, self.stop.copy()
-
-
-def decide_fp32(hist32, window: int, guard: int, tau: float):
-    """The test at the row's latest position in float32 arithmetic.
-
-    ``hist32`` holds the row's float32 entropies since its reset, oldest
-    first.  Returns (mean32, fires): the float32 window sum divided by
-    |W_e|, and whether e > guard and sum > tau * |W_e| (tau rounded to
-    float32, the product taken in float32)."""
-    h = np.asarray(hist32, dtype=np.float32)
-    e = len(h)
-    win = h[-window:]
-    n = np.float32(len(win))
-    acc = np.float32(0.0)
-    for x in win:
-        acc = np.float32(acc + x)
-    mean = np.float32(acc / n)
-    fires = bool(e > guard and acc > np.float32(np.float32(tau) * n))
-    return mean, fires

@@ -9,7 +9,8 @@ the CUDA cache state with an ``OracleCache`` after each step:
   1e-6);
 * retained sets: equal to the oracle's TopB-with-window set, except for
   swaps between rows whose oracle scores lie within 1e-4 relative of each
-  other (ties go to the lower position).  After a valid but different set the
+  other; between rows of exactly equal oracle score the lower position must
+  be the one kept (``check_swaps``).  After a valid but different set the
   oracle adopts the CUDA set, so both continue from the same state; the
   number of adoptions is reported.
 """
@@ -68,6 +69,36 @@ def _window_positions(pos, W):
     return set(np.sort(pos)[::-1][:W].tolist())
 
 
+def check_swaps(kept, dropped, slack, where, what, relative):
+    """A retained set that differs from the oracle's TopB is valid only if
+    every dropped candidate ranks at most a near-tie above the lowest kept
+    one, and exact ties follow the order of Eq. 1's TopB as read here:
+    between two rows of equal oracle value the lower position is kept.
+
+    kept, dropped: (value, position) pairs of the non-window rows.  With
+    `relative`, a near-tie is value_dropped <= lowest_kept * (1 + SWAP_RTOL);
+    otherwise value_dropped <= lowest_kept + slack."""
+    if not kept:
+        return
+    lo = min(v for v, _ in kept)
+    for v, p in dropped:
+        bound = lo * (1.0 + SWAP_RTOL) if relative else lo + slack
+        if v > bound:
+            raise ParityError(
+                f"{where}: evicted pos {p} ({what} {v:.9g}) while keeping a "
+                f"row of {what} {lo:.9g}: not a near-tie")
+    # Exact ties: a kept row may not sit above a dropped row of the same
+    # value (the lower position wins).
+    top = {}
+    for v, p in kept:
+        top[v] = max(top.get(v, -1), p)
+    for v, p in dropped:
+        if v in top and top[v] > p:
+            raise ParityError(
+                f"{where}: exact tie at {what} {v:.17g}: kept pos {top[v]} "
+                f"and evicted the lower pos {p}")
+
+
 def check_unit(o_pos, o_score, g_pos, g_score, B, W, evict, where=""):
     """Compare one unit.  o_*: oracle rows before eviction (all n rows);
     g_*: CUDA rows after the step.  Returns (adopted, max_score_rel)."""
@@ -92,14 +123,9 @@ def check_unit(o_pos, o_score, g_pos, g_score, B, W, evict, where=""):
     ref = dict(zip(o_pos.tolist(), o_score.tolist()))
     adopted = False
     if got != want:
-        kept = [ref[p] for p in got - window]
+        kept = [(ref[p], p) for p in got - window]
         dropped = [(ref[p], p) for p in set(o_pos.tolist()) - got]
-        lo = min(kept) if kept else np.inf
-        for s, p in dropped:
-            if s > lo * (1.0 + SWAP_RTOL):
-                raise ParityError(
-                    f"{where}: evicted pos {p} (score {s:.9g}) while keeping a "
-                    f"row of score {lo:.9g}: not a near-tie")
+        check_swaps(kept, dropped, 0.0, where, "score", relative=True)
         adopted = True
     # Scores of the retained rows.
     s_ref = np.array([ref[p] for p in g_pos.tolist()])
@@ -192,15 +218,13 @@ def check_and_adopt_rkv(o: orc.OracleCache, exports, B, W, lam,
                             raise ParityError(f"{where}: window evicted")
                         zc = z[cand]
                         tol = RKV_SWAP_ATOL * float(np.abs(zc).max()) + 1e-9
-                        kept = [z[i] for i in np.nonzero(cand)[0]
+                        ci = np.nonzero(cand)[0]
+                        kept = [(float(z[i]), int(pos[i])) for i in ci
                                 if pos[i] in got]
-                        lo = min(kept) if kept else np.inf
-                        for i in np.nonzero(cand)[0]:
-                            if pos[i] not in got and z[i] > lo + tol:
-                                raise ParityError(
-                                    f"{where}: evicted pos {pos[i]} (z "
-                                    f"{z[i]:.9g}) while keeping z {lo:.9g}: "
-                                    "not a near-tie")
+                        dropped = [(float(z[i]), int(pos[i])) for i in ci
+                                   if pos[i] not in got]
+                        check_swaps(kept, dropped, tol, where, "z",
+                                    relative=False)
                         adopted = True
                 ref = dict(zip(pos.tolist(), o.score[s, l, h, :n].tolist()))
                 s_ref = np.array([ref[p] for p in g_pos.tolist()])

@@ -555,6 +555,8 @@ kvr_status kvr_cache_create(const kvr_cache_desc *desc, void *dev_buf,
                 : (float)(1.0 / std::sqrt((double)desc->head_dim));
   v.kv_bf16 = desc->kv_dtype == KVR_BF16;
   v.out_bf16 = desc->out_dtype == KVR_BF16;
+  v.wait_ns = kvr::kDefaultWaitNs;
+  v.hold_first = 0;
   c->len.assign((size_t)v.S * v.L, 0);
   c->next_pos.assign((size_t)v.S * v.L, 0);
   cudaError_t e = kvr::launch_init(v, as_stream(stream));
@@ -674,6 +676,21 @@ kvr_status kvr_cache_set_absorb_kernel(kvr_cache *c, int kernel) {
   if (!c) return fail(KVR_EINVAL, "null cache");
   if (kernel < 0 || kernel > 1) return fail(KVR_EINVAL, "kernel must be 0 or 1");
   c->absorb_kernel = kernel;
+  return KVR_OK;
+}
+
+kvr_status kvr_cache_set_wait_limit(kvr_cache *c, uint64_t ns) {
+  if (!c) return fail(KVR_EINVAL, "null cache");
+  if (ns > kvr::kDefaultWaitNs)
+    return fail(KVR_EINVAL, "wait limit %llu ns above the %llu ns default",
+                (unsigned long long)ns, kvr::kDefaultWaitNs);
+  c->view.wait_ns = ns ? ns : kvr::kDefaultWaitNs;
+  return KVR_OK;
+}
+
+kvr_status kvr_cache_set_hold_first_unit(kvr_cache *c, int enable) {
+  if (!c) return fail(KVR_EINVAL, "null cache");
+  c->view.hold_first = enable != 0;
   return KVR_OK;
 }
 
@@ -1061,10 +1078,11 @@ kvr_status kvr_sync_status(kvr_cache *c, void *stream) {
   if (!word) return KVR_OK;
   e = cudaMemset(c->view.err, 0, sizeof word);
   if (e != cudaSuccess) return cuda_fail("kvr_sync_status: clear", e);
-  return fail(KVR_EDEVICE, "device error word 0x%x (%s%s%s)", word,
+  return fail(KVR_EDEVICE, "device error word 0x%x (%s%s%s%s)", word,
               word & kvr::ERR_CAPACITY ? "capacity " : "",
               word & kvr::ERR_NONFINITE ? "non-finite " : "",
-              word & kvr::ERR_LENGTH ? "length" : "");
+              word & kvr::ERR_LENGTH ? "length " : "",
+              word & kvr::ERR_TIMEOUT ? "timeout" : "");
 }
 
 const char *kvr_last_error(void) { return g_err.c_str(); }

@@ -139,6 +139,9 @@ __device__ void produce(const ChunkParams &p, const CUtensorMap *tmK,
                         uint64_t *full, uint64_t *empty, int g, int mine,
                         int lane, volatile int *abort, int *issued) {
   const CacheView &c = p.c;
+  // Test hook: group 0 of CTA 0 never loads its first job (no copy is
+  // issued, so there is nothing to drain); its consumers' wait runs out.
+  if (c.hold_first && blockIdx.x == 0 && g == 0) return;
   int seq = 0;
   for (int k = g; k < mine; k += p.n_groups) {
     const int idx = (int)blockIdx.x + k * (int)gridDim.x;
@@ -163,7 +166,8 @@ __device__ void produce(const ChunkParams &p, const CUtensorMap *tmK,
       const int s = seq % p.n_stages;
       const uint32_t ph = (uint32_t)(seq / p.n_stages) & 1u;
       int got = 1;
-      if (lane == 0) got = mbar_wait(smem_u32(&empty[s]), ph ^ 1u, abort);
+      if (lane == 0)
+        got = mbar_wait(smem_u32(&empty[s]), ph ^ 1u, abort, c.wait_ns);
       got = __shfl_sync(0xffffffffu, got, 0);
       if (!got) {
         if (lane == 0) {
@@ -338,7 +342,8 @@ __global__ void __launch_bounds__(kMaxGroups * (kU + 1) * 32, 1)
         // One warp waits (bounded) and tells the group, so that both warps
         // take the same branch before the group's next barrier.
         if (w == 0 && lane == 0) {
-          const bool ok = mbar_wait(smem_u32(&full_bar[g][s]), ph, &s_abort);
+          const bool ok =
+              mbar_wait(smem_u32(&full_bar[g][s]), ph, &s_abort, c.wait_ns);
           s_ok[g] = ok ? 1 : 0;
           if (!ok) {
             atomicOr(c.err, ERR_TIMEOUT);
@@ -535,7 +540,8 @@ __global__ void __launch_bounds__(kMaxGroups * (kU + 1) * 32, 1)
             fv1[v] = eb[v] * ib;
           }
         }
-        if (cp == 0 && w == 0 && lane == 0 && !(Za > 0.5f && Za < INFINITY))
+        if (w == 0 && lane == 0 &&
+            !(Za > 0.5f && Za < INFINITY && Zb > 0.5f && Zb < INFINITY))
           atomicOr(c.err, ERR_NONFINITE);
       }
       const Job jb = job_of(p, idx);

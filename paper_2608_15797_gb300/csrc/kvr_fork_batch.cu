@@ -525,7 +525,8 @@ __global__ void __launch_bounds__((kMaxCand + 1) * 32, 1)
         l1 += __shfl_xor_sync(0xffffffffu, l1, off);
       }
       const float i0 = rcp(l0), i1 = rcp(l1);
-      if (lane == 0 && !(l0 > 0.5f && l0 < INFINITY)) atomicOr(c.err, ERR_NONFINITE);
+      if (lane < 4 && !(l0 > 0.5f && l0 < INFINITY && l1 > 0.5f && l1 < INFINITY))
+        atomicOr(c.err, ERR_NONFINITE);
       const Unit u = unit_of(p, idx);
       const size_t orow = (size_t)cand * per + u.row0;
       const size_t cu = (size_t)cand * units + u.ug;

@@ -293,7 +293,8 @@ __global__ void __launch_bounds__(32 * kMaxCand)
         l1 += __shfl_xor_sync(0xffffffffu, l1, off);
       }
       const float i0 = 1.f / l0, i1 = 1.f / l1;
-      if (lane == 0 && !(l0 >= 1.f && l0 < INFINITY)) atomicOr(c.err, ERR_NONFINITE);
+      if (lane < 4 && !(l0 >= 1.f && l0 < INFINITY && l1 >= 1.f && l1 < INFINITY))
+        atomicOr(c.err, ERR_NONFINITE);
       // Output of this candidate (fragments -> rows via movmatrix for bf16).
       const int c2 = (lane & 3) * 2, r0l = lane >> 2;
       constexpr int osz = kOutBf16 ? 2 : 4;

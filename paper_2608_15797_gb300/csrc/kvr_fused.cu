@@ -156,13 +156,16 @@ __device__ __forceinline__ void issue_unit(const FusedParams &p,
 
 #include "kvr_fused_unit.cuh"
 
+static_assert(kDefaultWaitNs == kWaitNs, "one default wait bound");
+
 // Bounded wait until the producer has recorded unit k (or a later one) as
 // issued into this stage; false on timeout or abort.
-__device__ bool wait_issued(volatile int *issued, int k, volatile int *abort) {
+__device__ bool wait_issued(volatile int *issued, int k, volatile int *abort,
+                            uint64_t limit_ns) {
   if (*issued >= k) return true;
   const uint64_t t0 = global_ns();
   while (*issued < k) {
-    if (*abort || global_ns() - t0 > kWaitNs) return false;
+    if (*abort || global_ns() - t0 > limit_ns) return false;
   }
   return true;
 }
@@ -221,11 +224,15 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
     for (int k = 0; k < mine; ++k) {
       const int s = k % p.n_stages;
       if (s % kProducers != j) continue;
+      // Test hook: the first unit of CTA 0 is never loaded (no copy is
+      // issued, so there is nothing to drain); its group's wait runs out.
+      if (p.c.hold_first && blockIdx.x == 0 && k == 0) continue;
       const uint32_t ph = (uint32_t)(k / p.n_stages) & 1u;
       // Lane 0 waits (bounded) and tells the warp; __syncwarp orders the
       // other lanes' copies after the consumers' release it observed.
       int ok = 1;
-      if (lane == 0) ok = mbar_wait(smem_u32(&empty_bar[s]), ph ^ 1u, &s_abort);
+      if (lane == 0)
+        ok = mbar_wait(smem_u32(&empty_bar[s]), ph ^ 1u, &s_abort, p.c.wait_ns);
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (!ok) {
         if (lane == 0) {
@@ -250,8 +257,9 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
       // One warp waits (bounded) and tells the group, so that every warp
       // of the group takes the same branch before the next named barrier.
       if (w == 0) {
-        const bool ok = wait_issued(&issued_k[s], k, &s_abort) &&
-                        mbar_wait(smem_u32(&full_bar[s]), ph, &s_abort);
+        const bool ok =
+            wait_issued(&issued_k[s], k, &s_abort, p.c.wait_ns) &&
+            mbar_wait(smem_u32(&full_bar[s]), ph, &s_abort, p.c.wait_ns);
         if (lane == 0) {
           s_ok[grp] = ok ? 1 : 0;
           if (!ok) {

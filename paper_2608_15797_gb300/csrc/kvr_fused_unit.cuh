@@ -254,7 +254,7 @@ __device__ __forceinline__ void unit_back(const FusedParams &p,
   //    rescale warp v's terms of heads c2 and c2 + 1: exp2(max_v - max) / Z.
   //    Warps with no live row (sum 0) take no part.
   float fv0[U], fv1[U];
-  float Z0;
+  float Z0, Z1;
   if constexpr (U > 1) {
     group_bar(bar_id, 32 * U);
     float4 r[U];
@@ -280,12 +280,17 @@ __device__ __forceinline__ void unit_back(const FusedParams &p,
       fv1[v] *= i1;
     }
     Z0 = S0;  // >= 1: the warp holding the maximum contributes exp2(0)
+    Z1 = S1;
   } else {
     fv0[0] = rcp(f.z0);
     fv1[0] = rcp(f.z1);
     Z0 = f.z0;
+    Z1 = f.z1;
   }
-  if (w == 0 && lane == 0 && !(Z0 > 0.5f && Z0 < INFINITY))
+  // Lanes 0-3 hold the sums of all eight heads (2 each); a NaN or an
+  // infinity in q, k or the scale leaves one of them non-finite.
+  if (w == 0 && lane < 4 &&
+      !(Z0 > 0.5f && Z0 < INFINITY && Z1 > 0.5f && Z1 < INFINITY))
     atomicOr(p.c.err, ERR_NONFINITE);
   float f0 = fv0[0], f1 = fv1[0];
 #pragma unroll

@@ -45,6 +45,9 @@ cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block,
   return cudaLaunchKernelEx(&cfg, kern, static_cast<Args &&>(args)...);
 }
 
+// Default bound of a step kernel's wait on an asynchronous copy (2 s).
+constexpr unsigned long long kDefaultWaitNs = 2000000000ull;
+
 // Device view of one cache: every pointer points into the caller's buffer.
 // A unit u = (s * L + l) * H + h.
 struct CacheView {
@@ -60,6 +63,13 @@ struct CacheView {
   float scale;      // softmax scale (1/sqrt(d) by default)
   int kv_bf16;      // 1: bf16 elements, 0: fp32
   int out_bf16;     // 1: bf16 output, 0: fp32
+  // Bound of the step kernels' waits on this cache's asynchronous copies
+  // (kvr_cache_set_wait_limit; 2 s by default).
+  unsigned long long wait_ns;
+  // Test hook (kvr_cache_set_hold_first_unit): the fused and chunked step
+  // kernels never load the first unit of CTA 0, so its consumers' bounded
+  // wait runs out and the launch ends with ERR_TIMEOUT.
+  int hold_first;
 };
 
 // Work description of one decode call over layers [lb, lb + nl).

@@ -10,7 +10,9 @@
 namespace kvr {
 namespace ptx {
 
-constexpr uint64_t kWaitNs = 2000000000ull;  // bound of every mbarrier wait
+// Default bound of every mbarrier wait; a cache can lower it for the waits
+// on its data (CacheView::wait_ns).  Drains after an abort keep this bound.
+constexpr uint64_t kWaitNs = 2000000000ull;
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -44,13 +46,15 @@ __device__ __forceinline__ uint64_t global_ns() {
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
   return t;
 }
-// Bounded wait; false on timeout or when another warp raised `abort`.
+// Bounded wait (limit_ns); false on timeout or when another warp raised
+// `abort`.
 __device__ inline bool mbar_wait(uint32_t bar, uint32_t parity,
-                          volatile int *abort) {
+                                 volatile int *abort,
+                                 uint64_t limit_ns = kWaitNs) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_ns();
   while (!mbar_try_wait(bar, parity)) {
-    if (*abort || global_ns() - t0 > kWaitNs) return false;
+    if (*abort || global_ns() - t0 > limit_ns) return false;
   }
   return true;
 }

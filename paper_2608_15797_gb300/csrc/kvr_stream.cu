@@ -138,14 +138,19 @@ __global__ void __launch_bounds__(32 * kWarps)
 #pragma unroll
   for (int mt = 0; mt < 8; ++mt) o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.f;
 
+  int failed_at = -1;  // the stage whose wait gave up (CTA-uniform)
   for (int st = 0; st < n_st; ++st) {
     const int buf = st % kStages;
-    if (!mbar_wait(smem_u32(&full_bar[buf]), (uint32_t)(st / kStages) & 1u,
-                   &s_abort)) {
-      if (lane == 0) {
+    const bool got = mbar_wait(smem_u32(&full_bar[buf]),
+                               (uint32_t)(st / kStages) & 1u, &s_abort,
+                               c.wait_ns);
+    // Every thread takes the same branch, so the barriers below match.
+    if (__syncthreads_or(got ? 0 : 1)) {
+      if (tid == 0) {
         atomicOr(c.err, ERR_TIMEOUT);
         s_abort = 1;
       }
+      failed_at = st;
       break;
     }
     unsigned char *K0 = smem + buf * kStageBytes, *K1 = K0 + kRows * 128;
@@ -243,10 +248,12 @@ __global__ void __launch_bounds__(32 * kWarps)
     if (tid == 0 && st + kStages < n_st) issue(st + kStages);
   }
   __syncthreads();
-  if (s_abort) {
+  if (failed_at >= 0) {
+    // Stages failed_at .. failed_at + kStages - 1 (those below n_st) were
+    // issued and not consumed: wait (bounded) for their copies to land.
     if (tid == 0) {
       volatile int never = 0;
-      for (int st = 0; st < n_st; ++st)
+      for (int st = failed_at; st < min(n_st, failed_at + kStages); ++st)
         mbar_wait(smem_u32(&full_bar[st % kStages]), (uint32_t)(st / kStages) & 1u,
                   &never);
     }

@@ -72,6 +72,8 @@ _SIGS = {
     "kvr_cache_lengths": (_S, [_P, _P]),
     "kvr_cache_launch_count": (_S, [_P, _P]),
     "kvr_cache_set_fused": (_S, [_P, _I]),
+    "kvr_cache_set_wait_limit": (_S, [_P, ctypes.c_uint64]),
+    "kvr_cache_set_hold_first_unit": (_S, [_P, _I]),
     "kvr_cache_set_fused_tuning": (_S, [_P, _I, _I]),
     "kvr_cache_set_chunk_tuning": (_S, [_P, _I, _I]),
     "kvr_fork_set_kernel": (_S, [_P, _I]),
@@ -263,7 +265,10 @@ class Cache:
 
     def __init__(self, n_seq, n_layers, n_kv_heads, group, head_dim, capacity,
                  kv_dtype="bf16", out_dtype="bf16", softmax_scale=0.0,
-                 device="cuda", stream=None):
+                 device="cuda", stream=None, buf=None):
+        """buf: an optional caller-owned uint8 device tensor of at least
+        kvr_cache_required_bytes (256-byte aligned); by default one is
+        allocated."""
         self.desc = make_desc(n_seq, n_layers, n_kv_heads, group, head_dim,
                               capacity, kv_dtype, out_dtype, softmax_scale)
         self.S, self.L, self.H, self.G, self.d = (n_seq, n_layers, n_kv_heads,
@@ -273,7 +278,12 @@ class Cache:
         self.nbytes = kvr_cache_required_bytes(self.desc)
         if self.nbytes == 0:
             raise KvrError(KVR_EINVAL, "Cache", "invalid descriptor")
-        self.buf = torch.empty(self.nbytes, dtype=torch.uint8, device=device)
+        if buf is None:
+            buf = torch.empty(self.nbytes, dtype=torch.uint8, device=device)
+        elif buf.numel() < self.nbytes or buf.dtype != torch.uint8:
+            raise ValueError("buf must be uint8 with at least "
+                             f"{self.nbytes} bytes")
+        self.buf = buf
         self.handle = kvr_cache_create(self.desc, self.buf, self.nbytes, stream)
 
     def __del__(self):
@@ -409,6 +419,18 @@ class Cache:
     def set_fused(self, enable: bool):
         kvr_cache_set_fused(self.handle, enable)
 
+    def set_wait_limit(self, ns: int):
+        """Bound of the step kernels' waits on copies (0: the 2 s default)."""
+        _check(lib.kvr_cache_set_wait_limit(self.handle, int(ns)),
+               "kvr_cache_set_wait_limit")
+
+    def set_hold_first_unit(self, enable: bool):
+        """Testing hook: the step kernels' first unit is never loaded, so
+        its bounded wait runs out (kvr_cache_set_hold_first_unit)."""
+        _check(lib.kvr_cache_set_hold_first_unit(self.handle, 1 if enable
+                                                 else 0),
+               "kvr_cache_set_hold_first_unit")
+
     def set_chunk_tuning(self, groups: int, stages: int = 0):
         """groups -1 keeps the chunked kernel off (older per-unit kernels)."""
         kvr_cache_set_chunk_tuning(self.handle, groups, stages)
@@ -478,15 +500,22 @@ class Fork:
     """N candidates of a Cache sharing its live rows (owner of the buffer)."""
 
     def __init__(self, cache: Cache, n_cand: int, tail_cap: int, stream=None,
-                 kernel: int = 0):
+                 kernel: int = 0, buf=None):
         """kernel: 0 the library's choice, 1 candidate-batched, 2 chunked,
-        3 one CTA per unit, 4 generic (kvr_fork_set_kernel)."""
+        3 one CTA per unit, 4 generic (kvr_fork_set_kernel).  buf: an
+        optional caller-owned uint8 device tensor of at least
+        kvr_fork_required_bytes."""
         self.cache, self.N, self.tcap = cache, n_cand, tail_cap
         self.nbytes = kvr_fork_required_bytes(cache.handle, n_cand, tail_cap)
         if self.nbytes == 0:
             raise KvrError(KVR_EINVAL, "Fork", "invalid fork arguments")
-        self.buf = torch.empty(self.nbytes, dtype=torch.uint8,
-                               device=cache.buf.device)
+        if buf is None:
+            buf = torch.empty(self.nbytes, dtype=torch.uint8,
+                              device=cache.buf.device)
+        elif buf.numel() < self.nbytes or buf.dtype != torch.uint8:
+            raise ValueError("buf must be uint8 with at least "
+                             f"{self.nbytes} bytes")
+        self.buf = buf
         self.handle = kvr_fork_candidates(cache.handle, n_cand, tail_cap,
                                           self.buf, self.nbytes, stream)
         if kernel:

@@ -15,6 +15,64 @@ from oracle import parity
 from paper_2608_15797_gb300 import inputs, kvr
 
 
+# Canary guard regions: every device buffer the parity runs hand to the
+# library sits between two GUARD-byte regions filled with CANARY, and the
+# regions are checked after each run, so a write past either end of a
+# caller buffer fails the test that made it.
+GUARD, CANARY = 4096, 0xA5
+
+
+class Guarded:
+    """A uint8 device buffer of nbytes with canary regions on both sides
+    (the buffer keeps the allocation's 256-byte alignment)."""
+
+    def __init__(self, nbytes, device="cuda"):
+        self.raw = torch.full((nbytes + 2 * GUARD,), CANARY, dtype=torch.uint8,
+                              device=device)
+        self.buf = self.raw[GUARD:GUARD + nbytes]
+
+    def intact(self) -> bool:
+        return bool((self.raw[:GUARD] == CANARY).all().item() and
+                    (self.raw[GUARD + self.buf.numel():] == CANARY).all().item())
+
+
+def guarded_tensor(shape, dtype, owner=None, device="cuda"):
+    """An uninitialised tensor inside a Guarded buffer; the guard is kept on
+    `owner._guards` for check_guards."""
+    n = int(np.prod(shape)) * torch.empty((), dtype=dtype).element_size()
+    g = Guarded(n, device)
+    if owner is not None:
+        owner.__dict__.setdefault("_guards", []).append(g)
+    return g.buf.view(dtype).view(*shape)
+
+
+def check_guards(*owners):
+    """Every canary region of the owners' buffers is unchanged."""
+    torch.cuda.synchronize()
+    for o in owners:
+        for g in o.__dict__.get("_guards", []):
+            if not g.intact():
+                raise parity.ParityError("a canary region next to a caller "
+                                         "buffer was overwritten")
+
+
+def guarded_cache(*args, **kw) -> kvr.Cache:
+    """kvr.Cache in a Guarded buffer."""
+    probe = kvr.make_desc(*args[:6], kw.get("kv_dtype", "bf16"),
+                          kw.get("out_dtype", "bf16"))
+    g = Guarded(kvr.kvr_cache_required_bytes(probe))
+    c = kvr.Cache(*args, buf=g.buf, **kw)
+    c._guards = [g]
+    return c
+
+
+def guarded_fork(c: kvr.Cache, n_cand, tail_cap, kernel=0) -> kvr.Fork:
+    g = Guarded(kvr.kvr_fork_required_bytes(c.handle, n_cand, tail_cap))
+    f = kvr.Fork(c, n_cand, tail_cap, kernel=kernel, buf=g.buf)
+    f._guards = [g]
+    return f
+
+
 def dev(x: np.ndarray, dtype: str) -> torch.Tensor:
     """Element-type-exact float32 host values -> device tensor of dtype."""
     return torch.from_numpy(np.ascontiguousarray(x)).to(
@@ -30,8 +88,8 @@ def make_pair(w: inputs.Workload, seed: int, S: int, cap: int,
     With `sample` (a list of sequence indices) the oracle holds only those
     sequences, in that order; the others get device-drawn prompts of the
     same lengths, which no check reads (sequences are independent)."""
-    c = kvr.Cache(S, w.n_layers, w.n_kv_heads, w.group, w.head_dim, cap,
-                  kv_dtype=w.dtype, out_dtype=out_dtype)
+    c = guarded_cache(S, w.n_layers, w.n_kv_heads, w.group, w.head_dim, cap,
+                      kv_dtype=w.dtype, out_dtype=out_dtype)
     c.set_fused(fused)
     c.set_chunk_tuning(*chunk)
     samp = list(range(S)) if sample is None else list(sample)
@@ -69,12 +127,16 @@ def lockstep(c: kvr.Cache, o: orc.OracleCache, w: inputs.Workload, seed: int,
     for t in range(step0, step0 + steps):
         q, kn, vn = inputs.step_inputs(w, seed, t, S, n_layers=le - lb)
         qd, kd, vd = (dev(a, w.dtype) for a in (q, kn, vn))
+        if t == step0:
+            out_buf = guarded_tensor((S, le - lb, c.H * c.G, c.d),
+                                     c.out_torch_dtype, owner=c)
+        out = out_buf
         if not evict:
-            out = c.attend_score(qd, kd, vd, layers=(lb, le))
+            c.attend_score(qd, kd, vd, out=out, layers=(lb, le))
         elif fused:
-            out = c.step(qd, kd, vd, budget, window, layers=(lb, le))
+            c.step(qd, kd, vd, budget, window, out=out, layers=(lb, le))
         else:
-            out = c.attend_score(qd, kd, vd, layers=(lb, le))
+            c.attend_score(qd, kd, vd, out=out, layers=(lb, le))
             c.evict(budget, window, layers=(lb, le))
         ref = o.step(q[samp], kn[samp], vn[samp], evict=False, layer_begin=lb,
                      layer_end=le)
@@ -87,6 +149,7 @@ def lockstep(c: kvr.Cache, o: orc.OracleCache, w: inputs.Workload, seed: int,
         stats.merge(st)
         stats.steps = t - step0 + 1
     c.sync_status()
+    check_guards(c)
     return stats
 
 
@@ -104,14 +167,18 @@ def fork_lockstep(c: kvr.Cache, o: orc.OracleCache, w: inputs.Workload,
     Returns (oracle after commit, chosen, stats)."""
     S = c.S
     parent_pos = [c.export(s, kv=False) for s in range(S)]
-    f = kvr.Fork(c, n_cand, tail_cap or steps, kernel=kernel)
+    f = guarded_fork(c, n_cand, tail_cap or steps, kernel=kernel)
     cands = o.fork(n_cand)
     stats = parity.Stats()
     for t in range(steps):
         per = [inputs.step_inputs(w, seed, 10_000 + t, S, cand=k + 1)
                for k in range(n_cand)]
         Q, K, V = (np.stack([p[i] for p in per]) for i in range(3))
-        out = f.attend_score(dev(Q, w.dtype), dev(K, w.dtype), dev(V, w.dtype))
+        if t == 0:
+            out_buf = guarded_tensor((n_cand, S, c.L, c.H * c.G, c.d),
+                                     c.out_torch_dtype, owner=f)
+        out = f.attend_score(dev(Q, w.dtype), dev(K, w.dtype), dev(V, w.dtype),
+                             out=out_buf)
         torch.cuda.synchronize()
         out = out.float().cpu().numpy()
         for k in range(n_cand):
@@ -153,4 +220,5 @@ def fork_lockstep(c: kvr.Cache, o: orc.OracleCache, w: inputs.Workload,
     exports = [c.export(s, kv=False) for s in range(S)]
     stats.merge(parity.check_and_adopt(committed, exports, budget, window))
     c.sync_status()
+    check_guards(c, f)
     return committed, chosen, stats

@@ -6,9 +6,11 @@ up to 64 terms per thread, its base-2 exponentials (relative error about
 2^-22) and the merges of about 15 partials bound the relative error of
 sum 2^(y - m) and of its weighted twin by about 5e-6, which moves H by at
 most 5e-6 * (1 + H).  The moving mean and the stop position are decided in
-fp32, so they are checked bit for bit against the oracle's float32 decision
-on the kernel's own entropies, and against the fp64 detector wherever the
-mean is not within the tolerance of tau.
+fp32 from those entropies; the mean is checked against the fp64 detector's
+within 2e-5 * (1 + m) + 4e-6 * m, and the stop position against the fp64
+detector's, except for rows whose fp64 mean came within that tolerance of
+tau at a tested position (either decision is correct there).  The number of
+such rows is bounded in every run.
 """
 import json
 import math
@@ -58,18 +60,26 @@ def _sigma_schedule(rows, e):
     return s
 
 
+def _mean_tol(m):
+    # each entropy within _tol, and the kernel's fp32 window sum of at most
+    # 64 of them adds about 64 * 2^-24 relative
+    return 2e-5 * (1.0 + np.abs(m)) + 4e-6 * np.abs(m)
+
+
 def run_lockstep(rows, vocab, steps, dtype="bf16", stride=None, window=12,
                  guard=24, tau=7.0, temperature=1.0, seed=0, offset=None,
                  resets=(), kernel=0):
-    """Drive the kernel and the oracle through `steps` tokens; check every
-    output.  Returns (near_ties, stops)."""
+    """Drive the kernel and the fp64 oracle through `steps` tokens; check
+    every output.  Returns (exempt, stops): the number of rows whose fp64
+    moving mean came within the mean tolerance of tau at a tested position
+    (their stop position is exempt from the comparison from then on, since
+    either decision is correct there), and the kernel's stop positions."""
     det = kvr.EntropyDetector(rows, vocab, window, guard, tau, temperature,
                               dtype)
     det.set_kernel(kernel)
     ref = ent.EntropyDetector(rows, window, guard, tau)
     hist32 = [[] for _ in range(rows)]  # the kernel's entropies, per row
-    stop32 = np.zeros(rows, np.int64)
-    near = 0
+    stop_k = np.zeros(rows, np.int64)
     tied = np.zeros(rows, bool)
     for e in range(steps):
         for (at, b, en) in resets:
@@ -78,7 +88,7 @@ def run_lockstep(rows, vocab, steps, dtype="bf16", stride=None, window=12,
                 ref.reset(b, en)
                 for r in range(b, en):
                     hist32[r] = []
-                    stop32[r] = 0
+                    stop_k[r] = 0
                     tied[r] = False
         x = inputs.candidate_logits(seed, e, rows, vocab,
                                     _sigma_schedule(rows, e), boost=0.0,
@@ -86,42 +96,46 @@ def run_lockstep(rows, vocab, steps, dtype="bf16", stride=None, window=12,
         if offset is not None:
             x = inputs.round_to(x + np.float32(offset), dtype)
         H_ref = ent.token_entropy(x, temperature)
-        live = stop32 == 0
         H, mean, stopped = det.step(_to_dev(x, dtype, stride))
         H = H.cpu().numpy()
         mean = mean.cpu().numpy()
         stopped = stopped.cpu().numpy()
-        # entropy, live rows; stopped rows report NaN and are not read
-        assert np.all(np.isnan(H[~live])) and np.all(np.isnan(mean[~live]))
-        err = np.abs(H[live].astype(np.float64) - H_ref[live])
-        assert np.all(err <= _tol(H_ref[live])), (e, err.max())
-        # fp32 decision on the kernel's own entropies: bit for bit
-        for r in np.nonzero(live)[0]:
+        live_k = stop_k == 0           # rows the kernel ran this token
+        live_ref = ref.stop == 0       # rows the fp64 detector runs
+        # stopped rows report NaN and are not read
+        assert np.all(np.isnan(H[~live_k])) and np.all(np.isnan(mean[~live_k]))
+        err = np.abs(H[live_k].astype(np.float64) - H_ref[live_k])
+        assert np.all(err <= _tol(H_ref[live_k])), (e, err.max())
+        for r in np.nonzero(live_k)[0]:
             hist32[r].append(np.float32(H[r]))
-            m32, fires = ent.decide_fp32(hist32[r], window, guard, tau)
-            assert mean[r] == m32, (e, r, mean[r], m32)
-            if fires:
-                stop32[r] = len(hist32[r])
-        assert np.array_equal(stopped, stop32), (e, stopped, stop32)
-        # fp64 detector on the oracle's entropies, away from ties
-        m64, _ = ref.step(np.where(live, H_ref, 0.0))
-        for r in np.nonzero(live)[0]:
+        # the fp64 detector on the oracle's entropies (Sec. 3.2)
+        m64, _ = ref.step(np.where(live_ref, H_ref, 0.0))
+        for r in np.nonzero(live_k & live_ref & ~tied)[0]:
+            assert abs(mean[r] - m64[r]) <= _mean_tol(m64[r]), \
+                (e, r, mean[r], m64[r])
             if len(ref.hist[r]) > guard and \
-                    abs(m64[r] - tau) <= 2e-5 * (1 + tau):
+                    abs(m64[r] - tau) <= _mean_tol(tau):
                 tied[r] = True
-                near += 1
-        for r in range(rows):
-            if not tied[r]:
-                assert ref.stop[r] == stop32[r], (e, r, ref.stop[r], stop32[r])
+        # the stop position is sticky, and set only at the current position
+        assert np.array_equal(stopped[~live_k], stop_k[~live_k])
+        for r in np.nonzero(live_k)[0]:
+            assert stopped[r] in (0, len(hist32[r])), (e, r, stopped[r])
+        stop_k = stopped.astype(np.int64)
+        for r in np.nonzero(~tied)[0]:
+            assert ref.stop[r] == stop_k[r], (e, r, ref.stop[r], stop_k[r])
     det.sync_status()
     exported = det.export()
-    assert np.array_equal(exported[2], stop32)
+    assert np.array_equal(exported[2], stop_k)
     for r in range(rows):
         n = min(len(hist32[r]), window)
         assert exported[1][r] == len(hist32[r])
         assert np.array_equal(exported[0][r, :n],
                               np.array(hist32[r][-n:] if n else [], np.float32))
-    return near, stop32
+    # Exemptions are rare: at most the quarter of rows the schedule keeps
+    # near tau, plus two.
+    exempt = int(tied.sum())
+    assert exempt <= rows // 4 + 2, exempt
+    return exempt, stop_k
 
 
 KERNELS = {"stream": 1, "pieces": 2}
@@ -131,8 +145,8 @@ KERNELS = {"stream": 1, "pieces": 2}
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])
 @pytest.mark.parametrize("vocab", [7, 1000, 16385, 40000])
 def test_entropy_lockstep_shapes(dtype, vocab, kernel):
-    near, stops = run_lockstep(12, vocab, 40, dtype, kernel=KERNELS[kernel])
-    assert near <= 6
+    exempt, stops = run_lockstep(12, vocab, 40, dtype, kernel=KERNELS[kernel])
+    assert exempt <= 6
 
 
 @pytest.mark.parametrize("kernel", KERNELS)
@@ -145,9 +159,9 @@ def test_entropy_row_counts(rows, kernel):
 @pytest.mark.parametrize("kernel", KERNELS)
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])
 def test_entropy_qwen_vocab(dtype, kernel):
-    near, stops = run_lockstep(16, inputs.VOCAB, 40, dtype,
+    exempt, stops = run_lockstep(16, inputs.VOCAB, 40, dtype,
                                kernel=KERNELS[kernel])
-    assert near <= 8
+    assert exempt <= 8
     # the schedule's incoherent rows stop at the first tested position
     assert all(stops[r] == 25 for r in range(1, 16, 4))
     assert all(stops[r] == 0 for r in range(0, 16, 4))

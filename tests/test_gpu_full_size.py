@@ -8,10 +8,12 @@ launch exactly as a full oracle would; the other sequences run alongside
 with device-drawn inputs that no check reads.
 
 - decode step (Eq. 1 + TopB eviction, Sec. 2.1): 7B geometry, 64 sequences x
-  28 layers x 4 KV heads = 7,168 units a launch, B = 64, W = 8, bf16 in and
-  out.  The first step evicts every unit from its prior context (80-600
-  rows here: the bench's longer prior contexts change only that untimed
-  first step); the steady-state steps run the fused kernel on 73-row units.
+  28 layers x 4 KV heads = 7,168 units a launch, B = 64, 128, 256 and 512,
+  W = 8, bf16 in and out.  The first step evicts every unit from its prior
+  context (B + W + 16 to B + W + 600 rows here: the bench's longer prior
+  contexts change only that untimed first step); the steady-state steps run
+  the fused kernel on 73-row units (B = 64) or the chunked kernel on 137,
+  265 and 521-row units.
 - R-KV step (App. C, lambda = 0.1): the same 64 x 28 x 4 units at B + W = 72
   rows, attend+score then the R-KV eviction, as bench.py --mode rkv.
 - chunk absorb (Algorithm 1's single forward pass over an accepted step): 64
@@ -43,15 +45,25 @@ def _cuda():
     torch.cuda.set_device(0)
 
 
-def test_decode_step_7b_s64_b64_sampled():
-    w = inputs.WORKLOADS["7b_s64_b64"]
-    S = w.n_seq
-    lens = inputs.prior_lengths(61, S, 80, 600)
-    c, o = harness.make_pair(w, 61, S, cap=int(lens.max()) + 1,
+@pytest.mark.parametrize("B", [64, 128, 256, 512])
+def test_decode_step_7b_s64_sampled(B):
+    """The throughput sweep's launches: B = 64 runs the fused kernel on
+    73-row units, B = 128 / 256 / 512 the chunked kernel on 137 / 265 /
+    521-row units; either way 7,168 units a launch over persistent CTAs, so
+    every CTA works through many units and reuses its ring stages."""
+    w = inputs.WORKLOADS[f"7b_s64_b{B}"]
+    S, m = w.n_seq, B + w.window
+    lens = inputs.prior_lengths(61 + B, S, m + 16, m + 600)
+    c, o = harness.make_pair(w, 61 + B, S, cap=int(lens.max()) + 1,
                              prompt_lens=lens, out_dtype="bf16", sample=SAMPLE)
-    st = harness.lockstep(c, o, w, 61, 7, w.budget, w.window, sample=SAMPLE)
+    launches = c.launch_count()
+    st = harness.lockstep(c, o, w, 61 + B, 7, w.budget, w.window,
+                          sample=SAMPLE)
     assert st.units == 7 * len(SAMPLE) * w.n_layers * w.n_kv_heads
-    assert (c.lengths() == w.budget + w.window).all()
+    assert (c.lengths() == m).all()
+    # the first step evicts hundreds of rows (attend+score, then eviction);
+    # the six steady steps are one launch each
+    assert c.launch_count() - launches == 2 + 6
 
 
 def test_rkv_step_7b_s64_b64_sampled():
