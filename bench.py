@@ -61,6 +61,11 @@ def parse():
                    help="shortest prior context (profiling uses a small case)")
     p.add_argument("--prior-max", type=int, default=inputs.PRIOR_LEN_RANGE[1])
     p.add_argument("--e2e-steps", type=int, default=1000)
+    p.add_argument("--repeats", type=int, default=7,
+                   help="the headline's K-step region is timed this many "
+                        "times; value is the median")
+    p.add_argument("--no-rows", action="store_true",
+                   help="skip the other rows' sub-records of the default line")
     p.add_argument("--fused-groups", type=int, default=0,
                    help="units computed at once per SM by the fused kernel "
                         "(0: the library's choice)")
@@ -336,28 +341,33 @@ def run_kvr(args, rank, world, local_rank):
 
     K = args.steps
     # Two events bracket the K steps: an event between launches would stop
-    # a launch from overlapping the tail of the one before it.
+    # a launch from overlapping the tail of the one before it.  The K-step
+    # region is timed `repeats` times (each bracketed by a barrier and a
+    # synchronize on both sides); the value is the median region.
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
     sampler = ClockSampler(local_rank) if rank == 0 else None
     if sampler:
         sampler.start()
-    if world > 1:
-        torch.distributed.barrier()
-    torch.cuda.synchronize()
-    launches0 = cache.launch_count()
+    regions, launches = [], 0
     t_begin = time.time()
-    t0.record(stream)
-    for i in range(K):
-        step(i)
-    t1.record(stream)
-    torch.cuda.synchronize()
+    for rep in range(max(1, args.repeats)):
+        if world > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize()
+        launches0 = cache.launch_count()
+        t0.record(stream)
+        for i in range(K):
+            step(rep * K + i)
+        t1.record(stream)
+        torch.cuda.synchronize()
+        launches = cache.launch_count() - launches0
+        if world > 1:
+            torch.distributed.barrier()
+        regions.append(max_over_ranks(t0.elapsed_time(t1), dev))
     t_end = time.time()
-    launches = cache.launch_count() - launches0
-    if world > 1:
-        torch.distributed.barrier()
     clocks = sampler.stop(t_begin, t_end) if sampler else None
-    total_ms = t0.elapsed_time(t1)
+    total_ms = float(np.median(regions))
     # One launch per steady-state step: the average launch duration is the
     # region's time over its launches (gaps between launches included).
     per_launch_ms = total_ms / max(1, launches)
@@ -388,8 +398,6 @@ def run_kvr(args, rank, world, local_rank):
     per_layer_ms = t0.elapsed_time(t1) / Kl
     cache.sync_status()
     del lpool, lout
-
-    total_ms = max_over_ranks(total_ms, dev)
 
     # End to end through the public call with HOST buffers
     # (kvr_decode_step_host): every step's inputs copied in from pinned host
@@ -440,7 +448,7 @@ def run_kvr(args, rank, world, local_rank):
     unit_bytes = cost_model.step_unit_bytes(B + W, d, G, 2, 2, B, W)
     launch_bytes = unit_bytes * S * L * H
     return dict(total_ms=total_ms, per_launch_ms=per_launch_ms, K=K,
-                per_layer_ms=per_layer_ms, Kl=Kl,
+                regions=regions, per_layer_ms=per_layer_ms, Kl=Kl,
                 first_ms=first_ms, clocks=clocks, e2e_ms=e2e_ms, Ke=Ke,
                 e2e_serial_ms=e2e_serial_ms,
                 bi=bi, bo=bo, launch_bytes=launch_bytes, lens=lens,
@@ -1033,6 +1041,149 @@ def run_fork_copy(args):
                 kernel="kvr_decode_step over the candidate sequences")
 
 
+def run_sweep_row(args, B):
+    """The throughput sweep at budget B (7B geometry, 64 sequences, W=8):
+    the same measurement as the headline's value (one kvr_decode_step over
+    all 28 layers a step, median of `repeats` K-step regions), without the
+    end-to-end and per-layer legs."""
+    import torch
+    from paper_2608_15797_gb300 import kvr
+    w = inputs.WORKLOADS[f"7b_s64_b{B}"]
+    S, L, H, G, d, W = (w.n_seq, w.n_layers, w.n_kv_heads, w.group,
+                        w.head_dim, w.window)
+    dev = torch.device("cuda", 0)
+    lo = max(args.prior_min, B + W + 1)
+    lens = inputs.prior_lengths(args.seed + B, S, lo, max(lo, args.prior_max))
+    cache = kvr.Cache(S, L, H, G, d, int(lens.max()) + 1, "bf16", "bf16",
+                      device=dev)
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(args.seed + 3 * B)
+    for s in range(S):
+        n = int(lens[s])
+        k = (torch.randn(L, H, n, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+        v = (torch.randn(L, H, n, d, generator=gen, device=dev) * w.sigma).to(torch.bfloat16)
+        cache.load(s, k, v)
+        del k, v
+    pool = [tuple((torch.randn(*shp, generator=gen, device=dev) * w.sigma)
+                  .to(torch.bfloat16) for shp in ((S, L, H * G, d),
+                                                  (S, L, H, d), (S, L, H, d)))
+            for _ in range(8)]
+    out = torch.empty(S, L, H * G, d, dtype=torch.bfloat16, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step(i):
+        kvr.kvr_decode_step(cache.handle, 0, L, *pool[i % 8], out, B, W,
+                            stream)
+
+    step(0)  # the first step evicts every unit to B + W
+    torch.cuda.synchronize()
+    assert (cache.lengths() == B + W).all()
+    for i in range(max(3, args.warmup)):
+        step(i)
+    K = args.steps
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    regions, launches = [], 0
+    for rep in range(max(1, args.repeats)):
+        torch.cuda.synchronize()
+        n0 = cache.launch_count()
+        t0.record(stream)
+        for i in range(K):
+            step(rep * K + i)
+        t1.record(stream)
+        torch.cuda.synchronize()
+        launches = cache.launch_count() - n0
+        regions.append(t0.elapsed_time(t1))
+    cache.sync_status()
+    total = float(np.median(regions))
+    unit_bytes = cost_model.step_unit_bytes(B + W, d, G, 2, 2, B, W)
+    return dict(metric=metric_name(w), total_ms=total, per_ms=total / K, K=K,
+                launches=launches, launch_bytes=unit_bytes * S * L * H,
+                regions=regions,
+                config={"workload": f"7b_s64_b{B}", "budget": B, "window": W,
+                        "prior_len": f"U[{lo},{max(lo, args.prior_max)}]"},
+                kernel="kvr_decode_step (chunked kernel, one launch a step)")
+
+
+def row_record(r, unit, peak, peak_kind, value=None):
+    """A compact sub-record of the default line for one row's result."""
+    achieved = r["launch_bytes"] / (r["per_ms"] / 1e3) / 1e9
+    rec = {"metric": r["metric"],
+           "value": value if value is not None else r["K"] / (r["total_ms"] / 1e3),
+           "unit": unit, "steps": r["K"],
+           "ms_per_step": r["total_ms"] / r["K"], "config": r.get("config"),
+           "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak,
+                        "unit": "GB/s", "frac": achieved / peak,
+                        "peak_kind": peak_kind,
+                        "algorithmic_bytes_per_launch": r["launch_bytes"],
+                        "launch_ms": r["per_ms"], "kernel": r.get("kernel")},
+           "gpu_launches": r["launches"]}
+    if "regions" in r:
+        rec["regions_ms"] = [round(x, 5) for x in r["regions"]]
+    for key in ("commit_ms", "fork_ms", "score_ms", "amortized_steps_per_s"):
+        if key in r:
+            rec[key] = r[key]
+    return rec
+
+
+def sub_records(args):
+    """The other rows, each a few milliseconds of timed region at its
+    benchmarked size: the B = 128/256/512 sweep, the 72B candidate step and
+    its commit, the paper's candidates-by-copy mode, chunk absorb, the R-KV
+    step, the entropy test and the full-context helper."""
+    import copy
+    import torch
+    peaks, peak_kind = measured_peaks()
+    peak = float(peaks["hbm_gbs"])
+    a = copy.copy(args)
+    a.warmup = max(3, min(args.warmup, 10))
+    a.steps = max(8, min(args.steps, 64))
+    a.repeats = max(1, min(args.repeats, 5))
+    a.seqs = 0
+    out = {}
+    torch.cuda.empty_cache()
+
+    def run(name, fn, unit, **kw):
+        try:
+            out[name] = row_record(fn(), unit, peak, peak_kind, **kw)
+        except Exception as e:  # reported, never silent
+            out[name] = {"error": f"{type(e).__name__}: {e}"}
+        torch.cuda.synchronize()
+        torch.cuda.empty_cache()
+
+    for B in (128, 256, 512):
+        run(f"sweep_b{B}", lambda B=B: run_sweep_row(a, B), "steps/s")
+    run("candidates_72b_bon8", lambda: run_fork(a), "candidate tokens/s")
+    run("candidates_by_copy_72b_bon8", lambda: run_fork_copy(a),
+        "candidate tokens/s")
+    a_abs = copy.copy(a)
+    a_abs.absorb_kernel = 0
+    r_abs = {}
+
+    def absorb():
+        r = run_absorb(a_abs)
+        r.update(metric="absorbed 64-token steps/s (7B, B=64, W=8, 64 "
+                        "sequences x 28 layers a call)",
+                 kernel="kvr_absorb_chunk (absorb_tc_kernel, tcgen05)",
+                 config={"workload": "7b absorb", "chunk": r["C"]})
+        r_abs.update(r)
+        return r
+    run("absorb_7b_c64", absorb, "calls/s")
+    run("rkv_7b_b64", lambda: run_rkv(a), "steps/s")
+
+    def entropy():
+        r = run_entropy(a)
+        r.update(metric=f"candidate rows screened/s by the entropy test "
+                        f"({r['rows']} rows x {r['V']} {r['dtype']} logits a "
+                        f"launch)",
+                 kernel="kvr_entropy_step (entropy_stream_kernel)",
+                 config={"rows": r["rows"], "vocab": r["V"]})
+        return r
+    run("entropy_512x152064", entropy, "launches/s")
+    run("helper_1p5b_16k", lambda: run_helper(a), "steps/s")
+    return out
+
+
 def print_row_line(args, r):
     peaks, peak_kind = measured_peaks()
     peak = float(peaks["hbm_gbs"])
@@ -1285,7 +1436,13 @@ def main():
         "latency_1seq": lat,
         "clocks": r["clocks"],
         "cpu_baseline": cpu,
+        "timing": {"regions_ms": [round(x, 5) for x in r["regions"]],
+                   "value_from": "median of the K-step regions",
+                   "spread": (max(r["regions"]) - min(r["regions"])) /
+                             float(np.median(r["regions"]))},
     }
+    if world == 1 and not args.no_rows:
+        line["rows"] = sub_records(args)
     print(json.dumps(line))
     if world > 1:
         torch.distributed.destroy_process_group()
