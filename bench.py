@@ -4,8 +4,10 @@ Workload (default): Qwen2.5-Math-7B decode geometry (28 layers, 28 query /
 4 KV heads, head_dim 128, bf16), a batch of 64 independent sequences with
 prior context lengths drawn uniformly from [512, 16384], budget B=64 and
 recent window W=8.  The prompts are loaded with zero scores; the first decode
-step evicts each unit down to B+W (timed separately as `first_step_ms`);
-after that every step is the steady state: append, attend over B+W+1 rows,
+step evicts each unit down to B+W (timed separately as `first_step_ms`); the
+sequences then move into a steady-state cache of capacity B+W+1 (a dense
+slab; `kvr_cache_copy_sequences`, timed as `move_to_steady_cache_ms`), and
+every step after that is the steady state: append, attend over B+W+1 rows,
 accumulate scores, evict one row per (sequence, layer, KV head).
 
 One "step" = one decode token for all 64 sequences and all 28 layers, run as
@@ -330,6 +332,28 @@ def run_kvr(args, rank, world, local_rank):
     first_ms = ev0.elapsed_time(ev1)
     cache.sync_status()
     assert (cache.lengths() == B + W).all()
+    # The prompt-sized cache (capacity max prior + 1, a 4 MB unit stride at
+    # 16k) served only the first eviction: every sequence moves into a
+    # steady-state cache of capacity B + W + 1, a dense slab, through the
+    # library's sequence copy, and the timed steps run there.
+    steady = kvr.Cache(S, L, H, G, d, B + W + 1, kv_dtype="bf16",
+                       out_dtype="bf16", device=dev)
+    if args.fused_groups or args.fused_group_warps:
+        kvr.kvr_cache_set_fused_tuning(steady.handle, args.fused_groups,
+                                       args.fused_group_warps)
+    if args.chunk_groups or args.chunk_stages:
+        kvr.kvr_cache_set_chunk_tuning(steady.handle, args.chunk_groups,
+                                       args.chunk_stages)
+    ev0.record(stream)
+    steady.copy_from(cache, np.arange(S, dtype=np.int32),
+                     np.arange(S, dtype=np.int32), stream)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    move_ms = ev0.elapsed_time(ev1)
+    del cache
+    torch.cuda.empty_cache()
+    cache = steady
+    cache.sync_status()
 
     def step(i):
         q, kn, vn = pool[i % n_pool]
@@ -449,7 +473,8 @@ def run_kvr(args, rank, world, local_rank):
     launch_bytes = unit_bytes * S * L * H
     return dict(total_ms=total_ms, per_launch_ms=per_launch_ms, K=K,
                 regions=regions, per_layer_ms=per_layer_ms, Kl=Kl,
-                first_ms=first_ms, clocks=clocks, e2e_ms=e2e_ms, Ke=Ke,
+                first_ms=first_ms, move_ms=move_ms, clocks=clocks,
+                e2e_ms=e2e_ms, Ke=Ke,
                 e2e_serial_ms=e2e_serial_ms,
                 bi=bi, bo=bo, launch_bytes=launch_bytes, lens=lens,
                 launches=launches)
@@ -625,7 +650,12 @@ def run_crossover(args):
         # mean rows attended over the timed calls
         full.append((ell + Wm + (K + 1) / 2.0, t))
         del cache, ws
-    evict = {}
+    # Two evictors at each B' = B + W: the accumulated-attention step (one
+    # fused kvr_decode_step) and the paper's R-KV eviction (App. C, lambda
+    # 0.1, kvr_decode_step_rkv with its key-similarity pass: one launch at
+    # B' = 72, attend+score then kvr_evict_compact_rkv at B' = 640), both
+    # from a cache already at B + W rows.
+    evict, evict_rkv = {}, {}
     for B, Wn in ((64, 8), (512, 128)):
         cache = loaded(B + Wn, B + Wn + 1)
         t = timed(lambda: kvr.kvr_decode_step(cache.handle, 0, L, q, kn, vn, out,
@@ -633,29 +663,40 @@ def run_crossover(args):
         cache.sync_status()
         evict[B + Wn] = t
         del cache
+        cache = loaded(B + Wn, B + Wn + 1)
+
+        def rkv_step():
+            kvr.kvr_decode_step_rkv(cache.handle, 0, L, q, kn, vn, out, B, Wn,
+                                    0.1, stream)
+        evict_rkv[B + Wn] = timed(rkv_step)
+        cache.sync_status()
+        del cache
     ls = np.array([x for x, _ in full])
     ts = np.array([y for _, y in full])
     fit = ls >= 512  # the bandwidth-bound part of the curve
     b, a = np.polyfit(ls[fit], ts[fit], 1)
-    res = {}
-    for bp, te in evict.items():
-        t_bp = float(np.interp(bp, ls, ts))
-        # first context at which full attention costs as much as the step
-        above = np.nonzero(ts >= te)[0]
-        if len(above) and above[0] > 0:
-            i = above[0]
-            lstar = float(ls[i - 1] + (te - ts[i - 1]) * (ls[i] - ls[i - 1]) /
-                          (ts[i] - ts[i - 1]))
-        elif len(above):
-            lstar = float(ls[0])
-        else:
-            lstar = float((te - a) / b)
-        res[bp] = {"t_evict_us": te, "t_full_at_Bphys_us": t_bp,
-                   "alpha": te / t_bp - 1.0, "lstar_rows": lstar,
-                   "lstar_over_Bphys": lstar / bp}
+
+    def crossover(ev):
+        res = {}
+        for bp, te in ev.items():
+            t_bp = float(np.interp(bp, ls, ts))
+            # first context at which full attention costs as much as the step
+            above = np.nonzero(ts >= te)[0]
+            if len(above) and above[0] > 0:
+                i = above[0]
+                lstar = float(ls[i - 1] + (te - ts[i - 1]) *
+                              (ls[i] - ls[i - 1]) / (ts[i] - ts[i - 1]))
+            elif len(above):
+                lstar = float(ls[0])
+            else:
+                lstar = float((te - a) / b)
+            res[bp] = {"t_evict_us": te, "t_full_at_Bphys_us": t_bp,
+                       "alpha": te / t_bp - 1.0, "lstar_rows": lstar,
+                       "lstar_over_Bphys": lstar / bp}
+        return res
     return dict(full=[{"context": float(x), "us_per_step": float(y)} for x, y in full],
-                fit={"a_us": float(a), "b_us_per_row": float(b)}, res=res, S=S,
-                K=K)
+                fit={"a_us": float(a), "b_us_per_row": float(b)},
+                res=crossover(evict), res_rkv=crossover(evict_rkv), S=S, K=K)
 
 
 def run_absorb(args):
@@ -912,6 +953,11 @@ def run_rkv(args):
 
     def rkv_step(i):
         q, kn, vn = pool[i % 8]
+        kvr.kvr_decode_step_rkv(cache.handle, 0, L, q, kn, vn, out, B, Wn,
+                                lam, stream)
+
+    def rkv_two_launches(i):
+        q, kn, vn = pool[i % 8]
         kvr.kvr_decode_attend_score(cache.handle, 0, L, q, kn, vn, out, stream)
         kvr.kvr_evict_compact_rkv(cache.handle, 0, L, B, Wn, lam, stream)
 
@@ -935,25 +981,26 @@ def run_rkv(args):
     K = args.steps
     n0 = cache.launch_count()
     rkv_ms = timed(rkv_step, K)
-    launches = cache.launch_count() - n0 - 2 * max(3, args.warmup)
+    launches = cache.launch_count() - n0 - max(3, args.warmup)
     score_ms = timed(score_step, K)
+    two_ms = timed(rkv_two_launches, K)
     cache.sync_status()
-    n = B + Wn + 1
+    # One pass: the step's bytes (the key-similarity pass reads the keys
+    # already staged for attention).
     attend = cost_model.step_unit_bytes(B + Wn, d, G, 2, 2, B, Wn)
-    # R-KV eviction: every key once, scores and positions, one row moved
-    evict = n * d * 2 + 8 * n + 2 * 2 * d * 2 + 8 + 16
     units = S * L * H
     return dict(total_ms=rkv_ms, per_ms=rkv_ms / K, K=K, launches=launches,
-                launch_bytes=(attend + evict) * units,
-                score_ms=score_ms / K,
+                launch_bytes=attend * units,
+                score_ms=score_ms / K, two_launch_ms=two_ms / K,
                 metric=f"evicted decode steps/s with R-KV eviction at 7B "
                        f"geometry, B={B}, W={Wn}, lambda={lam} ({S} sequences"
                        f" x {L} layers per step)",
                 config={"workload": "7b_s64_b64 R-KV", "n_seq": S, "layers": L,
                         "kv_heads": H, "group": G, "head_dim": d, "budget": B,
                         "window": Wn, "lambda": lam},
-                kernel="kvr_decode_attend_score + kvr_evict_compact_rkv "
-                       "(bytes: the step's and one more read of every key)")
+                kernel="kvr_decode_step_rkv (one launch: attention, scores "
+                       "and the R-KV key-similarity pass over the staged "
+                       "keys, selection, compaction)")
 
 
 def run_fork_copy(args):
@@ -1078,6 +1125,13 @@ def run_sweep_row(args, B):
     step(0)  # the first step evicts every unit to B + W
     torch.cuda.synchronize()
     assert (cache.lengths() == B + W).all()
+    steady = kvr.Cache(S, L, H, G, d, B + W + 1, "bf16", "bf16", device=dev)
+    steady.copy_from(cache, np.arange(S, dtype=np.int32),
+                     np.arange(S, dtype=np.int32), stream)
+    torch.cuda.synchronize()
+    del cache
+    torch.cuda.empty_cache()
+    cache = steady
     for i in range(max(3, args.warmup)):
         step(i)
     K = args.steps
@@ -1101,7 +1155,8 @@ def run_sweep_row(args, B):
                 launches=launches, launch_bytes=unit_bytes * S * L * H,
                 regions=regions,
                 config={"workload": f"7b_s64_b{B}", "budget": B, "window": W,
-                        "prior_len": f"U[{lo},{max(lo, args.prior_max)}]"},
+                        "prior_len": f"U[{lo},{max(lo, args.prior_max)}]",
+                        "steady_capacity": B + W + 1},
                 kernel="kvr_decode_step (chunked kernel, one launch a step)")
 
 
@@ -1120,7 +1175,8 @@ def row_record(r, unit, peak, peak_kind, value=None):
            "gpu_launches": r["launches"]}
     if "regions" in r:
         rec["regions_ms"] = [round(x, 5) for x in r["regions"]]
-    for key in ("commit_ms", "fork_ms", "score_ms", "amortized_steps_per_s"):
+    for key in ("commit_ms", "fork_ms", "score_ms", "amortized_steps_per_s",
+                "two_launch_ms"):
         if key in r:
             rec[key] = r[key]
     return rec
@@ -1200,7 +1256,8 @@ def print_row_line(args, r):
                          "algorithmic_bytes_per_launch": r["launch_bytes"],
                          "launch_ms": r["per_ms"], "kernel": r["kernel"]},
             "gpu_launches": r["launches"]}
-    for key in ("commit_ms", "fork_ms", "amortized_steps_per_s", "score_ms"):
+    for key in ("commit_ms", "fork_ms", "amortized_steps_per_s", "score_ms",
+                "two_launch_ms"):
         if key in r:
             line[key] = r[key]
     if "fork_bytes" in r:
@@ -1258,7 +1315,12 @@ def main():
                            "layers": 28, "kv_heads": 4, "group": 7,
                            "head_dim": 128},
                 "alpha_640": r640["alpha"], "crossover_72": r72,
-                "crossover_640": r640, "full_context": r["full"],
+                "crossover_640": r640,
+                "rkv": {"evictor": "R-KV, lambda 0.1 (kvr_decode_step_rkv)",
+                        "alpha_640": r["res_rkv"][640]["alpha"],
+                        "crossover_640": r["res_rkv"][640],
+                        "crossover_72": r["res_rkv"][72]},
+                "full_context": r["full"],
                 "fit": r["fit"],
                 "paper": {"lstar_rows": 2500, "alpha": 2.9, "B_phys": 640,
                           "note": "the paper's measurement on its own "
@@ -1399,6 +1461,7 @@ def main():
                    "group": w.group, "head_dim": w.head_dim,
                    "budget": w.budget, "window": w.window,
                    "prior_len": f"U[{args.prior_min},{args.prior_max}]",
+                   "steady_capacity": w.budget + w.window + 1,
                    "elem": "bf16",
                    "l2": f"inputs larger than L2: {r['launch_bytes'] / 1e6:.0f} MB"
                          " touched per step, no flush",
@@ -1406,6 +1469,7 @@ def main():
         "hbm_gbs": achieved,
         "hbm_frac_of_8tbs": achieved / NOMINAL_HBM_GBS,
         "first_step_ms": r["first_ms"],
+        "move_to_steady_cache_ms": r["move_ms"],
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak,
                      "unit": "GB/s", "frac": achieved / peak,
                      "peak_kind": peak_kind,

@@ -145,6 +145,21 @@ kvr_status kvr_decode_step(kvr_cache *cache, int layer_begin, int layer_end,
                            const void *q, const void *k_new, const void *v_new,
                            void *out, int budget, int window, void *stream);
 
+/* Steps 1-4 with the R-KV eviction in one pass (App. C, lambda; App. D:
+ * the eviction's key-similarity pass): equivalent to
+ * kvr_decode_attend_score followed by kvr_evict_compact_rkv with the same
+ * reading of R-KV.  Where every unit holds at most 128 rows after the
+ * append and at most one is evicted (bf16, head_dim 128, G <= 8) it is one
+ * launch: the redundancy of each row comes from the keys already staged
+ * for attention, so no key is read twice; otherwise it runs the two calls.
+ * Arguments as kvr_decode_step, plus 0 <= lambda <= 1 (KVR_EINVAL
+ * otherwise). */
+kvr_status kvr_decode_step_rkv(kvr_cache *cache, int layer_begin,
+                               int layer_end, const void *q,
+                               const void *k_new, const void *v_new, void *out,
+                               int budget, int window, float lambda,
+                               void *stream);
+
 /* kvr_decode_step with the step's inputs and output in HOST memory, as a
  * serving loop feeds it (Sec. 2.1 Eq. 1, one decode step of every sequence).
  * Enqueued on stream, in order: the copies of q_host, k_new_host and
@@ -507,7 +522,9 @@ kvr_status kvr_cache_export(const kvr_cache *cache, int seq, void *host_k,
  *   score  [S][L][H][row_stride] fp32: the accumulated importance score of
  *          the row in each slot (Sec. 2.1)
  *   pos    [S][L][H][row_stride] int32: the row's position (token index)
- *   state  [S][L][H][4] int32: live length, next position, 0, 0
+ *   state  [S][L][H][4] int32: live length, next position, 1 while the
+ *          library holds a current sum of the unit's normalised keys for
+ *          kvr_decode_step_rkv (else 0), 0
  * Slots [0, live length) of a unit hold its rows, in no particular order.
  * The values are those after the last call enqueued on the cache's stream;
  * read them stream-ordered.  Any output pointer may be NULL. */

@@ -240,6 +240,7 @@ __device__ void finish_unit(const AbsorbParams &p, const Unit &u,
   if (tid == 0) {
     c.state[4 * u.ug] = nk;
     c.state[4 * u.ug + 1] = u.t0 + C;
+    c.state[4 * u.ug + 2] = 0;  // the R-KV key sum no longer matches
   }
 }
 

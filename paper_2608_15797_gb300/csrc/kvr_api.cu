@@ -60,7 +60,7 @@ bool desc_ok(const kvr_cache_desc *d) {
 
 // Byte offsets of every array inside the cache buffer.
 struct Layout {
-  size_t K, V, score, pos, state, err, logits, total;
+  size_t K, V, score, pos, state, err, logits, rsum, total;
 };
 
 Layout layout_of(const kvr_cache_desc *d) {
@@ -83,6 +83,8 @@ Layout layout_of(const kvr_cache_desc *d) {
   off = align_up(off + 16);
   l.logits = off;
   off = align_up(off + rows * d->group * sizeof(float));
+  l.rsum = off;
+  off = align_up(off + units * (size_t)d->head_dim * sizeof(float));
   l.total = off;
   return l;
 }
@@ -282,7 +284,8 @@ const std::pair<CUtensorMap, CUtensorMap> *slab_maps(kvr_cache *c,
 }
 
 bool try_fused(kvr_cache *c, const StepArgs &a, bool evict, int budget,
-               int window, cudaStream_t stream, cudaError_t *err) {
+               int window, cudaStream_t stream, cudaError_t *err,
+               bool rkv = false, float lam = 0.f) {
   const CacheView &v = c->view;
   if (!c->fused || !v.kv_bf16 || v.d != 128 || v.G > 8) return false;
   if (a.max_rows > 128) return false;
@@ -298,8 +301,8 @@ bool try_fused(kvr_cache *c, const StepArgs &a, bool evict, int budget,
   const int Rb = std::max(8, (a.max_rows - 1 + 7) / 8 * 8);
   const int U = kvr::fused_group_warps(R, c->fused_group_warps);
   if (U < 1) return false;
-  const int stage = kvr::fused_stage_bytes(R);
-  const int gbytes = kvr::fused_group_bytes(U);
+  const int stage = kvr::fused_stage_bytes(R, rkv);
+  const int gbytes = kvr::fused_group_bytes(U, rkv);
   const int avail = c->smem_optin - 1024 /*alignment*/ - 512 /*static*/;
   // Consumer groups hold a stage only while reading it; the rest of shared
   // memory is ring.  By default as many groups as there are stages (at most
@@ -335,6 +338,8 @@ bool try_fused(kvr_cache *c, const StepArgs &a, bool evict, int budget,
   p.evict = evict ? 1 : 0;
   p.scale_log2e = v.scale * 1.4426950408889634f;
   p.inv_g = 1.f / (float)v.G;
+  p.rkv = rkv ? 1 : 0;
+  p.lam = lam;
   const int units = v.S * a.nl * v.H;
   const int grid = std::min(c->sm_count, units);
   *err = kvr::launch_fused_step(maps->first, maps->second, p, grid,
@@ -543,6 +548,7 @@ kvr_status kvr_cache_create(const kvr_cache_desc *desc, void *dev_buf,
   v.state = reinterpret_cast<int32_t *>(b + lay.state);
   v.err = reinterpret_cast<unsigned *>(b + lay.err);
   v.logits = reinterpret_cast<float *>(b + lay.logits);
+  v.rsum = reinterpret_cast<float *>(b + lay.rsum);
   v.S = desc->n_seq;
   v.L = desc->n_layers;
   v.H = desc->n_kv_heads;
@@ -884,6 +890,31 @@ kvr_status kvr_decode_step(kvr_cache *c, int lb, int le, const void *q,
   return kvr_evict_compact(c, lb, le, budget, window, stream);
 }
 
+kvr_status kvr_decode_step_rkv(kvr_cache *c, int lb, int le, const void *q,
+                               const void *k_new, const void *v_new,
+                               void *out, int budget, int window, float lambda,
+                               void *stream) {
+  kvr_status st = check_step(c, lb, le, q, k_new, v_new, out);
+  if (st != KVR_OK) return st;
+  st = check_evict(budget, window);
+  if (st != KVR_OK) return st;
+  if (!(lambda >= 0.f && lambda <= 1.f))
+    return fail(KVR_EINVAL, "mix weight %g outside [0, 1]", (double)lambda);
+  StepArgs a = step_args(c, lb, le, q, k_new, v_new, out);
+  cudaError_t e = cudaSuccess;
+  if (try_fused(c, a, true, budget, window, as_stream(stream), &e, true,
+                lambda)) {
+    if (e != cudaSuccess) return cuda_fail("kvr_decode_step_rkv", e);
+    c->launches += 1;
+    mirror_append(c, lb, le);
+    mirror_evict(c, lb, le, budget, window);
+    return KVR_OK;
+  }
+  st = kvr_decode_attend_score(c, lb, le, q, k_new, v_new, out, stream);
+  if (st != KVR_OK) return st;
+  return kvr_evict_compact_rkv(c, lb, le, budget, window, lambda, stream);
+}
+
 kvr_status kvr_decode_step_host(kvr_cache *c, int lb, int le,
                                 const void *q_host, const void *k_new_host,
                                 const void *v_new_host, void *out_host,
@@ -1033,6 +1064,7 @@ kvr_status kvr_cache_import(kvr_cache *c, int seq, const void *host_k,
     for (size_t i = 0; i < units; ++i) {
       st[4 * i] = host_len[i];
       st[4 * i + 1] = host_next_pos[i];
+      st[4 * i + 2] = 0;  // no R-KV key sum for the imported rows
     }
     e = cudaMemcpy(v.state + seq * units * 4, st.data(),
                    st.size() * sizeof(int32_t), cudaMemcpyHostToDevice);

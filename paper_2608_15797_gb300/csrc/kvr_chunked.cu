@@ -686,6 +686,7 @@ __global__ void __launch_bounds__(kMaxGroups * (kU + 1) * 32, 1)
           if (lane == 0) {
             c.state[4 * jb.ug] = victim < 0 ? m + 1 : m;
             c.state[4 * jb.ug + 1] = t + 1;
+            c.state[4 * jb.ug + 2] = 0;  // R-KV key sum no longer valid
           }
         }
       }

@@ -59,7 +59,11 @@ __global__ void __launch_bounds__(kThreads)
     dst.score[ud * dst.sstride + r] = src.score[us * src.sstride + r];
     dst.pos[ud * dst.sstride + r] = src.pos[us * src.sstride + r];
   }
-  if (threadIdx.x < 4) dst.state[4 * ud + threadIdx.x] = src.state[4 * us + threadIdx.x];
+  // Length and next position; the R-KV key sum is not copied, so the
+  // copy's is marked stale.
+  if (threadIdx.x < 4)
+    dst.state[4 * ud + threadIdx.x] =
+        threadIdx.x == 2 ? 0 : src.state[4 * us + threadIdx.x];
 }
 
 }  // namespace

@@ -71,6 +71,18 @@ __device__ int block_collect(int lo, int hi, Pred pred, int *list,
   return total;
 }
 
+// A float's order as an unsigned integer, negative values included.
+__device__ __forceinline__ unsigned ord_bits(float z) {
+  const unsigned b = __float_as_uint(z);
+  return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+
+// R-KV key: higher z first, then lower position.
+__device__ __forceinline__ unsigned long long rkv_key(float z, int32_t p) {
+  return (static_cast<unsigned long long>(ord_bits(z)) << 32) |
+         static_cast<unsigned long long>(0xFFFFFFFFu - static_cast<unsigned>(p));
+}
+
 // TopB key: higher score first, then lower position (scores are >= 0, so
 // their IEEE bit patterns order like the values).
 __device__ __forceinline__ unsigned long long rank_key(float s, int32_t p) {

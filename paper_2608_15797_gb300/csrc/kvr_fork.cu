@@ -307,6 +307,7 @@ __global__ void __launch_bounds__(kThreads)
   if (tid == 0) {
     c.state[4 * x.u] = nk;
     c.state[4 * x.u + 1] = base_pos + nt;
+    c.state[4 * x.u + 2] = 0;  // the R-KV key sum no longer matches
   }
 }
 

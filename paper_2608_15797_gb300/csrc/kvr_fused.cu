@@ -46,6 +46,7 @@
 #include <cuda_bf16.h>
 #include <stdint.h>
 
+#include "kvr_device.cuh"
 #include "kvr_internal.h"
 #include "kvr_ptx.cuh"
 
@@ -66,9 +67,11 @@ __device__ __forceinline__ void group_bar(int id, int threads) {
 
 // Byte offsets inside one stage of R staged rows (R a multiple of 16, so
 // every box starts on a 1024-byte boundary as the 128B swizzle needs).
+// The R-KV step also stages the unit's kept sum of normalised keys (rs,
+// 128 fp32).
 struct StageLayout {
-  uint32_t k0, k1, v0, v1, q, kn, vn, sc, ps, st, bytes;
-  __host__ __device__ explicit StageLayout(int R) {
+  uint32_t k0, k1, v0, v1, q, kn, vn, sc, ps, st, rs, bytes;
+  __host__ __device__ explicit StageLayout(int R, bool rkv = false) {
     k0 = 0;
     k1 = k0 + R * 128;
     v0 = k1 + R * 128;
@@ -79,19 +82,24 @@ struct StageLayout {
     sc = vn + 256;
     ps = sc + 4 * R;
     st = ps + 4 * R;
-    bytes = ((st + 16) + 1023) / 1024 * 1024;
+    rs = st + 16;
+    bytes = ((rs + (rkv ? 512 : 0)) + 1023) / 1024 * 1024;
   }
 };
 
 // Byte offsets inside one consumer group's private exchange area (after the
-// ring): five 16-byte slots per warp, then the warps' partial outputs
-// ([warp][8 head-dim tiles][32 lanes] float4).  A one-warp group needs none.
+// ring): kSlots 16-byte slots per warp (five; six for the R-KV step), then
+// the warps' partial outputs ([warp][8 head-dim tiles][32 lanes] float4).
+// A one-warp group needs none.
 struct GroupLayout {
-  uint32_t xs, ox, bytes;
-  __host__ __device__ explicit GroupLayout(int U) {
+  uint32_t xs, ox, bytes, slots;
+  __host__ __device__ explicit GroupLayout(int U, bool rkv = false) {
+    slots = rkv ? 6 : 5;
     xs = 0;
-    ox = (U * 5 * 16 + 127) / 128 * 128;
-    bytes = U > 1 ? ox + U * 8 * 32 * 16 : 0;
+    ox = (U * slots * 16 + 127) / 128 * 128;
+    // (the R-KV step also passes its parts of the key sum through the
+    // partial-output area, one-warp groups included)
+    bytes = (U > 1 || rkv) ? ox + U * 8 * 32 * 16 : 0;
   }
 };
 
@@ -121,7 +129,7 @@ __device__ __forceinline__ void issue_unit(const FusedParams &p,
                                            const CUtensorMap *tmV,
                                            unsigned char *stage, uint32_t bar,
                                            int idx, int lane) {
-  const StageLayout L(p.R);
+  const StageLayout L(p.R, p.rkv != 0);
   const UnitIdx x = unit_idx(p, idx);
   const uint32_t s0 = smem_u32(stage);
   if (lane == 0) {
@@ -151,6 +159,10 @@ __device__ __forceinline__ void issue_unit(const FusedParams &p,
                (i < nsc ? sc + i * 16 : ps + (i - nsc) * 16));
   if (lane == 31)
     cp_async16(s0 + L.st, p.c.state + x.ug * 4);
+  if (p.rkv)  // the kept key sum (used only if the state marks it valid)
+    cp_async16(s0 + L.rs + lane * 16,
+               reinterpret_cast<const unsigned char *>(p.c.rsum + x.ug * 128) +
+                   lane * 16);
   cp_async_arrive_noinc(bar);
 }
 
@@ -170,7 +182,7 @@ __device__ bool wait_issued(volatile int *issued, int k, volatile int *abort,
   return true;
 }
 
-template <int T, int U, bool kOutBf16>
+template <int T, int U, bool kOutBf16, bool kRkv>
 __global__ void __launch_bounds__(kMaxThreads, 1)
     fused_step_kernel(const __grid_constant__ CUtensorMap tmK,
                       const __grid_constant__ CUtensorMap tmV,
@@ -189,7 +201,7 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
   const int mine = (int)blockIdx.x < n_units
                        ? (n_units - 1 - (int)blockIdx.x) / (int)gridDim.x + 1
                        : 0;
-  const StageLayout L(16 * T);
+  const StageLayout L(16 * T, kRkv);
   const int consumers = p.n_groups * U;
 
   if (threadIdx.x == 0) {
@@ -250,7 +262,7 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
   } else if (warp < consumers) {
     const int grp = warp / U, w = warp % U, bar_id = 1 + grp;
     unsigned char *garea =
-        smem + p.n_stages * L.bytes + grp * GroupLayout(U).bytes;
+        smem + p.n_stages * L.bytes + grp * GroupLayout(U, kRkv).bytes;
     for (int k = grp; k < mine; k += p.n_groups) {
       const int s = k % p.n_stages;
       const uint32_t ph = (uint32_t)(k / p.n_stages) & 1u;
@@ -272,9 +284,9 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
       if (!s_ok[grp]) break;
       mbar_try_wait(smem_u32(&full_bar[s]), ph);  // acquire for this thread
       UnitFront<(T + U - 1) / U> f;
-      const bool ok = unit_front<T, U>(p, smem + s * L.bytes,
-                                       (int)blockIdx.x + k * (int)gridDim.x,
-                                       w, lane, f);
+      const bool ok = unit_front<T, U, kRkv>(
+          p, smem + s * L.bytes, (int)blockIdx.x + k * (int)gridDim.x, w,
+          lane, f, garea, bar_id);
       // Each warp releases the stage once its own reads and writes of it
       // are done (the async-proxy fence orders them before the refill); the
       // rest of the unit runs from registers and the group's own area.
@@ -285,8 +297,8 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
         mbar_arrive(smem_u32(&empty_bar[s]));
       }
       if (ok) {
-        unit_publish<T, U>(garea, f, w, lane);
-        unit_back<T, U, kOutBf16>(p, garea, f, w, lane, bar_id);
+        unit_publish<T, U, kRkv>(garea, f, w, lane);
+        unit_back<T, U, kOutBf16, kRkv>(p, garea, f, w, lane, bar_id);
       }
     }
   }
@@ -303,11 +315,11 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
   }
 }
 
-template <int T, int U, bool kOutBf16>
+template <int T, int U, bool kOutBf16, bool kRkv>
 cudaError_t launch_tu(const CUtensorMap &tmK, const CUtensorMap &tmV,
                       const FusedParams &p, int grid, int smem_bytes,
                       cudaStream_t st) {
-  auto kern = fused_step_kernel<T, U, kOutBf16>;
+  auto kern = fused_step_kernel<T, U, kOutBf16, kRkv>;
   cudaError_t e = cudaFuncSetAttribute(
       kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
   if (e != cudaSuccess) return e;
@@ -315,14 +327,15 @@ cudaError_t launch_tu(const CUtensorMap &tmK, const CUtensorMap &tmV,
                     smem_bytes, st, tmK, tmV, p);
 }
 
-template <bool kOutBf16>
+template <bool kOutBf16, bool kRkv>
 cudaError_t launch_t(const CUtensorMap &tmK, const CUtensorMap &tmV,
                      const FusedParams &p, int grid, int smem_bytes,
                      cudaStream_t st) {
   // (tiles, warps per unit): one tile per warp, or two.
 #define KVR_TU(T_, U_)                                                   \
   if (p.R == 16 * T_ && p.group_warps == U_)                             \
-    return launch_tu<T_, U_, kOutBf16>(tmK, tmV, p, grid, smem_bytes, st);
+    return launch_tu<T_, U_, kOutBf16, kRkv>(tmK, tmV, p, grid,          \
+                                             smem_bytes, st);
   KVR_TU(1, 1)
   KVR_TU(2, 1) KVR_TU(2, 2)
   KVR_TU(3, 2) KVR_TU(3, 3)
@@ -337,7 +350,9 @@ cudaError_t launch_t(const CUtensorMap &tmK, const CUtensorMap &tmV,
 
 }  // namespace
 
-int fused_stage_bytes(int R) { return (int)StageLayout(R).bytes; }
+int fused_stage_bytes(int R, bool rkv) {
+  return (int)StageLayout(R, rkv).bytes;
+}
 
 int fused_group_warps(int R, int requested) {
   if (R % 16 != 0 || R < 16 || R > 128) return 0;
@@ -346,7 +361,9 @@ int fused_group_warps(int R, int requested) {
   return T <= 3 ? one : two;  // measured: two tiles per warp from T = 4 on
 }
 
-int fused_group_bytes(int U) { return (int)GroupLayout(U).bytes; }
+int fused_group_bytes(int U, bool rkv) {
+  return (int)GroupLayout(U, rkv).bytes;
+}
 int fused_max_groups() { return kMaxGroups; }
 int fused_max_threads() { return kMaxThreads; }
 int fused_producer_warps() { return kProducers; }
@@ -358,8 +375,12 @@ cudaError_t launch_fused_step(const CUtensorMap &tmK, const CUtensorMap &tmV,
       p.n_groups < 1 || p.n_groups > kMaxGroups || p.n_stages > kMaxStages ||
       32 * (p.n_groups * p.group_warps + kProducers) > kMaxThreads)
     return cudaErrorInvalidValue;
-  return p.c.out_bf16 ? launch_t<true>(tmK, tmV, p, grid, smem_bytes, st)
-                      : launch_t<false>(tmK, tmV, p, grid, smem_bytes, st);
+  if (p.rkv)
+    return p.c.out_bf16
+               ? launch_t<true, true>(tmK, tmV, p, grid, smem_bytes, st)
+               : launch_t<false, true>(tmK, tmV, p, grid, smem_bytes, st);
+  return p.c.out_bf16 ? launch_t<true, false>(tmK, tmV, p, grid, smem_bytes, st)
+                      : launch_t<false, false>(tmK, tmV, p, grid, smem_bytes, st);
 }
 
 }  // namespace kvr

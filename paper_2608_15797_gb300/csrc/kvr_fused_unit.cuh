@@ -38,16 +38,90 @@ struct UnitFront {
   int ps[TW][2];            // their positions
   int4 nrow;                // own_new warp: 16 bytes of the new k (lanes
                             // 0-15) or v (lanes 16-31) row
+  float rr[TW][2];          // R-KV step: mean cosine of rows r0, r0 + 8
+                            // with the other live rows
+  float s4[4];              // R-KV step, the warp owning the new row: the
+                            // key sum after the append, dims 4 lane .. + 3
 };
 
-template <int T, int U>
+// 1 / |k| of one key held as four dims a lane (0 for a zero key); every
+// lane gets the same value.  The library's kept key sum adds and removes a
+// row's normalised key with this same arithmetic.
+__device__ __forceinline__ float warp_inv_norm(const float (&k)[4]) {
+  float ss = fmaf(k[3], k[3], fmaf(k[2], k[2], fmaf(k[1], k[1], k[0] * k[0])));
+  ss = dev::warp_sum(ss);
+  return ss > 0.f ? rsqrtf(ss) : 0.f;
+}
+
+// x as three bf16 terms t[0] + t[1] + t[2] (the third rounded when packed).
+__device__ __forceinline__ void split3(float x, float (&t)[3]) {
+  const float h = __bfloat162float(__float2bfloat16_rn(x));
+  const float r = x - h;
+  const float m = __bfloat162float(__float2bfloat16_rn(r));
+  t[0] = h;
+  t[1] = m;
+  t[2] = r - m;
+}
+
+// The key sum S as the B operand of K S (m16n8k16; columns 0-2 the three
+// terms of S): lane 4 t + p holds term t of dims 16 ks + 2 p, + 1 (word 0)
+// and 16 ks + 8 + 2 p, + 1 (word 1).  Each lane holds S for dims
+// 4 lane .. + 3 in s4; the terms pass through this warp's scratch sbx
+// ([8][12][2] words) in that order.
+__device__ __forceinline__ void key_sum_fragments(const float (&s4)[4],
+                                                  uint32_t *sbx, int lane,
+                                                  uint32_t (&sb)[8][2]) {
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const int d = 4 * lane + 2 * h;
+    const int ks = d >> 4, j = d & 15, reg = j >> 3, pp = (j & 7) >> 1;
+    float a[3], b[3];
+    split3(s4[2 * h], a);
+    split3(s4[2 * h + 1], b);
+#pragma unroll
+    for (int t = 0; t < 3; ++t)
+      sbx[(ks * 12 + 4 * t + pp) * 2 + reg] = pack_bf16(a[t], b[t]);
+  }
+  __syncwarp();
+#pragma unroll
+  for (int ks = 0; ks < 8; ++ks) {
+    if (lane < 12) {
+      const uint2 v = *reinterpret_cast<const uint2 *>(sbx + (ks * 12 + lane) * 2);
+      sb[ks][0] = v.x;
+      sb[ks][1] = v.y;
+    } else {
+      sb[ks][0] = sb[ks][1] = 0u;
+    }
+  }
+}
+
+// Dims 4 lane .. 4 lane + 3 of a bf16 row of 128.
+__device__ __forceinline__ void row4(const void *row, int lane, float (&k)[4]) {
+  const uint2 w = *reinterpret_cast<const uint2 *>(
+      static_cast<const unsigned char *>(row) + 8 * lane);
+  k[0] = __uint_as_float(w.x << 16);
+  k[1] = __uint_as_float(w.x & 0xffff0000u);
+  k[2] = __uint_as_float(w.y << 16);
+  k[3] = __uint_as_float(w.y & 0xffff0000u);
+}
+
+// x as three bf16 terms (x0 + x1 + x2 carries the 24-bit mantissa): term t.
+__device__ __forceinline__ float bf16_term(float x, int t) {
+  const float h = __bfloat162float(__float2bfloat16_rn(x));
+  if (t == 0) return h;
+  const float m = __bfloat162float(__float2bfloat16_rn(x - h));
+  return t == 1 ? m : x - h - m;
+}
+
+template <int T, int U, bool kRkv>
 __device__ __forceinline__ bool unit_front(const FusedParams &p,
                                            unsigned char *stage, int idx,
                                            int w, int lane,
-                                           UnitFront<(T + U - 1) / U> &f) {
+                                           UnitFront<(T + U - 1) / U> &f,
+                                           unsigned char *garea, int bar_id) {
   constexpr int TW = (T + U - 1) / U;  // tiles per warp (at most)
   constexpr int R = 16 * T;
-  const StageLayout L(R);
+  const StageLayout L(R, kRkv);
   {
     const UnitIdx x = unit_idx(p, idx);
     f.ug = x.ug;
@@ -87,6 +161,11 @@ __device__ __forceinline__ bool unit_front(const FusedParams &p,
         const int r = r_lo + (i >> 4), c16 = i & 15;
         *reinterpret_cast<int4 *>((c16 < 8 ? V0 : V1) + r * 128 +
                                   (c16 & 7) * 16) = make_int4(0, 0, 0, 0);
+        // A fresh R-KV key sum reads every row of the tile: padding keys
+        // must be zeros too (rows past the box are stale).
+        if (kRkv && ST[2] != 1)
+          *reinterpret_cast<int4 *>((c16 < 8 ? K0 : K1) + r * 128 +
+                                    (c16 & 7) * 16) = make_int4(0, 0, 0, 0);
       }
   }
   __syncwarp();
@@ -103,12 +182,19 @@ __device__ __forceinline__ bool unit_front(const FusedParams &p,
   }
 
   // 3. Logits of the owned tiles: m16n8 per 16 rows, 8 k-steps split over
-  //    two accumulator chains.
+  //    two accumulator chains.  The R-KV step also takes the tile's Gram
+  //    blocks K K^T from the same A fragments (K rows are a row-major B
+  //    operand as they stand): their diagonals are the squared key norms,
+  //    and inv holds 1 / |k| of rows r0 and r0 + 8 (0 for a zero key and
+  //    for rows past the live ones).
   float (&acc)[TW][4] = f.pr;
+  float inv[TW][2];
 #pragma unroll
   for (int j = 0; j < TW; ++j) {
     float a2[4] = {0.f, 0.f, 0.f, 0.f};
+    float g0[4] = {0.f, 0.f, 0.f, 0.f}, g1[4] = {0.f, 0.f, 0.f, 0.f};
     acc[j][0] = acc[j][1] = acc[j][2] = acc[j][3] = 0.f;
+    inv[j][0] = inv[j][1] = 0.f;
     const int tt = w + j * U;
     if (tt < T) {
       const int row = tt * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
@@ -123,9 +209,158 @@ __device__ __forceinline__ bool unit_front(const FusedParams &p,
           mma_bf16(a2, a0, a1, a2r, a3, qb[ks][0], qb[ks][1]);
         else
           mma_bf16(acc[j], a0, a1, a2r, a3, qb[ks][0], qb[ks][1]);
+        if constexpr (kRkv) {
+          mma_bf16(g0, a0, a1, a2r, a3, a0, a2r);  // columns: rows 0-7
+          mma_bf16(g1, a0, a1, a2r, a3, a1, a3);   // columns: rows 8-15
+        }
       }
 #pragma unroll
       for (int e = 0; e < 4; ++e) acc[j][e] += a2[e];
+      if constexpr (kRkv) {
+        // Diagonal (r, r) of a block sits in lane 4 r + r / 2, register
+        // r & 1 (rows 0-7) or 2 + (r & 1) (rows 8-15).
+        const int rl = lane >> 2;
+        const float x = (rl & 1) ? g0[1] : g0[0];
+        const float y = (rl & 1) ? g1[3] : g1[2];
+        const int src = 4 * rl + (rl >> 1);
+        const float na = __shfl_sync(0xffffffffu, x, src);
+        const float nb = __shfl_sync(0xffffffffu, y, src);
+        const int ra = tt * 16 + rl, rb = ra + 8;
+        inv[j][0] = (ra < n && na > 0.f) ? rsqrtf(na) : 0.f;
+        inv[j][1] = (rb < n && nb > 0.f) ? rsqrtf(nb) : 0.f;
+      }
+    }
+  }
+
+  if constexpr (kRkv) {
+    // 3b. R-KV redundancy (App. C, the library's reading): r_i, the mean
+    //     cosine of key i with the other n - 1 live keys, is
+    //     (k_i . S / |k_i| - 1) / (n - 1) with S the sum of the normalised
+    //     live keys (no n x n similarity).  Both products run on the tensor
+    //     cores with the fp32 vector split into three bf16 terms (columns
+    //     0-2 of the B operand; their sum carries the full mantissa):
+    //     S^T = K^T (1/|k|) in the PV product's form, then K S.
+    const int c2 = (lane & 3) * 2, rl = lane >> 2;
+    float *SX = reinterpret_cast<float *>(garea + GroupLayout(U, true).ox);
+    const float *RS = reinterpret_cast<const float *>(stage + L.rs);
+    // A kept sum (state word 2 set by the previous R-KV step of this unit)
+    // needs only the new key added: S = kept + k_new / |k_new|.  Otherwise
+    // the group sums every live row's normalised key afresh.
+    const bool warm = ST[2] == 1;
+    uint32_t sb[8][2];
+    if (warm) {
+      float kn4[4], s4[4];
+      row4(KN, lane, kn4);
+      const float inv_new = warp_inv_norm(kn4);
+      const float4 rs = reinterpret_cast<const float4 *>(RS)[lane];
+      s4[0] = fmaf(kn4[0], inv_new, rs.x);
+      s4[1] = fmaf(kn4[1], inv_new, rs.y);
+      s4[2] = fmaf(kn4[2], inv_new, rs.z);
+      s4[3] = fmaf(kn4[3], inv_new, rs.w);
+      // This warp's own partial-output slot is free until unit_publish.
+      key_sum_fragments(s4, reinterpret_cast<uint32_t *>(SX) + w * 1024, lane,
+                        sb);
+      if (f.own_new)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) f.s4[e] = s4[e];
+    } else {
+      float fs[8][4];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) fs[i][0] = fs[i][1] = fs[i][2] = fs[i][3] = 0.f;
+#pragma unroll
+      for (int j = 0; j < TW; ++j) {
+        const int tt = w + j * U;
+        if (tt >= T) continue;
+        // Columns (c2, c2 + 1) of rows r0 and r0 + 8: terms 0, 1 in lanes
+        // c2 = 0, term 2 in lanes c2 = 2.
+        const float ia = inv[j][0], ib = inv[j][1];
+        const uint32_t h0 =
+            c2 == 0 ? pack_bf16(bf16_term(ia, 0), bf16_term(ia, 1))
+                    : (c2 == 2 ? pack_bf16(bf16_term(ia, 2), 0.f) : 0u);
+        const uint32_t h1 =
+            c2 == 0 ? pack_bf16(bf16_term(ib, 0), bf16_term(ib, 1))
+                    : (c2 == 2 ? pack_bf16(bf16_term(ib, 2), 0.f) : 0u);
+        const uint32_t pb0 = movm_t(h0), pb1 = movm_t(h1);
+        const int row = tt * 16 + (lane & 7) + ((lane >> 4) << 3);
+        const uint32_t b0 = smem_u32(K0) + row * 128, b1 = smem_u32(K1) + row * 128;
+#pragma unroll
+        for (int mt = 0; mt < 8; ++mt) {
+          const int c16 = 2 * mt + ((lane >> 3) & 1);
+          const uint32_t addr = (c16 >> 3 ? b1 : b0) + (((c16 & 7) ^ (row & 7)) << 4);
+          uint32_t a0, a1, a2, a3;
+          ldsm_x4_t(addr, a0, a1, a2, a3);
+          mma_bf16(fs[mt], a0, a1, a2, a3, pb0, pb1);
+        }
+      }
+      // This warp's part of S, dims mt * 16 + r0 (+ 8): columns 0 + 1 in
+      // the lane with c2 = 0, column 2 one lane up.
+#pragma unroll
+      for (int mt = 0; mt < 8; ++mt) {
+        const float t2a = __shfl_down_sync(0xffffffffu, fs[mt][0], 1);
+        const float t2b = __shfl_down_sync(0xffffffffu, fs[mt][2], 1);
+        if (c2 == 0) {
+          SX[w * 128 + mt * 16 + rl] = fs[mt][0] + fs[mt][1] + t2a;
+          SX[w * 128 + mt * 16 + rl + 8] = fs[mt][2] + fs[mt][3] + t2b;
+        }
+      }
+      group_bar(bar_id, 32 * U);
+      // S as the dots' B operand (as above); the warps' parts are added in
+      // warp order.
+#pragma unroll
+      for (int ks = 0; ks < 8; ++ks) {
+        float v[4] = {0.f, 0.f, 0.f, 0.f};
+        if (lane < 12) {
+          const int d0 = 16 * ks + 2 * (lane & 3);
+#pragma unroll
+          for (int u = 0; u < U; ++u) {
+            v[0] += SX[u * 128 + d0];
+            v[1] += SX[u * 128 + d0 + 1];
+            v[2] += SX[u * 128 + d0 + 8];
+            v[3] += SX[u * 128 + d0 + 9];
+          }
+          const int t = lane >> 2;
+#pragma unroll
+          for (int e = 0; e < 4; ++e) v[e] = bf16_term(v[e], t);
+        }
+        sb[ks][0] = pack_bf16(v[0], v[1]);
+        sb[ks][1] = pack_bf16(v[2], v[3]);
+      }
+      if (f.own_new)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          float x = 0.f;
+#pragma unroll
+          for (int u = 0; u < U; ++u) x += SX[u * 128 + 4 * lane + e];
+          f.s4[e] = x;
+        }
+      // Every warp has read the parts before any writes the area again
+      // (unit_publish).
+      group_bar(bar_id, 32 * U);
+    }
+    const float inv_n1 = n > 1 ? 1.f / (float)(n - 1) : 0.f;
+#pragma unroll
+    for (int j = 0; j < TW; ++j) {
+      f.rr[j][0] = f.rr[j][1] = 0.f;
+      const int tt = w + j * U;
+      if (tt >= T) continue;
+      float dd[4] = {0.f, 0.f, 0.f, 0.f};
+      const int row = tt * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+      const uint32_t b0 = smem_u32(K0) + row * 128, b1 = smem_u32(K1) + row * 128;
+#pragma unroll
+      for (int ks = 0; ks < 8; ++ks) {
+        const int cc = ((ks & 3) << 1) + (lane >> 4);
+        const uint32_t addr = (ks >> 2 ? b1 : b0) + ((cc ^ (row & 7)) << 4);
+        uint32_t a0, a1, a2r, a3;
+        ldsm_x4(addr, a0, a1, a2r, a3);
+        mma_bf16(dd, a0, a1, a2r, a3, sb[ks][0], sb[ks][1]);
+      }
+      const float t2a = __shfl_down_sync(0xffffffffu, dd[0], 1);
+      const float t2b = __shfl_down_sync(0xffffffffu, dd[2], 1);
+      float da = dd[0] + dd[1] + t2a, db = dd[2] + dd[3] + t2b;
+      da = __shfl_sync(0xffffffffu, da, lane & ~3);
+      db = __shfl_sync(0xffffffffu, db, lane & ~3);
+      f.rr[j][0] = (da * inv[j][0] - (inv[j][0] > 0.f ? 1.f : 0.f)) * inv_n1;
+      f.rr[j][1] = (db * inv[j][1] - (inv[j][1] > 0.f ? 1.f : 0.f)) * inv_n1;
     }
   }
 
@@ -221,15 +456,16 @@ __device__ __forceinline__ bool unit_front(const FusedParams &p,
 
 // The warp's statistics and partial output into the group area (U > 1);
 // after this the partial-output registers are free.
-template <int T, int U>
+template <int T, int U, bool kRkv>
 __device__ __forceinline__ void unit_publish(unsigned char *garea,
                                              const UnitFront<(T + U - 1) / U> &f,
                                              int w, int lane) {
   if constexpr (U > 1) {
-    const GroupLayout GL(U);
+    const GroupLayout GL(U, kRkv);
     float4 *XS4 = reinterpret_cast<float4 *>(garea + GL.xs);
     float4 *OX = reinterpret_cast<float4 *>(garea + GL.ox);
-    if (lane < 4) XS4[w * 5 + lane] = make_float4(f.ref0, f.ref1, f.z0, f.z1);
+    if (lane < 4)
+      XS4[w * GL.slots + lane] = make_float4(f.ref0, f.ref1, f.z0, f.z1);
 #pragma unroll
     for (int mt = 0; mt < 8; ++mt)
       OX[(w * 8 + mt) * 32 + lane] =
@@ -237,13 +473,15 @@ __device__ __forceinline__ void unit_publish(unsigned char *garea,
   }
 }
 
-template <int T, int U, bool kOutBf16>
+constexpr float kLog2e = 1.4426950408889634f;
+
+template <int T, int U, bool kOutBf16, bool kRkv>
 __device__ __forceinline__ void unit_back(const FusedParams &p,
                                           unsigned char *garea,
                                           UnitFront<(T + U - 1) / U> &f,
                                           int w, int lane, int bar_id) {
   constexpr int TW = (T + U - 1) / U;
-  const GroupLayout GL(U);
+  const GroupLayout GL(U, kRkv);
   const int G = p.c.G;
   const int m = f.m, n = m + 1, t = f.t;
   const int r0 = lane >> 2, c2 = (lane & 3) * 2;
@@ -261,7 +499,7 @@ __device__ __forceinline__ void unit_back(const FusedParams &p,
     float M0 = -INFINITY, M1 = -INFINITY;
 #pragma unroll
     for (int v = 0; v < U; ++v) {
-      r[v] = XS4[v * 5 + (lane & 3)];
+      r[v] = XS4[v * GL.slots + (lane & 3)];
       if (r[v].z > 0.f) M0 = fmaxf(M0, r[v].x);
       if (r[v].w > 0.f) M1 = fmaxf(M1, r[v].y);
     }
@@ -361,8 +599,10 @@ __device__ __forceinline__ void unit_back(const FusedParams &p,
   unsigned long long best = ~0ull;
   int bi = -1;
   float new_score = 0.f;
+  float sv[TW][2];  // R-KV step: updated scores of the owned rows
 #pragma unroll
   for (int j = 0; j < TW; ++j) {
+    sv[j][0] = sv[j][1] = 0.f;
     float sa = (g0 ? f.pr[j][0] * f0 : 0.f) + (g1 ? f.pr[j][1] * f1 : 0.f);
     float sb = (g0 ? f.pr[j][2] * f0 : 0.f) + (g1 ? f.pr[j][3] * f1 : 0.f);
     sa += __shfl_xor_sync(0xffffffffu, sa, 1);
@@ -378,8 +618,9 @@ __device__ __forceinline__ void unit_back(const FusedParams &p,
           const float s = f.sc[j][hsel] + (hsel ? sb : sa) * p.inv_g;
           if (r < m) gsc[r] = s;
           else new_score = s;
+          sv[j][hsel] = s;
           const int pr = f.ps[j][hsel];
-          if (pr <= wlo) {
+          if (!kRkv && pr <= wlo) {
             const unsigned long long key =
                 ((unsigned long long)__float_as_uint(s) << 32) |
                 (unsigned long long)(0xFFFFFFFFu - (unsigned)pr);
@@ -394,6 +635,76 @@ __device__ __forceinline__ void unit_back(const FusedParams &p,
   }
   // The lane that scored the new row passes its score to the whole warp.
   new_score = __shfl_sync(0xffffffffu, new_score, ((m & 15) & 7) * 4);
+  if constexpr (kRkv) {
+    // R-KV (App. C, the library's reading) over the candidates C (rows
+    // outside the window): I = s / sum_C s, R = softmax_C(r) and
+    // z = lam I - (1 - lam) R; the victim is the lowest (z, -position).
+    // Each warp reduces its own candidates (sum of s, max of r and the
+    // sum of exp(r - max)); the group merges them in warp order.
+    float ssum = 0.f, rmax = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < TW; ++j)
+#pragma unroll
+      for (int hsel = 0; hsel < 2; ++hsel) {
+        const int r = (w + j * U) * 16 + r0 + 8 * hsel;
+        if ((lane & 3) == 0 && w + j * U < T && r < n &&
+            f.ps[j][hsel] <= wlo) {
+          ssum += sv[j][hsel];
+          rmax = fmaxf(rmax, f.rr[j][hsel]);
+        }
+      }
+    ssum = dev::warp_sum(ssum);
+    rmax = dev::warp_max(rmax);
+    float esum = 0.f;
+#pragma unroll
+    for (int j = 0; j < TW; ++j)
+#pragma unroll
+      for (int hsel = 0; hsel < 2; ++hsel) {
+        const int r = (w + j * U) * 16 + r0 + 8 * hsel;
+        if ((lane & 3) == 0 && w + j * U < T && r < n &&
+            f.ps[j][hsel] <= wlo)
+          esum += ex2((f.rr[j][hsel] - rmax) * kLog2e);
+      }
+    esum = dev::warp_sum(esum);
+    float Ssum = ssum, M = rmax, E = esum;
+    if constexpr (U > 1) {
+      if (lane == 0) XS4[w * GL.slots + 5] = make_float4(ssum, rmax, esum, 0.f);
+      group_bar(bar_id, 32 * U);
+      Ssum = 0.f;
+      M = -INFINITY;
+#pragma unroll
+      for (int v = 0; v < U; ++v) {
+        const float4 x = XS4[v * GL.slots + 5];
+        Ssum += x.x;
+        if (x.z > 0.f) M = fmaxf(M, x.y);
+      }
+      E = 0.f;
+#pragma unroll
+      for (int v = 0; v < U; ++v) {
+        const float4 x = XS4[v * GL.slots + 5];
+        if (x.z > 0.f) E += x.z * ex2((x.y - M) * kLog2e);
+      }
+    }
+    const float inv_s = Ssum > 0.f ? 1.f / Ssum : 0.f;
+    const float inv_e = E > 0.f ? 1.f / E : 0.f;
+#pragma unroll
+    for (int j = 0; j < TW; ++j)
+#pragma unroll
+      for (int hsel = 0; hsel < 2; ++hsel) {
+        const int r = (w + j * U) * 16 + r0 + 8 * hsel;
+        const int pr = f.ps[j][hsel];
+        if ((lane & 3) == 0 && w + j * U < T && r < n && pr <= wlo) {
+          const float z = p.lam * (sv[j][hsel] * inv_s) -
+                          (1.f - p.lam) *
+                              (ex2((f.rr[j][hsel] - M) * kLog2e) * inv_e);
+          const unsigned long long key = dev::rkv_key(z, pr);
+          if (key < best) {
+            best = key;
+            bi = r;
+          }
+        }
+      }
+  }
   {
     // Warp argmin of the key: lowest score bits, then highest position
     // (keys are distinct because positions are).
@@ -416,12 +727,12 @@ __device__ __forceinline__ void unit_back(const FusedParams &p,
   if constexpr (U > 1) {
     uint4 *XW = reinterpret_cast<uint4 *>(XS4);
     if (lane == 0)
-      XW[w * 5 + 4] = make_uint4((uint32_t)best, (uint32_t)(best >> 32),
-                                 (uint32_t)bi, 0u);
+      XW[w * GL.slots + 4] = make_uint4((uint32_t)best, (uint32_t)(best >> 32),
+                                        (uint32_t)bi, 0u);
     group_bar(bar_id, 32 * U);
 #pragma unroll
     for (int v = 0; v < U; ++v) {
-      const uint4 a = XW[v * 5 + 4];
+      const uint4 a = XW[v * GL.slots + 4];
       const unsigned long long kb = ((unsigned long long)a.y << 32) | a.x;
       if (kb < best) {
         best = kb;
@@ -436,6 +747,25 @@ __device__ __forceinline__ void unit_back(const FusedParams &p,
   if (f.own_new) {
     const int victim = (p.evict && n > p.budget + p.window) ? bi : -1;
     const int slot = victim < 0 ? m : (victim < m ? victim : -1);
+    if constexpr (kRkv) {
+      // The kept key sum after the step: the evicted row's normalised key
+      // (from the slab, or the new row's own when it is the one evicted)
+      // comes out, read before the new row overwrites its slot.
+      if (victim >= 0) {
+        float kv[4];
+        row4(victim < m ? reinterpret_cast<const unsigned char *>(p.c.K) +
+                              (f.ug * (size_t)p.c.cap + victim) * 256
+                        : reinterpret_cast<const unsigned char *>(p.k_new) +
+                              f.krow * 256,
+             lane, kv);
+        const float iv = warp_inv_norm(kv);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) f.s4[e] = fmaf(-kv[e], iv, f.s4[e]);
+      }
+      *reinterpret_cast<float4 *>(p.c.rsum + f.ug * 128 + 4 * lane) =
+          make_float4(f.s4[0], f.s4[1], f.s4[2], f.s4[3]);
+      __syncwarp();
+    }
     if (slot >= 0) {
       const int chunk = lane & 15;
       __nv_bfloat16 *dst =
@@ -450,6 +780,7 @@ __device__ __forceinline__ void unit_back(const FusedParams &p,
     if (lane == 0) {
       p.c.state[4 * f.ug] = victim < 0 ? m + 1 : m;
       p.c.state[4 * f.ug + 1] = t + 1;
+      p.c.state[4 * f.ug + 2] = kRkv ? 1 : 0;  // the kept key sum is current
     }
   }
 }

@@ -188,6 +188,7 @@ __global__ void __launch_bounds__(kThreads)
   if (tid == 0) {
     c.state[4 * x.u] = n;
     c.state[4 * x.u + 1] = newest + 1;
+    c.state[4 * x.u + 2] = 0;  // the R-KV key sum no longer matches
   }
 }
 
@@ -273,7 +274,10 @@ __global__ void __launch_bounds__(kThreads)
       pu[dst] = pu[src];
     }
   }
-  if (tid == 0) c.state[4 * x.u] = nk;
+  if (tid == 0) {
+    c.state[4 * x.u] = nk;
+    c.state[4 * x.u + 2] = 0;  // the R-KV key sum no longer matches
+  }
 }
 
 // Copy one sequence's prompt rows [L][H][n][d] into its slabs.
@@ -303,6 +307,7 @@ __global__ void load_kernel(CacheView c, int seq, const T *k, const T *v,
   if (blockIdx.y == 0 && threadIdx.x == 0) {
     c.state[4 * u] = n;
     c.state[4 * u + 1] = first_pos + n;
+    c.state[4 * u + 2] = 0;  // no R-KV key sum yet
   }
 }
 

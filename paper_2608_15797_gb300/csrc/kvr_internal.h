@@ -55,9 +55,13 @@ struct CacheView {
   void *V;          // [u][cap][d]
   float *score;     // [u][sstride]
   int32_t *pos;     // [u][sstride]
-  int32_t *state;   // [u][4]: live length, next position, 0, 0
+  int32_t *state;   // [u][4]: live length, next position, rsum valid, 0
   unsigned *err;    // device error word
   float *logits;    // [u][G][cap] scratch for units beyond on-chip size
+  float *rsum;      // [u][d] R-KV: sum of the live rows' normalised keys,
+                    // kept by kvr_decode_step_rkv's one-launch step; valid
+                    // while the unit's state word 2 is 1 (every other call
+                    // that changes the unit's rows writes 0 there)
   int S, L, H, G, d, cap;
   int sstride;      // cap rounded up to 16 (64-byte aligned score/pos rows)
   float scale;      // softmax scale (1/sqrt(d) by default)
@@ -135,13 +139,18 @@ struct FusedParams {
   int group_warps;             // warps sharing one unit
   int budget, window, evict;
   float scale_log2e, inv_g;
+  // R-KV eviction (App. C) instead of the accumulated-attention TopB: the
+  // evicted row is the candidate of lowest z = lam * I - (1 - lam) * R.
+  int rkv;
+  float lam;
 };
-int fused_stage_bytes(int R);
+int fused_stage_bytes(int R, bool rkv = false);
 // Warps that share one unit of R staged rows: `requested` if it is one of
 // the supported choices (one or two row tiles per warp), else the default.
 int fused_group_warps(int R, int requested);
-// Bytes of one consumer group's exchange area (after the ring of stages).
-int fused_group_bytes(int U);
+// Bytes of one consumer group's exchange area (after the ring of stages);
+// the R-KV step needs one more statistics slot a warp.
+int fused_group_bytes(int U, bool rkv = false);
 int fused_max_groups();
 int fused_max_threads();
 int fused_producer_warps();

@@ -47,17 +47,8 @@ __device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
   return d;
 }
 
-// A float's order as an unsigned integer, negative values included.
-__device__ __forceinline__ unsigned ord_bits(float z) {
-  const unsigned b = __float_as_uint(z);
-  return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
-}
-
-// Higher z first, then lower position.
-__device__ __forceinline__ unsigned long long rkv_key(float z, int32_t p) {
-  return (static_cast<unsigned long long>(ord_bits(z)) << 32) |
-         static_cast<unsigned long long>(0xFFFFFFFFu - static_cast<unsigned>(p));
-}
+using dev::ord_bits;
+using dev::rkv_key;
 
 // The unit of this CTA: blocks run over (sequence, layer in [lb, lb + nl),
 // KV head), head fastest.
@@ -272,7 +263,10 @@ __global__ void __launch_bounds__(kThreads)
       pu_g[dst] = pu[src];
     }
   }
-  if (tid == 0) c.state[4 * x.u] = nk;
+  if (tid == 0) {
+    c.state[4 * x.u] = nk;
+    c.state[4 * x.u + 2] = 0;  // the kept key sum is the one-launch step's
+  }
 }
 
 // ---- one warp per unit (units of at most 128 rows: the steady state) -------
@@ -520,7 +514,10 @@ __global__ void __launch_bounds__(kThreads)
       pu[dst] = pu[src];
     }
   }
-  if (lane == 0) c.state[4 * u] = nk;
+  if (lane == 0) {
+    c.state[4 * u] = nk;
+    c.state[4 * u + 2] = 0;  // the kept key sum is the one-launch step's
+  }
 }
 
 template <typename T, int D>

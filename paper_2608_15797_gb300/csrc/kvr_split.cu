@@ -331,6 +331,7 @@ __global__ void __launch_bounds__(128) split_combine_kernel(const SplitParams p,
     c.score[ug * c.sstride + len] = 0.f;
     c.state[4 * ug] = len + 1;
     c.state[4 * ug + 1] = t + 1;
+    c.state[4 * ug + 2] = 0;  // the R-KV key sum no longer matches
   }
 }
 

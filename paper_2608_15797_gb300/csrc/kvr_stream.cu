@@ -391,6 +391,7 @@ __global__ void __launch_bounds__(32 * kWarps)
   if (tid == 0) {
     c.state[4 * ug] = victim < 0 ? m + 1 : m;
     c.state[4 * ug + 1] = t + 1;
+    c.state[4 * ug + 2] = 0;  // the R-KV key sum no longer matches
   }
 }
 

@@ -62,6 +62,8 @@ _SIGS = {
     "kvr_decode_attend_score_noalloc": (_S, [_P, _I, _I, _P, _P, _P, _P, _P]),
     "kvr_evict_compact": (_S, [_P, _I, _I, _I, _I, _P]),
     "kvr_decode_step": (_S, [_P, _I, _I, _P, _P, _P, _P, _I, _I, _P]),
+    "kvr_decode_step_rkv": (_S, [_P, _I, _I, _P, _P, _P, _P, _I, _I,
+                                 ctypes.c_float, _P]),
     "kvr_decode_step_host": (_S, [_P, _I, _I, _P, _P, _P, _P, _P, _P, _P, _P,
                                   _I, _I, _P]),
     "kvr_absorb_chunk": (_S, [_P, _I, _I, _I, _P, _P, _P, _P, _I, _I, _I, _P]),
@@ -174,6 +176,14 @@ def kvr_decode_step(h, layer_begin, layer_end, q, k_new, v_new, out, budget,
     _check(lib.kvr_decode_step(h, layer_begin, layer_end, _ptr(q), _ptr(k_new),
                                _ptr(v_new), _ptr(out), budget, window,
                                _stream(stream)), "kvr_decode_step")
+
+
+def kvr_decode_step_rkv(h, layer_begin, layer_end, q, k_new, v_new, out,
+                        budget, window, lam, stream=None):
+    _check(lib.kvr_decode_step_rkv(h, layer_begin, layer_end, _ptr(q),
+                                   _ptr(k_new), _ptr(v_new), _ptr(out), budget,
+                                   window, float(lam), _stream(stream)),
+           "kvr_decode_step_rkv")
 
 
 def kvr_decode_step_host(h, layer_begin, layer_end, q_host, k_new_host,
@@ -329,6 +339,15 @@ class Cache:
         out = self.new_out(le - lb) if out is None else out
         kvr_decode_step(self.handle, lb, le, q, k_new, v_new, out, budget,
                         window, stream)
+        return out
+
+    def step_rkv(self, q, k_new, v_new, budget, window, lam=0.1, out=None,
+                 layers=None, stream=None):
+        """A decode step with the R-KV eviction (kvr_decode_step_rkv)."""
+        lb, le = self._layers(layers)
+        out = self.new_out(le - lb) if out is None else out
+        kvr_decode_step_rkv(self.handle, lb, le, q, k_new, v_new, out, budget,
+                            window, lam, stream)
         return out
 
     def absorb(self, q, k_new, v_new, budget=0, window=0, evict=True,

@@ -11,11 +11,13 @@ with device-drawn inputs that no check reads.
   28 layers x 4 KV heads = 7,168 units a launch, B = 64, 128, 256 and 512,
   W = 8, bf16 in and out.  The first step evicts every unit from its prior
   context (B + W + 16 to B + W + 600 rows here: the bench's longer prior
-  contexts change only that untimed first step); the steady-state steps run
-  the fused kernel on 73-row units (B = 64) or the chunked kernel on 137,
-  265 and 521-row units.
+  contexts change only that untimed first step); the sequences then move
+  into a steady-state cache of capacity B + W + 1, as in bench.py, where
+  the steady-state steps run the fused kernel on 73-row units (B = 64) or
+  the chunked kernel on 137, 265 and 521-row units.
 - R-KV step (App. C, lambda = 0.1): the same 64 x 28 x 4 units at B + W = 72
-  rows, attend+score then the R-KV eviction, as bench.py --mode rkv.
+  rows, attend+score then the R-KV eviction, then the one-launch R-KV step
+  (kvr_decode_step_rkv) that bench.py --mode rkv times.
 - chunk absorb (Algorithm 1's single forward pass over an accepted step): 64
   sequences x 28 layers at B + W = 72 rows taking 64-token chunks, as
   bench.py --mode absorb.
@@ -57,13 +59,22 @@ def test_decode_step_7b_s64_sampled(B):
     c, o = harness.make_pair(w, 61 + B, S, cap=int(lens.max()) + 1,
                              prompt_lens=lens, out_dtype="bf16", sample=SAMPLE)
     launches = c.launch_count()
-    st = harness.lockstep(c, o, w, 61 + B, 7, w.budget, w.window,
+    harness.lockstep(c, o, w, 61 + B, 1, w.budget, w.window, sample=SAMPLE)
+    # the first step evicts hundreds of rows (attend+score, then eviction)
+    assert c.launch_count() - launches == 2
+    # As bench.py does: the sequences move into a steady-state cache of
+    # capacity B + W + 1 (a dense slab) and the timed steps run there.
+    d = harness.guarded_cache(S, w.n_layers, w.n_kv_heads, w.group,
+                              w.head_dim, m + 1, kv_dtype=w.dtype,
+                              out_dtype="bf16")
+    d.copy_from(c, np.arange(S, dtype=np.int32), np.arange(S, dtype=np.int32))
+    del c
+    launches = d.launch_count()
+    st = harness.lockstep(d, o, w, 61 + B, 6, w.budget, w.window, step0=1,
                           sample=SAMPLE)
-    assert st.units == 7 * len(SAMPLE) * w.n_layers * w.n_kv_heads
-    assert (c.lengths() == m).all()
-    # the first step evicts hundreds of rows (attend+score, then eviction);
-    # the six steady steps are one launch each
-    assert c.launch_count() - launches == 2 + 6
+    assert st.units == 6 * len(SAMPLE) * w.n_layers * w.n_kv_heads
+    assert (d.lengths() == m).all()
+    assert d.launch_count() - launches == 6   # one launch a steady step
 
 
 def test_rkv_step_7b_s64_b64_sampled():
@@ -71,8 +82,12 @@ def test_rkv_step_7b_s64_b64_sampled():
     S, m = 64, w.budget + w.window
     c, o = harness.make_pair(w, 62, S, cap=m + 1, prompt_lens=[m] * S,
                              out_dtype="bf16", sample=SAMPLE)
-    st = rkv_lockstep(c, o, w, 62, 6, w.budget, w.window, 0.1, sample=SAMPLE)
-    assert st.units == 6 * len(SAMPLE) * w.n_layers * w.n_kv_heads
+    st = rkv_lockstep(c, o, w, 62, 3, w.budget, w.window, 0.1, sample=SAMPLE)
+    n0 = c.launch_count()
+    st2 = rkv_lockstep(c, o, w, 62, 3, w.budget, w.window, 0.1, step0=3,
+                       sample=SAMPLE, fused=True)
+    assert c.launch_count() - n0 == 3   # the one-launch step bench.py times
+    assert st.units + st2.units == 6 * len(SAMPLE) * w.n_layers * w.n_kv_heads
     assert (c.lengths() == m).all()
 
 
