@@ -990,7 +990,7 @@ def run_rkv(args):
     attend = cost_model.step_unit_bytes(B + Wn, d, G, 2, 2, B, Wn)
     units = S * L * H
     return dict(total_ms=rkv_ms, per_ms=rkv_ms / K, K=K, launches=launches,
-                launch_bytes=attend * units,
+                launch_bytes=attend * units, profile="decode_step_rkv_7b_s64_b64",
                 score_ms=score_ms / K, two_launch_ms=two_ms / K,
                 metric=f"evicted decode steps/s with R-KV eviction at 7B "
                        f"geometry, B={B}, W={Wn}, lambda={lam} ({S} sequences"
@@ -1153,7 +1153,7 @@ def run_sweep_row(args, B):
     unit_bytes = cost_model.step_unit_bytes(B + W, d, G, 2, 2, B, W)
     return dict(metric=metric_name(w), total_ms=total, per_ms=total / K, K=K,
                 launches=launches, launch_bytes=unit_bytes * S * L * H,
-                regions=regions,
+                regions=regions, profile=f"decode_step_7b_s64_b{B}",
                 config={"workload": f"7b_s64_b{B}", "budget": B, "window": W,
                         "prior_len": f"U[{lo},{max(lo, args.prior_max)}]",
                         "steady_capacity": B + W + 1},
@@ -1170,6 +1170,8 @@ def row_record(r, unit, peak, peak_kind, value=None):
            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak,
                         "unit": "GB/s", "frac": achieved / peak,
                         "peak_kind": peak_kind,
+                        "traffic": committed_traffic(r["profile"])
+                        if "profile" in r else None,
                         "algorithmic_bytes_per_launch": r["launch_bytes"],
                         "launch_ms": r["per_ms"], "kernel": r.get("kernel")},
            "gpu_launches": r["launches"]}
@@ -1252,7 +1254,9 @@ def print_row_line(args, r):
             "hbm_gbs": achieved,
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak,
                          "unit": "GB/s", "frac": achieved / peak,
-                         "peak_kind": peak_kind, "traffic": None,
+                         "peak_kind": peak_kind,
+                         "traffic": committed_traffic(r["profile"])
+                         if "profile" in r else None,
                          "algorithmic_bytes_per_launch": r["launch_bytes"],
                          "launch_ms": r["per_ms"], "kernel": r["kernel"]},
             "gpu_launches": r["launches"]}
