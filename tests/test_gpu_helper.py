@@ -79,3 +79,30 @@ def test_workspace_and_shape_errors():
     with pytest.raises(kvr.KvrError) as e:
         kvr.attend_full(c32, q, kn, vn)
     assert e.value.status == kvr.KVR_EINVAL
+
+
+def test_helper_full_size_sampled():
+    """bench.py --mode helper's launch: 16 sequences x all 28 layers of the
+    1.5B geometry at context 16384, library-chosen splits, bf16 out.  The
+    oracle holds sequences 0 and 15 (sequences are independent; the others
+    run alongside on device-drawn prompts) and checks their outputs at every
+    step, and the appended rows' lengths and positions."""
+    w = inputs.WORKLOADS["1p5b_full16k"]
+    S, samp, ctx = 16, [0, 15], w.prompt
+    c, o = harness.make_pair(w, 46, S, cap=ctx + 3, prompt_lens=[ctx] * S,
+                             out_dtype="bf16", sample=samp)
+    n0 = c.launch_count()
+    for t in range(2):
+        q, kn, vn = inputs.step_inputs(w, 46, t, S)
+        out = kvr.attend_full(c, *(harness.dev(a, "bf16") for a in (q, kn, vn)))
+        ref = o.step(q[samp], kn[samp], vn[samp], evict=False)
+        torch.cuda.synchronize()
+        parity.check_out(out[samp].float().cpu().numpy(), ref,
+                         what=f"out at {t}")
+        assert (c.lengths() == ctx + t + 1).all()
+        for i, s in enumerate(samp):
+            ex = c.export(s, kv=False)
+            assert (ex["pos"][:, :, ctx + t] == ctx + t).all()
+    assert c.launch_count() - n0 == 2 * 2   # split partials + combine a step
+    c.sync_status()
+    harness.check_guards(c)
