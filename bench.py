@@ -1210,7 +1210,8 @@ def run_sweep_row(args, B):
                 config={"workload": f"7b_s64_b{B}", "budget": B, "window": W,
                         "prior_len": f"U[{lo},{max(lo, args.prior_max)}]",
                         "steady_capacity": B + W + 1},
-                kernel="kvr_decode_step (chunked kernel, one launch a step)")
+                kernel="kvr_decode_step (one launch a step: the fused kernel "
+                       "up to 160 rows a unit, the chunked one above)")
 
 
 def row_record(r, unit, peak, peak_kind, value=None):

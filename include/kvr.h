@@ -148,7 +148,7 @@ kvr_status kvr_decode_step(kvr_cache *cache, int layer_begin, int layer_end,
 /* Steps 1-4 with the R-KV eviction in one pass (App. C, lambda; App. D:
  * the eviction's key-similarity pass): equivalent to
  * kvr_decode_attend_score followed by kvr_evict_compact_rkv with the same
- * reading of R-KV.  Where every unit holds at most 128 rows after the
+ * reading of R-KV.  Where every unit holds at most 160 rows after the
  * append and at most one is evicted (bf16, head_dim 128, G <= 8) it is one
  * launch: the redundancy of each row comes from the keys already staged
  * for attention, so no key is read twice; otherwise it runs the two calls.
@@ -299,7 +299,7 @@ kvr_status kvr_cache_set_wait_limit(kvr_cache *cache, uint64_t ns);
 kvr_status kvr_cache_set_hold_first_unit(kvr_cache *cache, int enable);
 
 /* Choose whether kvr_decode_attend_score / kvr_decode_step may use the
- * fused single-pass kernel (bf16, head_dim 128, G <= 8, at most 128 live rows
+ * fused single-pass kernel (bf16, head_dim 128, G <= 8, at most 160 live rows
  * per unit, at most one eviction per unit; the default) or must use the
  * generic kernels for every shape.  Both compute the same step; this exists
  * for testing and measurement.  enable: 0 or 1. */

@@ -288,7 +288,7 @@ bool try_fused(kvr_cache *c, const StepArgs &a, bool evict, int budget,
                bool rkv = false, float lam = 0.f) {
   const CacheView &v = c->view;
   if (!c->fused || !v.kv_bf16 || v.d != 128 || v.G > 8) return false;
-  if (a.max_rows > 128) return false;
+  if (a.max_rows > kvr::fused_max_rows()) return false;
   if (evict && (long long)a.max_rows > (long long)budget + window + 1)
     return false;
   const size_t rows = (size_t)v.S * v.L * v.H * v.cap;

@@ -1,5 +1,5 @@
 // kvr_fused.cu -- the fused steady-state decode step for bf16, head_dim 128,
-// G <= 8 and at most 128 live rows per unit: append + Attn(q_t, C) (Eq. 1)
+// G <= 8 and at most 160 live rows per unit: append + Attn(q_t, C) (Eq. 1)
 // + accumulated-attention update (Sec. 2.1) + TopB eviction of the single
 // surplus row (Eq. 1 with the Sec. 4.1 window) + in-place compaction, in one
 // pass over K and V.
@@ -56,6 +56,7 @@ namespace {
 using namespace ptx;
 
 constexpr int kMaxStages = 8;
+constexpr int kMaxTiles = 10;   // 16-row tiles a unit: at most 160 rows
 constexpr int kMaxGroups = 4;      // units in flight on the consumer side
 constexpr int kProducers = 2;      // TMA-issuing warps
 constexpr int kMaxThreads = 512;   // consumer warps + the producers
@@ -344,6 +345,7 @@ cudaError_t launch_t(const CUtensorMap &tmK, const CUtensorMap &tmV,
   KVR_TU(6, 3) KVR_TU(6, 6)
   KVR_TU(7, 4) KVR_TU(7, 7)
   KVR_TU(8, 4) KVR_TU(8, 8)
+  KVR_TU(9, 5) KVR_TU(10, 5)
 #undef KVR_TU
   return cudaErrorInvalidValue;
 }
@@ -355,8 +357,11 @@ int fused_stage_bytes(int R, bool rkv) {
 }
 
 int fused_group_warps(int R, int requested) {
-  if (R % 16 != 0 || R < 16 || R > 128) return 0;
+  if (R % 16 != 0 || R < 16 || R > 16 * kMaxTiles) return 0;
   const int T = R / 16, one = T, two = (T + 1) / 2;
+  // Past 8 tiles only two tiles a warp (one a warp would need 9-10 warps
+  // a group; the register file holds two such groups at most).
+  if (T > 8) return two;
   if (requested == one || requested == two) return requested;
   return T <= 3 ? one : two;  // measured: two tiles per warp from T = 4 on
 }
@@ -365,6 +370,7 @@ int fused_group_bytes(int U, bool rkv) {
   return (int)GroupLayout(U, rkv).bytes;
 }
 int fused_max_groups() { return kMaxGroups; }
+int fused_max_rows() { return 16 * kMaxTiles; }
 int fused_max_threads() { return kMaxThreads; }
 int fused_producer_warps() { return kProducers; }
 

@@ -124,7 +124,7 @@ cudaError_t launch_copy_seqs(const CacheView &dst, const CacheView &src,
                              const SeqPairs &p, int n_pairs, int row_bytes,
                              cudaStream_t st);
 
-// Fused steady-state step (kvr_fused.cu): bf16, d = 128, G <= 8, at most 128
+// Fused steady-state step (kvr_fused.cu): bf16, d = 128, G <= 8, at most 160
 // live rows per unit after the append, at most one eviction per unit.
 struct FusedParams {
   CacheView c;
@@ -152,6 +152,7 @@ int fused_group_warps(int R, int requested);
 // the R-KV step needs one more statistics slot a warp.
 int fused_group_bytes(int U, bool rkv = false);
 int fused_max_groups();
+int fused_max_rows();   // live rows a unit after the append (160)
 int fused_max_threads();
 int fused_producer_warps();
 cudaError_t launch_fused_step(const CUtensorMap &tmK, const CUtensorMap &tmV,

@@ -23,8 +23,9 @@ formulas and the inputs.
 The prompt rows are imported in a random slot order per unit, so the lower
 position is not the lower slot.  The cases run the kernel each budget
 dispatches to at the benchmarked geometry: the fused step (7B, 64 sequences
-x 28 layers x 4 KV heads, B = 64), the chunked step (B = 128, 256, 512, the
-same 7,168 units a launch, so each persistent CTA takes many units), the
+x 28 layers x 4 KV heads, B = 64 and 128: five and nine row tiles a unit),
+the chunked step (B = 256, 512; the same 7,168 units a launch, so each
+persistent CTA takes many units), the
 streaming step (units of 1,409 rows) and the generic pair; a prompt longer
 than B + W makes step 1 the generic first eviction.  The candidate case
 forks a fresh 72B parent into 8 candidates and commits one: its cut from
@@ -122,7 +123,8 @@ def _check_state(c, B, P, t, where):
 @pytest.mark.parametrize("B,S,L,extra,fused", [
     (64, 64, 28, 0, True),      # fused step at the headline's size
     (64, 64, 28, 40, True),     # generic first eviction, then fused
-    (128, 64, 28, 0, True),     # chunked step
+    (128, 64, 28, 0, True),     # fused step, nine row tiles
+    (200, 16, 28, 0, True),     # chunked step (209 rows)
     (256, 64, 28, 0, True),
     (512, 64, 28, 0, True),
     (1400, 2, 4, 0, True),      # streaming step (1,409 rows)

@@ -26,9 +26,9 @@ pytestmark = pytest.mark.gpu
 
 W = 8
 # kernel -> (budget B, use the one-launch kernels): the fused step takes
-# units of at most 128 rows, the chunked one 129-1024, the streaming one
+# units of at most 160 rows, the chunked one 161-1024, the streaming one
 # 1025-2048; fused=False runs the generic pair.
-KERNELS = {"fused": (64, True), "chunked": (128, True), "stream": (1100, True),
+KERNELS = {"fused": (64, True), "chunked": (200, True), "stream": (1100, True),
            "generic": (64, False)}
 
 

@@ -13,8 +13,8 @@ with device-drawn inputs that no check reads.
   context (B + W + 16 to B + W + 600 rows here: the bench's longer prior
   contexts change only that untimed first step); the sequences then move
   into a steady-state cache of capacity B + W + 1, as in bench.py, where
-  the steady-state steps run the fused kernel on 73-row units (B = 64) or
-  the chunked kernel on 137, 265 and 521-row units.
+  the steady-state steps run the fused kernel on 73 and 137-row units
+  (B = 64, 128) or the chunked kernel on 265 and 521-row units.
 - R-KV step (App. C, lambda = 0.1): the same 64 x 28 x 4 units at B + W = 72
   rows, attend+score then the R-KV eviction, then the one-launch R-KV step
   (kvr_decode_step_rkv) that bench.py --mode rkv times.
@@ -49,10 +49,11 @@ def _cuda():
 
 @pytest.mark.parametrize("B", [64, 128, 256, 512])
 def test_decode_step_7b_s64_sampled(B):
-    """The throughput sweep's launches: B = 64 runs the fused kernel on
-    73-row units, B = 128 / 256 / 512 the chunked kernel on 137 / 265 /
-    521-row units; either way 7,168 units a launch over persistent CTAs, so
-    every CTA works through many units and reuses its ring stages."""
+    """The throughput sweep's launches: B = 64 and 128 run the fused kernel
+    on 73 and 137-row units (five and nine row tiles), B = 256 / 512 the
+    chunked kernel on 265 / 521-row units; either way 7,168 units a launch
+    over persistent CTAs, so every CTA works through many units and reuses
+    its ring stages."""
     w = inputs.WORKLOADS[f"7b_s64_b{B}"]
     S, m = w.n_seq, B + w.window
     lens = inputs.prior_lengths(61 + B, S, m + 16, m + 600)

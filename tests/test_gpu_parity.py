@@ -74,7 +74,8 @@ def test_budget_window_edges(B, W, fused):
 
 
 @pytest.mark.parametrize("G", [1, 4, 7, 8])
-@pytest.mark.parametrize("B,W", [(64, 8), (100, 19), (3, 5)])
+@pytest.mark.parametrize("B,W", [(64, 8), (100, 19), (3, 5), (128, 8),
+                                 (140, 19)])
 def test_fused_steady_state_shapes(G, B, W):
     """The fused kernel across group sizes and staged-row counts (the last
     16-row tile ragged or full), bf16 output, starting at B+W rows."""
@@ -181,13 +182,13 @@ def test_capacity_and_argument_errors():
 
 
 @pytest.mark.parametrize("chunk", [(0, 0), (-1, 0)], ids=["chunked", "stream"])
-@pytest.mark.parametrize("B,G,out", [(128, 7, "bf16"), (256, 7, "f32"),
-                                     (512, 8, "bf16"), (150, 1, "f32")])
+@pytest.mark.parametrize("B,G,out", [(160, 7, "bf16"), (256, 7, "f32"),
+                                     (512, 8, "bf16"), (170, 1, "f32")])
 def test_long_unit_fused_step(B, G, out, chunk):
-    """Budgets above the staged kernel's 128 rows (the throughput sweep's
-    B = 128 / 256 / 512, W = 8): the chunked kernel (and the older
-    one-CTA-per-unit streaming kernel), one launch per step, in lock-step
-    with the oracle from B + W rows on."""
+    """Budgets above the staged kernel's 160 rows (the throughput sweep's
+    B = 256 / 512, W = 8, and two in between): the chunked kernel (and the
+    older one-CTA-per-unit streaming kernel), one launch per step, in
+    lock-step with the oracle from B + W rows on."""
     W = 8
     w = inputs.Workload("long_b", 2, 2, G, 128, "bf16", B, W, B + W, 5, sigma=1.0)
     c, o = harness.make_pair(w, 13, 2, cap=B + W + 1,
@@ -198,10 +199,11 @@ def test_long_unit_fused_step(B, G, out, chunk):
     assert c.launch_count() - n0 == 5
 
 
-@pytest.mark.parametrize("rows", [128, 129, 1024, 1025, 2048, 2049])
+@pytest.mark.parametrize("rows", [128, 144, 160, 161, 1024, 1025, 2048, 2049])
 def test_kernel_row_limits(rows):
     """Units at each one-launch kernel's row limit and one row past it (rows
-    counted with the appended one): staged fused <= 128, chunked <= 1024,
+    counted with the appended one): staged fused <= 160 (8, 9 and 10 row
+    tiles at 128, 144 and 160), chunked <= 1024,
     streaming <= 2048, then the generic attend + evict pair.  Steady state,
     one eviction a step, ragged units, in lock-step with the oracle."""
     W = 8

@@ -117,9 +117,10 @@ def test_rkv_errors():
 
 # The one-launch R-KV step at each group shape of the fused kernel: units
 # of (B + W + 1) rows staged as T 16-row tiles over U warps (21 rows: T = 2,
-# U = 2; 73: T = 5, U = 3; 109: T = 7, U = 4; 8: one warp).
+# U = 2; 73: T = 5, U = 3; 109: T = 7, U = 4; 8: one warp; 137: T = 9,
+# U = 5; 160: T = 10, U = 5).
 @pytest.mark.parametrize("B,W,G", [(16, 4, 7), (64, 8, 7), (100, 8, 8),
-                                   (5, 2, 3)])
+                                   (5, 2, 3), (128, 8, 7), (151, 8, 8)])
 @pytest.mark.parametrize("lam", [0.0, 0.1, 1.0])
 def test_rkv_fused_step_shapes(B, W, G, lam):
     w = inputs.Workload("rf", 2, 3, G, 128, "bf16", B, W, B + W, 0, sigma=1.0)
