@@ -1,5 +1,5 @@
 // kvr_stream.cu -- the fused decode step for units too long for the staged
-// kernel of kvr_fused.cu (more than 128 live rows, up to kMaxRows): append +
+// kernel of kvr_fused.cu (more than its 160 live rows, up to kMaxRows): append +
 // Attn(q_t, C) (Eq. 1) + accumulated-attention update (Sec. 2.1) + eviction
 // of the single surplus row (TopB of Eq. 1 with the Sec. 4.1 window) +
 // in-place compaction, one CTA per (sequence, layer, KV head), K and V each
