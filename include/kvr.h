@@ -275,9 +275,17 @@ void kvr_fork_destroy(kvr_fork *fork);
  * else 4); 1 = candidate-batched (bf16, head_dim 128, G <= 8, N <= 8: a
  * warp per candidate, each prefix row read once per unit for all
  * candidates); 2 = chunked (one job per candidate and unit); 3 = one CTA per
- * unit; 4 = generic.  A choice that does not apply to a call runs the
- * generic kernel for that call.  Returns KVR_EINVAL outside [0, 4]. */
+ * unit; 4 = generic; 5 = candidate-batched on 5th-generation tensor cores
+ * (bf16, head_dim 128, G <= 8, N <= 8, at most 128 parent rows and 64 tail
+ * rows before the append: the N x G query rows of a unit are one
+ * contraction against each shared prefix block).  A choice that does not
+ * apply to a call runs the generic kernel for that call.  Returns
+ * KVR_EINVAL outside [0, 5]. */
 kvr_status kvr_fork_set_kernel(kvr_fork *fork, int kernel);
+
+/* The kernel (1..5, numbered as for kvr_fork_set_kernel) that ran the
+ * fork's last candidate step; 0 before the first step or for NULL. */
+int kvr_fork_last_kernel(const kvr_fork *fork);
 
 /* Bound, in nanoseconds, of each wait of the step kernels (fused,
  * chunked and streaming) on an asynchronous copy into shared memory for this

@@ -14,6 +14,7 @@
 #include <cstdio>
 #include <cstring>
 #include <string>
+#include <array>
 #include <vector>
 
 #include "../../include/kvr.h"
@@ -147,16 +148,36 @@ bool encode_slab(CUtensorMap *m, void *base, size_t rows, int R) {
 }
 
 // The N candidates' tails as one 3-D tensor {128 elements, units * tcap rows,
-// N candidates}: a box {64, T, N} fetches T rows of every candidate at once.
+// N candidates}: a box {64, T, Z} fetches T rows of Z candidates at once
+// (Z = N unless given).
 bool encode_tails3(CUtensorMap *m, void *base, size_t rows_per_cand, int n_cand,
-                   int T) {
+                   int T, int Z = 0) {
   auto fn = encode_tiled();
   if (!fn) return false;
   cuuint64_t dims[3] = {128, (cuuint64_t)rows_per_cand, (cuuint64_t)n_cand};
   cuuint64_t strides[2] = {256, (cuuint64_t)rows_per_cand * 256};
-  cuuint32_t box[3] = {64, (cuuint32_t)T, (cuuint32_t)n_cand};
+  cuuint32_t box[3] = {64, (cuuint32_t)T, (cuuint32_t)(Z ? Z : n_cand)};
   cuuint32_t estr[3] = {1, 1, 1};
   return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, base, dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// The N candidates' tails as a 4-D tensor {128 elements, nt rows, units, N}
+// (a unit's tail is tcap rows apart, a candidate's units * tcap): a box
+// {64, round_up16(nt), 1, min(N, 2)} fetches the first nt rows of one unit's
+// tails for two candidates and fills the rest of the box with zeros.
+bool encode_tails4(CUtensorMap *m, void *base, int nt, int tcap, size_t units,
+                   int n_cand) {
+  auto fn = encode_tiled();
+  if (!fn || nt < 1) return false;
+  cuuint64_t dims[4] = {128, (cuuint64_t)nt, (cuuint64_t)units, (cuuint64_t)n_cand};
+  cuuint64_t strides[3] = {256, (cuuint64_t)tcap * 256, (cuuint64_t)units * tcap * 256};
+  cuuint32_t box[4] = {64, (cuuint32_t)kvr::round_up16(nt), 1,
+                       (cuuint32_t)std::min(n_cand, 2)};
+  cuuint32_t estr[4] = {1, 1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, base, dims, strides, box,
             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
@@ -1133,7 +1154,12 @@ struct kvr_fork {
   CUtensorMap tmTK, tmTV;     // 16-row boxes
   bool batch_maps = false;    // 3-D tail maps (candidate-batched kernel)
   CUtensorMap tmTK3, tmTV3;
+  // Tail maps of the tensor-memory kernel, per tail length nt (encoded on
+  // first use): 0 not yet, 1 encoded, -1 cannot be encoded.
+  std::vector<signed char> tc_state;
+  std::vector<std::array<CUtensorMap, 2>> tc_tails;
   int kernel = 0;             // kvr_fork_set_kernel choice
+  int last_kernel = 0;        // the kernel that ran the last step (1..5)
 };
 
 namespace {
@@ -1245,6 +1271,8 @@ kvr_status kvr_fork_candidates(kvr_cache *p, int n_cand, int tail_cap,
         T > 0 &&
         encode_tails3(&f->tmTK3, v.TK, units * (size_t)tail_cap, n_cand, T) &&
         encode_tails3(&f->tmTV3, v.TV, units * (size_t)tail_cap, n_cand, T);
+    f->tc_state.assign(std::min(tail_cap, kvr::fork_tc_max_tail()) + 1, 0);
+    f->tc_tails.resize(f->tc_state.size());
   }
   p->forks += 1;
   *out = f;
@@ -1293,8 +1321,38 @@ kvr_status kvr_fork_decode_attend_score(kvr_fork *f, int lb, int le,
       nt_max = std::max(nt_max, f->tlen[(size_t)s * p->desc.n_layers + l]);
   const CacheView &pv = p->view;
   const std::pair<CUtensorMap, CUtensorMap> *maps = nullptr, *maps128 = nullptr;
-  const int want = p->fused ? f->kernel : 4;  // 0 auto, 1..4 one kernel
-  const bool batch_ok =
+  const int want = p->fused ? f->kernel : 4;  // 0 auto, 1..5 one kernel
+  // The tensor-memory kernel (chosen explicitly only: the candidate-batched
+  // kernel is faster at the sizes measured) wants every unit of the call at
+  // the same tail length (its tail maps end there).
+  bool nt_same = true;
+  for (int s = 0; s < p->desc.n_seq && nt_same; ++s)
+    for (int l = lb; l < le; ++l)
+      nt_same = nt_same && f->tlen[(size_t)s * p->desc.n_layers + l] == nt_max;
+  const CUtensorMap *tails = nullptr;
+  if (want == 5 && nt_same && (size_t)nt_max < f->tc_state.size()) {
+    signed char &st8 = f->tc_state[nt_max];
+    if (st8 == 0) {
+      const size_t units = (size_t)pv.S * pv.L * pv.H;
+      const int rows = std::max(nt_max, 1);
+      st8 = encode_tails4(&f->tc_tails[nt_max][0], f->view.TK, rows, f->view.tcap, units,
+                          f->view.N) &&
+                    encode_tails4(&f->tc_tails[nt_max][1], f->view.TV, rows, f->view.tcap,
+                                  units, f->view.N)
+                ? 1
+                : -1;
+    }
+    if (st8 == 1) tails = f->tc_tails[nt_max].data();
+  }
+  const bool tc_ok =
+      want == 5 && p->fused && tails && pv.G <= 8 &&
+      f->view.N <= kvr::fork_tc_max_cand() && device_facts(p) &&
+      kvr::fork_tc_smem_bytes() <= (size_t)p->smem_optin &&
+      max_prefix <= kvr::fork_tc_max_prefix() && nt_max <= kvr::fork_tc_max_tail() &&
+      (size_t)pv.S * pv.L * pv.H * pv.cap < (size_t)INT32_MAX &&
+      aligned16(q) && aligned16(k_new) && aligned16(v_new) && aligned16(out) &&
+      (maps = slab_maps(p, kvr::fork_tc_box_rows())) != nullptr;
+  const bool batch_ok = !tc_ok &&
       (want == 0 || want == 1) && p->fused && f->batch_maps && pv.G <= 8 &&
       f->view.N <= kvr::fork_batch_max_cand() && device_facts(p) &&
       kvr::fork_batch_smem_bytes(n_max, f->view.N) + 512 <=
@@ -1319,7 +1377,23 @@ kvr_status kvr_fork_decode_attend_score(kvr_fork *f, int lb, int le,
       (size_t)pv.S * pv.L * pv.H * pv.cap < (size_t)INT32_MAX &&
       aligned16(q) && aligned16(k_new) && aligned16(v_new) && aligned16(out) &&
       (maps = slab_maps(p, kvr::fork_mma_box_rows())) != nullptr;
-  if (batch_ok) {
+  if (tc_ok) {
+    kvr::ForkTcParams tp{};
+    tp.f = f->view;
+    tp.q = static_cast<const __nv_bfloat16 *>(q);
+    tp.k_new = static_cast<const __nv_bfloat16 *>(k_new);
+    tp.v_new = static_cast<const __nv_bfloat16 *>(v_new);
+    tp.out = out;
+    tp.lb = lb;
+    tp.nl = le - lb;
+    tp.scale_log2e = pv.scale * 1.4426950408889634f;
+    tp.inv_g = 1.f / (float)pv.G;
+    const int units = pv.S * (le - lb) * pv.H;
+    tp.nt = nt_max;
+    tp.np_max = max_prefix;
+    e = kvr::launch_fork_tc(maps->first, maps->second, &tails[0], &tails[1], tp,
+                            std::min(p->sm_count, units), as_stream(stream));
+  } else if (batch_ok) {
     kvr::ForkBatchParams bp{};
     bp.f = f->view;
     bp.q = static_cast<const __nv_bfloat16 *>(q);
@@ -1371,6 +1445,7 @@ kvr_status kvr_fork_decode_attend_score(kvr_fork *f, int lb, int le,
                                 as_stream(stream));
   }
   if (e != cudaSuccess) return cuda_fail("kvr_fork_decode_attend_score", e);
+  f->last_kernel = tc_ok ? 5 : batch_ok ? 1 : chunk_ok ? 2 : mma_ok ? 3 : 4;
   p->launches += 1;
   for (int s = 0; s < p->desc.n_seq; ++s)
     for (int l = lb; l < le; ++l) f->tlen[(size_t)s * p->desc.n_layers + l] += 1;
@@ -1465,10 +1540,12 @@ kvr_status kvr_fork_export(const kvr_fork *f, int cand, int seq,
   return KVR_OK;
 }
 
+int kvr_fork_last_kernel(const kvr_fork *f) { return f ? f->last_kernel : 0; }
+
 kvr_status kvr_fork_set_kernel(kvr_fork *f, int kernel) {
   if (!f) return fail(KVR_EINVAL, "null fork");
-  if (kernel < 0 || kernel > 4)
-    return fail(KVR_EINVAL, "fork kernel %d outside [0, 4]", kernel);
+  if (kernel < 0 || kernel > 5)
+    return fail(KVR_EINVAL, "fork kernel %d outside [0, 5]", kernel);
   f->kernel = kernel;
   return KVR_OK;
 }

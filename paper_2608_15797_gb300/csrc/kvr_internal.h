@@ -253,6 +253,32 @@ cudaError_t launch_fork_batch(const CUtensorMap &tmK, const CUtensorMap &tmV,
                               const ForkBatchParams &p, int grid,
                               cudaStream_t st);
 
+// Candidate step on 5th-generation tensor cores (kvr_fork_tc.cu): bf16,
+// d = 128, G <= 8, N <= fork_tc_max_cand(), at most fork_tc_max_prefix()
+// parent rows and fork_tc_max_tail() tail rows (before the append) per unit;
+// one persistent CTA per SM with two units in flight; every unit of the call
+// holds nt tail rows.  It takes the parent slab maps with
+// fork_tc_box_rows()-row boxes and the tails as 4-D maps {128, max(nt, 1),
+// units, N} (strides 256 B, tcap rows, units * tcap rows) with boxes {64,
+// nt rounded up to 16, 1, min(N, 2)}.
+struct ForkTcParams {
+  ForkView f;
+  const __nv_bfloat16 *q, *k_new, *v_new;  // [N][S][nl][...][128]
+  void *out;
+  int lb, nl;
+  int nt;      // tail rows before the append, the same in every unit
+  int np_max;  // largest prefix (parent rows) over the call's units
+  float scale_log2e, inv_g;
+};
+int fork_tc_max_cand();
+int fork_tc_max_prefix();
+int fork_tc_max_tail();
+int fork_tc_box_rows();
+size_t fork_tc_smem_bytes();
+cudaError_t launch_fork_tc(const CUtensorMap &tmK, const CUtensorMap &tmV,
+                           const CUtensorMap *tmTK, const CUtensorMap *tmTV,
+                           const ForkTcParams &p, int grid, cudaStream_t st);
+
 // Absorbing a chunk of tokens (kvr_absorb.cu): bf16, d = 128, G <= 8,
 // chunk <= absorb_max_chunk(), at most absorb_max_rows() rows after it.
 struct AbsorbParams {

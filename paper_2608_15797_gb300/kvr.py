@@ -79,6 +79,7 @@ _SIGS = {
     "kvr_cache_set_fused_tuning": (_S, [_P, _I, _I]),
     "kvr_cache_set_chunk_tuning": (_S, [_P, _I, _I]),
     "kvr_fork_set_kernel": (_S, [_P, _I]),
+    "kvr_fork_last_kernel": (_I, [_P]),
     "kvr_cache_set_absorb_kernel": (_S, [_P, _I]),
     "kvr_cache_scores": (_S, [_P, _P, _P, _P, _P]),
     "kvr_sync_status": (_S, [_P, _P]),
@@ -259,6 +260,10 @@ def kvr_cache_set_fused_tuning(h, groups: int, group_warps: int = 0):
 
 def kvr_fork_set_kernel(h, kernel: int):
     _check(lib.kvr_fork_set_kernel(h, kernel), "kvr_fork_set_kernel")
+
+
+def kvr_fork_last_kernel(h) -> int:
+    return int(lib.kvr_fork_last_kernel(h))
 
 
 def kvr_cache_set_chunk_tuning(h, groups: int, stages: int = 0):
@@ -521,7 +526,8 @@ class Fork:
     def __init__(self, cache: Cache, n_cand: int, tail_cap: int, stream=None,
                  kernel: int = 0, buf=None):
         """kernel: 0 the library's choice, 1 candidate-batched, 2 chunked,
-        3 one CTA per unit, 4 generic (kvr_fork_set_kernel).  buf: an
+        3 one CTA per unit, 4 generic, 5 candidate-batched on 5th-generation
+        tensor cores (kvr_fork_set_kernel).  buf: an
         optional caller-owned uint8 device tensor of at least
         kvr_fork_required_bytes."""
         self.cache, self.N, self.tcap = cache, n_cand, tail_cap
@@ -558,6 +564,10 @@ class Fork:
 
     def commit(self, chosen, budget, window, stream=None):
         kvr_fork_commit(self.handle, chosen, budget, window, stream)
+
+    def last_kernel(self) -> int:
+        """The kernel that ran the last candidate step (kvr_fork_last_kernel)."""
+        return kvr_fork_last_kernel(self.handle)
 
     def export(self, cand, seq, kv=False, stream=None):
         c = self.cache

@@ -164,12 +164,14 @@ def fork_lockstep(c: kvr.Cache, o: orc.OracleCache, w: inputs.Workload,
     candidate checking every candidate after every token (outputs; scores of
     every prefix and tail row, by position), then commit a seeded pick (the
     stand-in for the PRM argmax of Eq. 2) on both sides and check the parent.
-    Returns (oracle after commit, chosen, stats)."""
+    Returns (oracle after commit, chosen, stats); stats.kernels lists the
+    kernel that ran each token (kvr_fork_last_kernel)."""
     S = c.S
     parent_pos = [c.export(s, kv=False) for s in range(S)]
     f = guarded_fork(c, n_cand, tail_cap or steps, kernel=kernel)
     cands = o.fork(n_cand)
     stats = parity.Stats()
+    stats.kernels = []
     for t in range(steps):
         per = [inputs.step_inputs(w, seed, 10_000 + t, S, cand=k + 1)
                for k in range(n_cand)]
@@ -179,6 +181,7 @@ def fork_lockstep(c: kvr.Cache, o: orc.OracleCache, w: inputs.Workload,
                                      c.out_torch_dtype, owner=f)
         out = f.attend_score(dev(Q, w.dtype), dev(K, w.dtype), dev(V, w.dtype),
                              out=out_buf)
+        stats.kernels.append(f.last_kernel())
         torch.cuda.synchronize()
         out = out.float().cpu().numpy()
         for k in range(n_cand):
@@ -218,7 +221,9 @@ def fork_lockstep(c: kvr.Cache, o: orc.OracleCache, w: inputs.Workload,
         for name in ("K", "V", "score", "pos", "len", "next_pos"):
             getattr(committed, name)[s] = getattr(src, name)[s]
     exports = [c.export(s, kv=False) for s in range(S)]
+    kernels = stats.kernels
     stats.merge(parity.check_and_adopt(committed, exports, budget, window))
+    stats.kernels = kernels
     c.sync_status()
     check_guards(c, f)
     return committed, chosen, stats

@@ -24,9 +24,10 @@ def _cuda():
     torch.cuda.set_device(0)
 
 
-# The candidate kernels (kvr_fork_set_kernel): candidate-batched (the
-# default), chunked, one CTA per unit, generic.
-PATHS = {"batch": 1, "chunked": 2, "mma": 3, "generic": 4}
+# The candidate kernels (kvr_fork_set_kernel): candidate-batched on
+# 5th-generation tensor cores, candidate-batched on mma.sync (the default),
+# chunked, one CTA per unit, generic.
+PATHS = {"tc": 5, "batch": 1, "chunked": 2, "mma": 3, "generic": 4}
 
 
 def _evicted_pair(w, seed, S, cap, prompt_lens, warm_steps):
@@ -109,7 +110,7 @@ def test_single_candidate_equals_plain_deferred_eviction():
                     assert abs(ma[p] - mb[p]) <= 1e-4 * max(abs(mb[p]), 1e-6)
 
 
-@pytest.mark.parametrize("path", ["batch", "chunked", "mma"])
+@pytest.mark.parametrize("path", ["tc", "batch", "chunked", "mma"])
 def test_7b_best_of_4(path):
     """7B geometry stepwise best-of-4: an evicted cache (prompt 512, B=128,
     W=8; heavy keys), forked to 4 candidates that decode a 16-token step
@@ -122,7 +123,7 @@ def test_7b_best_of_4(path):
     assert (c.lengths() == w.budget + w.window).all()
 
 
-@pytest.mark.parametrize("path", ["batch", "chunked"])
+@pytest.mark.parametrize("path", ["tc", "batch", "chunked"])
 def test_72b_best_of_8(path):
     """72B geometry (80 layers, 8 KV heads, G=8), B=64, N=8 candidates, an
     8-token step (reduced from 64 to keep the oracle fast)."""
@@ -130,12 +131,13 @@ def test_72b_best_of_8(path):
                         sigma=1.0 / np.sqrt(128.0))
     c, o = _evicted_pair(w, 26, 1, cap=w.prompt + 1, prompt_lens=[w.prompt],
                          warm_steps=1)
-    harness.fork_lockstep(c, o, w, 26, 8, 8, w.budget, w.window,
-                          kernel=PATHS[path])
+    _, _, st = harness.fork_lockstep(c, o, w, 26, 8, 8, w.budget, w.window,
+                                     kernel=PATHS[path])
     assert (c.lengths() == w.budget + w.window).all()
+    assert st.kernels == [PATHS[path]] * 8
 
 
-@pytest.mark.parametrize("path", ["batch", "chunked"])
+@pytest.mark.parametrize("path", ["tc", "batch", "chunked"])
 def test_fork_empty_prefix_and_block_edges(path):
     """A parent with no live rows (an empty prefix) and one whose prefix is
     an exact multiple of the 32-row chunk, with 2 and 3 candidates (tail
@@ -155,3 +157,51 @@ def test_fork_prefix_longer_than_a_block():
     c, o = harness.make_pair(w, 28, 1, cap=240, prompt_lens=[200])
     harness.fork_lockstep(c, o, w, 28, 4, 12, w.budget, w.window,
                           kernel=PATHS["batch"])
+
+
+@pytest.mark.parametrize("n_cand,G,lens,steps,out", [
+    (8, 8, [72, 72], 64, "bf16"),   # the benchmarked shape: tails up to 64 rows
+    (3, 3, [16, 5], 20, "f32"),     # ragged prefixes, G < 8 (padding rows)
+    (1, 7, [128, 1], 17, "f32"),    # the longest prefix, and a 1-row one
+    (5, 8, [0, 33], 5, "bf16"),     # an empty prefix
+    (8, 1, [100, 64], 33, "f32"),   # G = 1
+    (2, 5, [47, 80], 49, "bf16"),   # odd prefix and tail lengths
+])
+def test_tc_fork_shapes(n_cand, G, lens, steps, out):
+    """The tensor-memory candidate kernel across candidate counts, group
+    sizes, prefix lengths (0 to its 128-row limit; partial 16-row boxes) and
+    tail lengths (partial and whole 16-row pieces, up to its 64-row limit),
+    with both output types; every token must run on it."""
+    w = inputs.Workload("ft", 2, 2, G, 128, "bf16", 12, 4, 0, 0, sigma=1.0)
+    # the oracle's candidates are copies that keep every row until the commit
+    c, o = harness.make_pair(w, 30, 2, cap=max(lens) + steps + 1,
+                             prompt_lens=lens, out_dtype=out)
+    _, _, st = harness.fork_lockstep(c, o, w, 30, n_cand, steps, w.budget,
+                                     w.window, kernel=5)
+    assert st.kernels == [5] * steps
+
+
+def test_tc_fork_many_units_per_cta():
+    """384 units (3 sequences x 16 layers x 8 KV heads) with ragged
+    prefixes, so every persistent CTA takes several units through both of
+    its unit slots and its ring and head buffers wrap many times."""
+    w = inputs.Workload("ftm", 16, 8, 4, 128, "bf16", 12, 4, 0, 0, sigma=1.0)
+    c, o = harness.make_pair(w, 31, 3, cap=128 + 18 + 1,
+                             prompt_lens=[72, 30, 128], out_dtype="bf16")
+    _, _, st = harness.fork_lockstep(c, o, w, 31, 4, 18, w.budget, w.window,
+                                     kernel=5)
+    assert st.kernels == [5] * 18
+
+
+def test_tc_fork_falls_back_past_its_limits():
+    """A prefix of 129 rows or a tail past 64 rows is outside the tensor-
+    memory kernel: those steps run another kernel, with the same results."""
+    w = inputs.Workload("ftl", 1, 2, 4, 128, "bf16", 12, 4, 0, 0, sigma=1.0)
+    c, o = harness.make_pair(w, 32, 1, cap=133, prompt_lens=[129])
+    _, _, st = harness.fork_lockstep(c, o, w, 32, 2, 3, w.budget, w.window,
+                                     kernel=5)
+    assert 5 not in st.kernels
+    c, o = harness.make_pair(w, 33, 1, cap=108, prompt_lens=[40])
+    _, _, st = harness.fork_lockstep(c, o, w, 33, 2, 67, w.budget, w.window,
+                                     kernel=5)
+    assert st.kernels[:65] == [5] * 65 and 5 not in st.kernels[65:]
