@@ -68,9 +68,11 @@ __device__ __forceinline__ void cp_async_commit_wait_all() {
 
 // Byte offset of 16-byte piece ch (0..15: columns 8ch..8ch+7) of row r
 // within a K or V area: two 64-column halves of kRows rows, 128B swizzle.
-__device__ __forceinline__ uint32_t swz(int r, int ch) {
-  return (ch >> 3) * kMaxRows * 128 + r * 128 + (((ch & 7) ^ (r & 7)) << 4);
+template <int kRows>
+__device__ __forceinline__ uint32_t swzr(int r, int ch) {
+  return (ch >> 3) * kRows * 128 + r * 128 + (((ch & 7) ^ (r & 7)) << 4);
 }
+__device__ __forceinline__ uint32_t swz(int r, int ch) { return swzr<kMaxRows>(r, ch); }
 
 struct AbsorbSmem {
   static constexpr int k = 0;                          // [2][kMaxRows][128 B]
@@ -101,7 +103,8 @@ struct UnitSmem {
   int *kept;
 };
 
-__device__ __forceinline__ bool unit_begin(const AbsorbParams &p, Unit &u) {
+__device__ __forceinline__ bool unit_begin(const AbsorbParams &p, Unit &u,
+                                           int max_rows = kMaxRows) {
   const CacheView &c = p.c;
   const int idx = blockIdx.x;
   u.h = idx % c.H;
@@ -111,7 +114,7 @@ __device__ __forceinline__ bool unit_begin(const AbsorbParams &p, Unit &u) {
   u.n0 = c.state[4 * u.ug];
   u.t0 = c.state[4 * u.ug + 1];
   u.n = u.n0 + p.chunk;
-  if (u.n0 < 0 || u.n > kMaxRows || u.n > c.cap) {
+  if (u.n0 < 0 || u.n > max_rows || u.n > c.cap) {
     if (threadIdx.x == 0) atomicOr(c.err, u.n > c.cap ? ERR_CAPACITY : ERR_LENGTH);
     return false;
   }
@@ -122,8 +125,10 @@ __device__ __forceinline__ bool unit_begin(const AbsorbParams &p, Unit &u) {
   return true;
 }
 
-// Rows [0, n0) from the slab, rows n0 + j from the chunk's new k/v; scores,
-// positions and zeroed increments.  Ends with the CTA synchronised.
+// Rows [0, n0) from the slab, rows n0 + j from the chunk's new k/v (K and V
+// areas of kRows rows per 64-column half); scores, positions and zeroed
+// increments.  Ends with the CTA synchronised.
+template <int kRows = kMaxRows>
 __device__ void load_unit(const AbsorbParams &p, const Unit &u,
                           const UnitSmem &m) {
   const CacheView &c = p.c;
@@ -140,14 +145,14 @@ __device__ void load_unit(const AbsorbParams &p, const Unit &u,
       ks = p.k_new + kr * 128;
       vs = p.v_new + kr * 128;
     }
-    cp_async16(sK + swz(r, ch), ks + ch * 8);
-    cp_async16(sV + swz(r, ch), vs + ch * 8);
+    cp_async16(sK + swzr<kRows>(r, ch), ks + ch * 8);
+    cp_async16(sV + swzr<kRows>(r, ch), vs + ch * 8);
   }
   // V rows past n up to the end of their 16-row tile are read by PV with a
   // zero probability; zero them so stale bits (NaN) cannot leak in.
   for (int i = tid; i < (((n + 15) & ~15) - n) * 16; i += kThreads) {
     const int r = n + (i >> 4), ch = i & 15;
-    *reinterpret_cast<int4 *>(m.v + swz(r, ch)) = make_int4(0, 0, 0, 0);
+    *reinterpret_cast<int4 *>(m.v + swzr<kRows>(r, ch)) = make_int4(0, 0, 0, 0);
   }
   for (int r = tid; r < n; r += kThreads) {
     m.sc[r] = r < n0 ? u.su[r] : 0.f;
@@ -158,7 +163,9 @@ __device__ void load_unit(const AbsorbParams &p, const Unit &u,
   __syncthreads();
 }
 
-// Scores, the TopB cut and compaction, then the unit's state.
+// Scores, the TopB cut and compaction, then the unit's state (K and V areas
+// and row lists of kRows rows).
+template <int kRows = kMaxRows>
 __device__ void finish_unit(const AbsorbParams &p, const Unit &u,
                             const UnitSmem &m, int *s_base, int *s_count,
                             int *s_wsum) {
@@ -203,7 +210,7 @@ __device__ void finish_unit(const AbsorbParams &p, const Unit &u,
     if (tid == 0) atomicOr(c.err, ERR_LENGTH);
     return;
   }
-  int *holes = m.lists, *movers = m.lists + kMaxRows;
+  int *holes = m.lists, *movers = m.lists + kRows;
   const int nh = dev::block_collect(0, nk, [&](int i) { return !keep(i); }, holes,
                                     s_wsum, s_base);
   const int nm = dev::block_collect(nk, n, keep, movers, s_wsum, s_base);
@@ -217,7 +224,7 @@ __device__ void finish_unit(const AbsorbParams &p, const Unit &u,
   const uint32_t sK = smem_u32(m.k), sV = smem_u32(m.v);
   auto write_row = [&](int src, int dst, int ln) {  // one warp-lane share
     const int ch = ln & 15;
-    const uint32_t from = (ln < 16 ? sK : sV) + swz(src, ch);
+    const uint32_t from = (ln < 16 ? sK : sV) + swzr<kRows>(src, ch);
     int4 val;
     asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
                  : "=r"(val.x), "=r"(val.y), "=r"(val.z), "=r"(val.w)
@@ -437,63 +444,102 @@ __global__ void __launch_bounds__(kThreads)
 
 // ---- the same absorb on 5th-generation tensor cores ------------------------
 //
+// Units of at most kTcMaxRows rows after the chunk, two CTAs an SM (about
+// 111 KB of shared memory and 256 tensor-memory columns each), so that one
+// unit's loads, selection and stores overlap the other's tensor work.
 // Query rows go in tiles of 128 (M), with the unit's keys as N (rows
 // rounded up to 16) and K = the head dimension.  Per tile:
-//   1. The tile's q rows are in shared memory (K-major, 128B swizzle, in the
-//      P lo buffer: loaded with the unit for the first tile, during the
-//      previous tile's output phase for the others) and one thread issues
-//      S = Q K^T into TMEM (fp32, N columns).
-//   2. Every warp reads its rows' logits from TMEM; warps w and w + 4 share
-//      TMEM lanes 32 (w % 4).. and take half the columns each.  They form the
-//      row statistics (an exchange through shared memory), then the exact
-//      probabilities, written as bf16 hi and lo terms into two P buffers
-//      (K-major, 128B swizzle: [64-key block][query row][128 B]).
-//   3. One thread issues O = P_hi V + P_lo V (V read MN-major) and the
-//      score column sums CS = P_hi^T 1 + P_lo^T 1 (the same P buffers read as
-//      an MN-major A operand, M = keys in 128-key tiles, K = the tile's query
-//      rows, N = 16 columns of ones) into TMEM.
-//      CS accumulates over the unit's tiles.
-//   4. The warps write their rows' outputs from TMEM.
-// After the last tile thread t adds the sum of key t (TMEM lane t % 128 of
-// key tile t / 128), times 1/G, to the unit's score increments.
-// Every mbarrier wait is bounded; TMEM is freed before the selection.
+//   1. The tile's q rows are in shared memory (K-major, 128B swizzle; the
+//      next tile's are fetched once this tile's S is done) and one thread
+//      issues S = Q K^T into tensor memory (fp32, N columns).
+//   2. Every warp reads its rows' logits from tensor memory; warps w and
+//      w + 4 share TMEM lanes 32 (w % 4).. and take half the columns each.
+//      They form the row statistics (an exchange through shared memory),
+//      then the exact probabilities: P in place of the logits (each 16-key
+//      chunk's 16 columns take its 8 hi and 8 lo columns of bf16 pairs, the
+//      A operand of PV), and their column sums over the tile's rows (a
+//      butterfly over the warp's 32 rows, then shared-memory atomics) for
+//      the scores.
+//   3. O = P_hi V + P_lo V one 64-column half of the head dimension at a
+//      time (64 tensor-memory columns), each half stored from tensor memory
+//      before the next is computed.
+// Every mbarrier wait is bounded; tensor memory is freed before the
+// selection.
+constexpr int kTcMaxRows = 144;                    // rows this kernel stages
 constexpr int kTcRows = 128;                       // query rows per tile
-constexpr int kTcS = 0;                            // TMEM columns: S
-constexpr int kTcO = kMaxRows;                     //               O
-constexpr int kTcCS = kMaxRows + 128;              //               CS
-constexpr int kTcCsTiles = (kMaxRows + 127) / 128;  // 128-key tiles of CS
-constexpr int kTcCols = 512;
-constexpr int kTcChunks = (kMaxRows / 2 + 15) / 16;  // a thread's column chunks
-static_assert(kTcCS + 16 * kTcCsTiles <= kTcCols, "TMEM columns");
-static_assert(kTcCsTiles * 128 <= 2 * kTcRows, "one key of CS a thread");
+constexpr uint32_t kTcS = 0;                       // TMEM columns: S / P
+constexpr uint32_t kTcO = kTcMaxRows;              //   O, one 64-column half
+constexpr int kTcCols = 256;
+constexpr int kTcChunks = (kTcMaxRows / 2 + 15) / 16;  // a thread's column chunks
+static_assert(kTcO + 64 <= kTcCols, "TMEM columns");
+static_assert(kTcMaxRows % 16 == 0, "whole 16-key chunks");
 
 struct TcSmem {  // offsets from a 1024-byte aligned base
-  static constexpr int k = 0;                              // [2][kMaxRows][128 B]
-  static constexpr int v = k + 2 * kMaxRows * 128;
-  static constexpr int ph = v + 2 * kMaxRows * 128;        // [3][128][128 B]
-  static constexpr int pl = ph + 3 * kTcRows * 128;
-  static constexpr int q = pl;                             // [2][128][128 B], aliases P lo
-  static constexpr int ones = pl + 3 * kTcRows * 128;      // [16][128 B] of 1.0
-  static constexpr int sc = ones + 16 * 128;
-  static constexpr int ps = sc + 4 * kMaxRows;
-  static constexpr int acc = ps + 4 * kMaxRows;
-  static constexpr int lists = acc + 4 * kMaxRows;
-  static constexpr int key = lists + 8 * kMaxRows;
-  static constexpr int kept = key + 8 * kMaxRows;
-  static constexpr int end = kept + 4 * kMaxRows;
-  // The last CS key tile reads P blocks up to 2 kTcCsTiles - 1: past the
-  // three P hi blocks lies P lo, past P lo the ones and the lists (rows of
-  // keys >= NS, never read back), so the buffer reaches that far.
-  static constexpr int cs_end = pl + 2 * kTcCsTiles * kTcRows * 128;
-  static constexpr int bytes = end > cs_end ? end : cs_end;
+  static constexpr int k = 0;                              // [2][kTcMaxRows][128 B]
+  static constexpr int v = k + 2 * kTcMaxRows * 128;
+  static constexpr int q = v + 2 * kTcMaxRows * 128;       // [2][128][128 B]
+  static constexpr int sc = q + 2 * kTcRows * 128;
+  static constexpr int ps = sc + 4 * kTcMaxRows;
+  static constexpr int acc = ps + 4 * kTcMaxRows;
+  static constexpr int lists = acc + 4 * kTcMaxRows;
+  static constexpr int key = lists + 8 * kTcMaxRows;       // also the (max, sum) exchange
+  static constexpr int kept = key + 8 * kTcMaxRows;
+  static constexpr int part = kept + 4 * kTcMaxRows;        // [4][kTcMaxRows] column sums
+  static constexpr int bytes = part + 16 * kTcMaxRows;
   static constexpr int alloc = bytes + 1024;               // room to align
 };
-static_assert(TcSmem::alloc <= 227 * 1024, "shared memory per CTA");
-static_assert(3 * 64 >= kMaxRows, "P holds kMaxRows keys in 64-key blocks");
-static_assert(TcSmem::cs_end <= TcSmem::bytes, "CS key tiles stay in the buffer");
+static_assert(8 * kTcMaxRows >= 8 * kTcRows, "the exchange fits in the key area");
+// Two CTAs an SM: 228 KB less 1 KB reserved per CTA, with room for the
+// static variables.
+static_assert(TcSmem::alloc + 512 <= 113 * 1024, "two CTAs an SM");
+
+// Column sums of v[16] (this lane's row) over the warp's 32 rows: after the
+// butterfly, lane l holds the sum of column (l >> 1) & 15... in the order
+// below; both lanes of a pair hold the same value.  Returns the column.
+__device__ __forceinline__ float colsum32(const float (&v)[16], int lane, int &col) {
+  float a[8], b[4], cc[2];
+  const bool b4 = (lane & 16) != 0, b3 = (lane & 8) != 0, b2 = (lane & 4) != 0,
+             b1 = (lane & 2) != 0;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const float send = b4 ? v[i] : v[i + 8], keep = b4 ? v[i + 8] : v[i];
+    a[i] = keep + __shfl_xor_sync(0xffffffffu, send, 16);
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float send = b3 ? a[i] : a[i + 4], keep = b3 ? a[i + 4] : a[i];
+    b[i] = keep + __shfl_xor_sync(0xffffffffu, send, 8);
+  }
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    const float send = b2 ? b[i] : b[i + 2], keep = b2 ? b[i + 2] : b[i];
+    cc[i] = keep + __shfl_xor_sync(0xffffffffu, send, 4);
+  }
+  const float send = b1 ? cc[0] : cc[1], keep = b1 ? cc[1] : cc[0];
+  float x = keep + __shfl_xor_sync(0xffffffffu, send, 2);
+  x += __shfl_xor_sync(0xffffffffu, x, 1);
+  col = (b4 ? 8 : 0) + (b3 ? 4 : 0) + (b2 ? 2 : 0) + (b1 ? 1 : 0);
+  return x;
+}
+
+__device__ __forceinline__ void mma_ts_all(uint32_t d, uint32_t a, uint64_t b, uint32_t id,
+                                           bool acc) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d),
+      "r"(a), "l"(b), "r"(id), "r"(acc ? 1 : 0)
+      : "memory");
+}
+__device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&v)[8]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"r"(taddr),
+      "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]),
+      "r"(v[7])
+      : "memory");
+}
 
 template <bool kOutBf16>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kThreads, 2)
     absorb_tc_kernel(const AbsorbParams p) {
   pdl_begin();
   extern __shared__ __align__(1024) unsigned char smem_raw[];
@@ -502,13 +548,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   __shared__ uint32_t s_tmem;
   __shared__ int s_abort;
   __shared__ __align__(8) uint64_t bar_s, bar_o;
-  __shared__ float2 s_ml[kTcRows];  // (max, sum) of the upper column halves
   unsigned char *smem = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
   const CacheView &c = p.c;
   const int G = c.G, C = p.chunk;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   Unit u;
-  if (!unit_begin(p, u)) return;
+  if (!unit_begin(p, u, kTcMaxRows)) return;
   const UnitSmem m{smem + TcSmem::k,
                    smem + TcSmem::v,
                    reinterpret_cast<float *>(smem + TcSmem::sc),
@@ -517,6 +562,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                    reinterpret_cast<int *>(smem + TcSmem::lists),
                    reinterpret_cast<unsigned long long *>(smem + TcSmem::key),
                    reinterpret_cast<int *>(smem + TcSmem::kept)};
+  float2 *s_ml = reinterpret_cast<float2 *>(smem + TcSmem::key);  // free until the selection
   if (warp == 0) tmem_alloc(smem_u32(&s_tmem), kTcCols);
   if (tid == 32) {
     mbar_init(smem_u32(&bar_s), 1);
@@ -524,8 +570,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     s_abort = 0;
     fence_mbar_init();
   }
-  for (int i = tid; i < 16 * 128 / 4; i += kThreads)  // bf16 1.0 pairs
-    reinterpret_cast<uint32_t *>(smem + TcSmem::ones)[i] = 0x3F803F80u;
   const int n = u.n, n0 = u.n0, h = u.h;
   const int MQ = C * G, n_mt = (MQ + kTcRows - 1) / kTcRows;
   const uint32_t aQ = smem_u32(smem + TcSmem::q);
@@ -554,29 +598,55 @@ __global__ void __launch_bounds__(kThreads, 1)
   };
   load_q(0);
   tc_fence_before();
-  load_unit(p, u, m);  // ends with the copies complete and __syncthreads
+  load_unit<kTcMaxRows>(p, u, m);  // ends with the copies complete and __syncthreads
   tc_fence_after();
   const uint32_t tm = s_tmem;
-  const int NS = (n + 15) & ~15;
-  const uint32_t id_s = idesc_bf16(kTcRows, NS, false);
-  const uint32_t id_o = idesc_bf16(kTcRows, 128, true);
-  const uint32_t id_c = idesc_bf16(128, 16, false, true);
-  const int n_ct = (NS + 127) >> 7;  // 128-key tiles of CS
   const uint32_t aK = smem_u32(m.k), aV = smem_u32(m.v);
-  const uint32_t aPH = smem_u32(smem + TcSmem::ph), aPL = smem_u32(smem + TcSmem::pl);
-  const uint32_t aOnes = smem_u32(smem + TcSmem::ones);
   const int wq = warp & 3;             // TMEM lane quarter of this warp
-  const bool upper = warp >= 4;        // second half of the columns
-  const int half = ((NS >> 1) + 15) & ~15;
-  const int c_lo = upper ? half : 0, c_hi = upper ? NS : half;
+  const bool upper = warp >= 4;        // second half of the tile's columns
   const int r = wq * 32 + lane;        // this thread's row of the tile
   const uint32_t trow = tm + ((uint32_t)(wq * 32) << 16);
   const float scale = p.scale_log2e, inv_g = p.inv_g;
+  float *ACC = m.acc;
+  float *PART = reinterpret_cast<float *>(smem + TcSmem::part);
   volatile int *abort = &s_abort;
+  // Keys that rows 32 q4 .. 32 q4 + 31 of tile mt may see: the causal
+  // limit of the last of them (row R is token R / G of the chunk), 0 when
+  // they are all past MQ.
+  auto lim_warp = [&](int mt, int q4) {
+    const int R0 = mt * kTcRows + 32 * q4;
+    if (R0 >= MQ) return 0;
+    return n0 + (min(R0 + 32, MQ) - 1) / G + 1;
+  };
+  // Columns of S tile mt: its keys rounded up to whole 16-key chunks
+  // (P is zero past the last row's limit, so no MMA reads further).
+  auto tile_cols = [&](int mt) {  // every tile has at least one row below MQ
+    return (n0 + (min(mt * kTcRows + kTcRows, MQ) - 1) / G + 1 + 15) & ~15;
+  };
+  auto issue_s = [&](int mt) {  // one thread
+    const uint32_t id_s = idesc_bf16(kTcRows, tile_cols(mt), false);
+    for (int k = 0; k < 8; ++k) {  // K = 128 head-dim columns, 16 a step
+      const uint32_t off = (k & 3) * 32;
+      tc_mma(tm + kTcS, sdesc_sw128(aQ + (k >> 2) * (kTcRows * 128) + off, 16, 1024),
+             sdesc_sw128(aK + (k >> 2) * (kTcMaxRows * 128) + off, 16, 1024), id_s, k > 0);
+    }
+    tc_commit(smem_u32(&bar_s));
+  };
+  const uint32_t id_o = idesc_bf16(kTcRows, 64, true);
+  auto issue_pv = [&](int hd, int NSt) {  // one thread: O half hd = P V[:, 64 hd ..]
+    for (int k = 0; k < NSt / 16; ++k) {  // K = keys, 16 a step
+      const uint64_t bv =
+          sdesc_sw128(aV + hd * (kTcMaxRows * 128) + k * 2048, kTcMaxRows * 128, 1024);
+      mma_ts_all(tm + kTcO, tm + kTcS + 16 * k, bv, id_o, k > 0);
+      mma_ts_all(tm + kTcO, tm + kTcS + 16 * k + 8, bv, id_o, true);
+    }
+    tc_commit(smem_u32(&bar_o));
+  };
   bool ok = true;
-  int phase = 0;
-  auto wait_all = [&](uint64_t *bar) {
-    const bool got = mbar_wait(smem_u32(bar), (uint32_t)(phase & 1), abort);
+  int ph_s = 0, ph_o = 0;
+  auto wait_all = [&](uint64_t *bar, int &ph) {
+    const bool got = mbar_wait(smem_u32(bar), (uint32_t)(ph & 1), abort);
+    ph ^= 1;
     const bool all = __syncthreads_and(got) != 0;
     if (!all && tid == 0) {
       atomicOr(c.err, ERR_TIMEOUT);
@@ -585,43 +655,39 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     return all;
   };
-  for (int mt = 0; mt < n_mt && ok; ++mt, ++phase) {
-    // 1. The tile's q rows have landed (issued earlier).
-    cp_async_commit_wait_all();
-    fence_proxy_async();
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    if (tid == 0) {
-      for (int k = 0; k < 8; ++k) {  // K = 128 head-dim columns, 16 a step
-        const uint32_t off = (k & 3) * 32;
-        tc_mma(tm + kTcS,
-               sdesc_sw128(aQ + (k >> 2) * (kTcRows * 128) + off, 16, 1024),
-               sdesc_sw128(aK + (k >> 2) * (kMaxRows * 128) + off, 16, 1024),
-               id_s, k > 0);
-      }
-      tc_commit(smem_u32(&bar_s));
-    }
-    if (!(ok = wait_all(&bar_s))) break;
+  // Tile 0's q rows have landed (the unit load ended with a barrier after
+  // every thread's copies completed).
+  fence_proxy_async();
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (tid == 0) issue_s(0);
+  for (int mt = 0; mt < n_mt && ok; ++mt) {
+    // 1. S = Q K^T for the tile's keys is in tensor memory.
+    if (!(ok = wait_all(&bar_s, ph_s))) break;
+    if (mt + 1 < n_mt) load_q(mt + 1);  // S has read this tile's q rows
+    const int NSt = tile_cols(mt);
+    const int half = ((NSt >> 1) + 15) & ~15;
+    const int c_lo = upper ? half : 0, c_hi = upper ? NSt : half;
+    const int nch = (c_hi - c_lo) >> 4;
+    const int lim_w = lim_warp(mt, wq);  // warp-uniform: chunks from here on are all masked
 
     // 2. This thread's logits (at most kTcChunks 16-column chunks) read
-    // from TMEM once, exponentiated once against the thread's own maximum;
-    // the row's maximum and sum come from an exchange with the partner warp,
-    // and the probabilities are the thread's terms rescaled.
+    // from TMEM once, exponentiated against the thread's own maximum; the
+    // row's maximum and sum come from an exchange with the partner warp.
     const int R = mt * kTcRows + r;
     const bool valid = R < MQ;
     const int lim = valid ? n0 + R / G + 1 : 0;  // keys the row may see
-    const int nch = (c_hi - c_lo) >> 4;
     float e[kTcChunks][16];
     float mx = -INFINITY;
 #pragma unroll
     for (int k = 0; k < kTcChunks; ++k)
-      if (k < nch) tmem_ld16f_nowait(trow + kTcS + c_lo + 16 * k, e[k]);
+      if (k < nch && c_lo + 16 * k < lim_w) tmem_ld16f_nowait(trow + kTcS + c_lo + 16 * k, e[k]);
     tmem_wait_ld();
     const uint64_t scale2 = pk2(scale, scale);
 #pragma unroll
     for (int k = 0; k < kTcChunks; ++k) {
-      if (k < nch) {
+      if (k < nch && c_lo + 16 * k < lim_w) {
         if (c_lo + 16 * k + 16 <= lim) {  // the whole chunk is visible
 #pragma unroll
           for (int j = 0; j < 16; j += 2) {
@@ -643,7 +709,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t sm2 = pk2(0.f, 0.f);  // even and odd terms
 #pragma unroll
     for (int k = 0; k < kTcChunks; ++k) {
-      if (k < nch) {
+      if (k < nch && c_lo + 16 * k < lim_w) {
 #pragma unroll
         for (int j = 0; j < 16; j += 2) {
           float d0, d1;
@@ -660,8 +726,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       upk2(sm2, s0, s1);
       sm = s0 + s1;
     }
+    // Warps w and w + 4 (the same 32 rows) exchange (max, sum) through
+    // shared memory on a named barrier of their own.
+    const uint32_t bar_id = 1 + wq;
     if (upper) s_ml[r] = make_float2(mx, sm);
-    __syncthreads();
+    asm volatile("bar.sync %0, 64;" ::"r"(bar_id) : "memory");
     float M = mx, L = sm;
     if (!upper) {
       const float2 o2 = s_ml[r];
@@ -670,77 +739,68 @@ __global__ void __launch_bounds__(kThreads, 1)
           (o2.x == -INFINITY ? 0.f : o2.y * ex2(o2.x - M));
       s_ml[r] = make_float2(M, L);
     }
-    __syncthreads();
+    asm volatile("bar.sync %0, 64;" ::"r"(bar_id) : "memory");
     if (upper) {
       const float2 o2 = s_ml[r];
       M = o2.x;
       L = o2.y;
     }
     if (valid && !upper && !(L >= 1.f && L < INFINITY)) atomicOr(c.err, ERR_NONFINITE);
-    // p = e * exp2(own max - row max) / row sum
+    // p = e * exp2(own max - row max) / row sum; rows past the tile's
+    // queries have f = 0 and finite e, so exact zeros.
     const float f = valid && L > 0.f && mx > -INFINITY ? ex2(mx - M) / L : 0.f;
     const uint64_t f2 = pk2(f, f);
 #pragma unroll
     for (int k = 0; k < kTcChunks; ++k) {
-      if (k < nch) {
-        const int c0 = c_lo + 16 * k;
-        uint32_t hi[8], lo[8];
+      if (k >= nch) continue;
+      const uint32_t cp = trow + kTcS + c_lo + 16 * k;
+      uint32_t hi[8], lo[8];
+      if (c_lo + 16 * k < lim_w) {
 #pragma unroll
         for (int j = 0; j < 16; j += 2) {
           const uint64_t p2 = mul2(pk2(e[k][j], e[k][j + 1]), f2);
           float p0, p1;
           upk2(p2, p0, p1);
+          e[k][j] = p0;
+          e[k][j + 1] = p1;
           const __nv_bfloat162 b = __floats2bfloat162_rn(p0, p1);
           hi[j >> 1] = *reinterpret_cast<const uint32_t *>(&b);
           float r0, r1;  // p - bf16(p), both terms at once
           upk2(add2(p2, pk2(-__low2float(b), -__high2float(b))), r0, r1);
           lo[j >> 1] = pack_bf16(r0, r1);
         }
-        const int kb = c0 >> 6, ch = (c0 & 63) >> 3;
-        const uint32_t o0 = kb * (kTcRows * 128) + r * 128 + (((ch) ^ (r & 7)) << 4);
-        const uint32_t o1 = kb * (kTcRows * 128) + r * 128 + (((ch + 1) ^ (r & 7)) << 4);
-        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(aPH + o0), "r"(hi[0]),
-                     "r"(hi[1]), "r"(hi[2]), "r"(hi[3]) : "memory");
-        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(aPH + o1), "r"(hi[4]),
-                     "r"(hi[5]), "r"(hi[6]), "r"(hi[7]) : "memory");
-        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(aPL + o0), "r"(lo[0]),
-                     "r"(lo[1]), "r"(lo[2]), "r"(lo[3]) : "memory");
-        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(aPL + o1), "r"(lo[4]),
-                     "r"(lo[5]), "r"(lo[6]), "r"(lo[7]) : "memory");
+        // P in place of the chunk's logits: 8 hi then 8 lo columns.
+        tmem_st8(cp, hi);
+        tmem_st8(cp + 8, lo);
+        // The chunk's column sums over the warp's 32 rows, one slot per
+        // lane quarter (summed in a fixed order below).
+        int col;
+        const float cs = colsum32(e[k], lane, col);
+        if ((lane & 1) == 0) PART[wq * kTcMaxRows + c_lo + 16 * k + col] = cs;
+      } else {  // every row of the warp is masked here: P = 0
+#pragma unroll
+        for (int j = 0; j < 8; ++j) hi[j] = 0u;
+        tmem_st8(cp, hi);
+        tmem_st8(cp + 8, hi);
       }
     }
-    fence_proxy_async();
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
 
-    // 3. O = P V and the column sums CS = P^T 1, hi and lo terms each.
-    if (tid == 0) {
-      for (int k = 0; k < NS / 16; ++k) {  // K = keys, 16 a step
-        const uint32_t pa = (k >> 2) * (kTcRows * 128) + (k & 3) * 32;
-        const uint64_t bv = sdesc_sw128(aV + k * 2048, kMaxRows * 128, 1024);
-        tc_mma(tm + kTcO, sdesc_sw128(aPH + pa, 16, 1024), bv, id_o, k > 0);
-        tc_mma(tm + kTcO, sdesc_sw128(aPL + pa, 16, 1024), bv, id_o, true);
-      }
-      for (int t = 0; t < n_ct; ++t) {  // M = 128 keys (two 64-key P blocks)
-        const uint32_t pb = t * 2 * (kTcRows * 128);
-        for (int k = 0; k < kTcRows / 16; ++k) {  // K = the tile's query rows
-          const uint64_t bo = sdesc_sw128(aOnes + (k & 3) * 32, 16, 1024);
-          tc_mma(tm + kTcCS + 16 * t,
-                 sdesc_sw128(aPH + pb + k * 2048, kTcRows * 128, 1024), bo, id_c,
-                 mt > 0 || k > 0);
-          tc_mma(tm + kTcCS + 16 * t,
-                 sdesc_sw128(aPL + pb + k * 2048, kTcRows * 128, 1024), bo, id_c,
-                 true);
-        }
-      }
-      tc_commit(smem_u32(&bar_o));
+    // 3. O = P V, one 64-column half of the head dimension at a time:
+    // P (hi and lo) from tensor memory, V MN-major from shared memory.
+    if (tid == 0) issue_pv(0, NSt);
+    // The scores: each key's column sums from the lane quarters whose
+    // chunk held it, in a fixed order.
+    if (tid < NSt && tid < n) {
+      float sc = 0.f;
+#pragma unroll
+      for (int q4 = 0; q4 < 4; ++q4)
+        if ((tid & ~15) < lim_warp(mt, q4)) sc += PART[q4 * kTcMaxRows + tid];
+      ACC[tid] += sc * inv_g;
     }
-    if (!(ok = wait_all(&bar_o))) break;
-    if (mt + 1 < n_mt) load_q(mt + 1);  // P lo is free until the next softmax
-
-    // 4. Outputs (this thread's row, half of the head dimension) and the
-    // column sums (every lane of warp 0 holds the same sums).
     constexpr int osz = kOutBf16 ? 2 : 4;
     unsigned char *orow = nullptr;
     if (valid) {
@@ -748,55 +808,64 @@ __global__ void __launch_bounds__(kThreads, 1)
       orow = reinterpret_cast<unsigned char *>(p.out) +
              ((((u.row0 + j) * c.H + h) * G + g) * 128) * osz;
     }
-    uint32_t ov[4][16];
-#pragma unroll
-    for (int k = 0; k < 4; ++k)
-      tmem_ld16_nowait(trow + kTcO + (upper ? 64 : 0) + 16 * k, ov[k]);
-    tmem_wait_ld();
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      const int c0 = (upper ? 64 : 0) + 16 * k;
-      const uint32_t(&v)[16] = ov[k];
+    for (int hd = 0; hd < 2 && ok; ++hd) {
+      if (!(ok = wait_all(&bar_o, ph_o))) break;
+      // This thread's row, 32 of the half's columns.
+      float ov[2][16];
+      const int c0 = (upper ? 32 : 0);
+      tmem_ld16f_nowait(trow + kTcO + c0, ov[0]);
+      tmem_ld16f_nowait(trow + kTcO + c0 + 16, ov[1]);
+      tmem_wait_ld();
+      if (hd == 1 && mt + 1 < n_mt) {  // the next tile's q rows
+        cp_async_commit_wait_all();
+        fence_proxy_async();
+      }
+      tc_fence_before();
+      __syncthreads();  // O (and, after the last half, P) has been read
+      tc_fence_after();
+      if (tid == 0) {
+        if (hd == 0)
+          issue_pv(1, NSt);
+        else if (mt + 1 < n_mt)
+          issue_s(mt + 1);
+      }
       if (valid) {
-        if (kOutBf16) {
-          uint32_t w[8];
 #pragma unroll
-          for (int j = 0; j < 8; ++j)
-            w[j] = pack_bf16(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));
-          reinterpret_cast<int4 *>(orow + c0 * 2)[0] = make_int4(w[0], w[1], w[2], w[3]);
-          reinterpret_cast<int4 *>(orow + c0 * 2)[1] = make_int4(w[4], w[5], w[6], w[7]);
-        } else {
+        for (int k = 0; k < 2; ++k) {
+          const int d0 = 64 * hd + c0 + 16 * k;
+          if (kOutBf16) {
+            uint32_t w[8];
 #pragma unroll
-          for (int j = 0; j < 4; ++j)
-            reinterpret_cast<int4 *>(orow + c0 * 4)[j] =
-                make_int4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+            for (int jj = 0; jj < 8; ++jj) w[jj] = pack_bf16(ov[k][2 * jj], ov[k][2 * jj + 1]);
+            reinterpret_cast<int4 *>(orow + d0 * 2)[0] = make_int4(w[0], w[1], w[2], w[3]);
+            reinterpret_cast<int4 *>(orow + d0 * 2)[1] = make_int4(w[4], w[5], w[6], w[7]);
+          } else {
+#pragma unroll
+            for (int jj = 0; jj < 4; ++jj)
+              reinterpret_cast<float4 *>(orow + d0 * 4)[jj] =
+                  make_float4(ov[k][4 * jj], ov[k][4 * jj + 1], ov[k][4 * jj + 2],
+                              ov[k][4 * jj + 3]);
+          }
         }
       }
     }
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-  }
-  // Key tid's sum over the unit's query rows: TMEM lane tid % 128 of CS
-  // tile tid / 128 (all 16 columns of a lane hold the same sum).
-  if (ok && n_mt > 0 && (!upper || n_ct > 1)) {
-    uint32_t v[16];
-    tmem_ld16(trow + kTcCS + (upper ? 16 : 0), v);
-    if (tid < n) m.acc[tid] += __uint_as_float(v[0]) * inv_g;
   }
   // After a timeout, wait (bounded) once more for tensor work in flight.
+  // Only the barrier whose wait gave up has a commit outstanding (its phase
+  // has the parity before the toggle); on the other, that parity names a
+  // completed phase and the wait returns at once.
   if (!ok) {
     volatile int never = 0;
     if (tid == 0) {
-      mbar_wait(smem_u32(&bar_s), (uint32_t)(phase & 1), &never);
-      mbar_wait(smem_u32(&bar_o), (uint32_t)(phase & 1), &never);
+      mbar_wait(smem_u32(&bar_s), (uint32_t)((ph_s ^ 1) & 1), &never);
+      mbar_wait(smem_u32(&bar_o), (uint32_t)((ph_o ^ 1) & 1), &never);
     }
   }
   tc_fence_before();
   __syncthreads();
   if (warp == 0) tmem_dealloc(tm, kTcCols);
   if (!ok) return;
-  finish_unit(p, u, m, &s_base, &s_count, s_wsum);
+  finish_unit<kTcMaxRows>(p, u, m, &s_base, &s_count, s_wsum);
 }
 
 }  // namespace
@@ -809,7 +878,9 @@ cudaError_t launch_absorb(const AbsorbParams &p, int kernel, cudaStream_t st) {
       !p.c.kv_bf16)
     return cudaErrorInvalidValue;
   const int units = p.c.S * p.nl * p.c.H;
-  const bool tc = kernel != 1;
+  // The tensor-memory kernel stages at most kTcMaxRows rows; larger units
+  // (up to kMaxRows) take the mma.sync kernel.
+  const bool tc = kernel != 1 && p.max_rows <= kTcMaxRows;
   const int smem = tc ? TcSmem::alloc : AbsorbSmem::bytes;
   auto kern = tc ? (p.c.out_bf16 ? absorb_tc_kernel<true> : absorb_tc_kernel<false>)
                  : (p.c.out_bf16 ? absorb_kernel<true> : absorb_kernel<false>);

@@ -862,6 +862,7 @@ kvr_status kvr_absorb_chunk(kvr_cache *c, int lb, int le, int chunk,
     p.lb = lb;
     p.nl = le - lb;
     p.chunk = chunk;
+    p.max_rows = m + chunk;
     p.budget = budget;
     p.window = window;
     p.evict = evict ? 1 : 0;

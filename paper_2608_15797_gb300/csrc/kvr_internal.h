@@ -286,12 +286,14 @@ struct AbsorbParams {
   const __nv_bfloat16 *q, *k_new, *v_new;  // [S][nl][chunk][...][128]
   void *out;
   int lb, nl, chunk;
+  int max_rows;  // largest unit after the chunk over the call
   int budget, window, evict;
   float scale_log2e, inv_g;
 };
 int absorb_max_chunk();
 int absorb_max_rows();
-// kernel: 0 the tensor-memory (tcgen05) kernel, 1 the mma.sync kernel.
+// kernel: 0 the tensor-memory (tcgen05) kernel (units of at most 144 rows
+// after the chunk; larger ones run the other), 1 the mma.sync kernel.
 cudaError_t launch_absorb(const AbsorbParams &p, int kernel, cudaStream_t st);
 
 // Persistent chunked step (kvr_chunked.cu): bf16, d = 128, G <= 8, at most

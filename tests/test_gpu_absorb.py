@@ -138,3 +138,17 @@ def test_absorb_full_unit_and_128_row_tiles(path):
     c, o = _pair(w, 56, 2, 192, [128, 127], path)
     absorb_lockstep(c, o, w, 56, 64, w.budget, w.window)
     harness.lockstep(c, o, w, 56, 2, w.budget, w.window, step0=400)
+
+
+@pytest.mark.parametrize("G,old", [(8, 80), (7, 72), (3, 79)])
+def test_absorb_tc_largest_unit(G, old):
+    """The tensor-memory kernel's largest units (old rows + a 64-token chunk
+    up to its 144-row limit; with G = 8 the 512 query rows fill four 128-row
+    tiles), units of unequal length in one launch, and a 145-row unit
+    routed to the mma.sync kernel in the same way."""
+    w = inputs.Workload("tl", 2, 2, G, 128, "bf16", 60, 8, old, 0, sigma=1.0)
+    c, o = _pair(w, 57 + G, 2, old + 64 + 1, [old, old - 9], "tc")
+    absorb_lockstep(c, o, w, 57 + G, 64, w.budget, w.window)
+    harness.lockstep(c, o, w, 57 + G, 2, w.budget, w.window, step0=500)
+    c, o = _pair(w, 60 + G, 1, 146, [81], "tc")
+    absorb_lockstep(c, o, w, 60 + G, 64, w.budget, w.window)
