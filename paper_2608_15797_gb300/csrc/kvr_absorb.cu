@@ -540,14 +540,16 @@ __device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&v)[8])
 
 template <bool kOutBf16>
 __global__ void __launch_bounds__(kThreads, 2)
-    absorb_tc_kernel(const AbsorbParams p) {
+    absorb_tc_kernel(const AbsorbParams p, const __grid_constant__ CUtensorMap tmQ) {
   pdl_begin();
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   __shared__ int s_base, s_count;
   __shared__ int s_wsum[kWarps];
   __shared__ uint32_t s_tmem;
   __shared__ int s_abort;
-  __shared__ __align__(8) uint64_t bar_s, bar_o;
+  __shared__ int s_q;  // thread 32's q state: bit 0 the phase to wait, bit 1 a load in flight
+  __shared__ int s_dq[4];  // (32 q4 + 31) / G: the last token of rows 32 q4 .. 32 q4 + 31
+  __shared__ __align__(8) uint64_t bar_s, bar_o, bar_q;
   unsigned char *smem = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
   const CacheView &c = p.c;
   const int G = c.G, C = p.chunk;
@@ -564,39 +566,31 @@ __global__ void __launch_bounds__(kThreads, 2)
                    reinterpret_cast<int *>(smem + TcSmem::kept)};
   float2 *s_ml = reinterpret_cast<float2 *>(smem + TcSmem::key);  // free until the selection
   if (warp == 0) tmem_alloc(smem_u32(&s_tmem), kTcCols);
+  const int n = u.n, n0 = u.n0, h = u.h;
+  const uint32_t aQ = smem_u32(smem + TcSmem::q);
+  // Tile mt holds tokens [mt Jt, mt Jt + Jt) of the chunk (Jt = 128 / G
+  // whole tokens) as rows token * G + g: one TMA box {64, G, 1, Jt} per
+  // 64-column half, 128-byte swizzle.  Rows past Jt G keep what they held
+  // and rows past the chunk hold other units' queries (or zeros past the
+  // tensor); both are masked below.
+  const int Jt = kTcRows / G, n_mt = (C + Jt - 1) / Jt;
+  const uint32_t q_bytes = 256u * (uint32_t)(G * Jt);
+  auto load_q = [&](int mt) {  // one thread
+    mbar_expect_tx(smem_u32(&bar_q), q_bytes);
+    for (int hf = 0; hf < 2; ++hf)
+      tma_load_4d(aQ + hf * (kTcRows * 128), &tmQ, 64 * hf, 0, h, (int)u.row0 + mt * Jt,
+                  smem_u32(&bar_q));
+  };
+  if (tid < 4) s_dq[tid] = (32 * tid + 31) / G;
   if (tid == 32) {
     mbar_init(smem_u32(&bar_s), 1);
     mbar_init(smem_u32(&bar_o), 1);
+    mbar_init(smem_u32(&bar_q), 1);
     s_abort = 0;
+    s_q = 2;
     fence_mbar_init();
+    load_q(0);
   }
-  const int n = u.n, n0 = u.n0, h = u.h;
-  const int MQ = C * G, n_mt = (MQ + kTcRows - 1) / kTcRows;
-  const uint32_t aQ = smem_u32(smem + TcSmem::q);
-  // Tile mt's q rows (row R = token j * G + head g), zeros past MQ, into the
-  // Q buffer with cp.async (completed by the next commit-and-wait).
-  // Two threads a row, eight 16-byte pieces each.
-  static_assert(kThreads == 2 * kTcRows, "two threads a q row");
-  auto load_q = [&](int mt) {
-    const int rr = tid >> 1, ch0 = (tid & 1) * 8, R = mt * kTcRows + rr;
-    const __nv_bfloat16 *src = nullptr;
-    if (R < MQ) {
-      const int j = R / G, g = R % G;
-      src = p.q + (((u.row0 + j) * c.H + h) * G + g) * 128;
-    }
-#pragma unroll
-    for (int k = 0; k < 8; ++k) {
-      const int ch = ch0 + k;
-      const uint32_t dst = aQ + (ch >> 3) * (kTcRows * 128) + rr * 128 +
-                           (((ch & 7) ^ (rr & 7)) << 4);
-      if (src)
-        cp_async16(dst, src + ch * 8);
-      else
-        asm volatile("st.shared.v4.b32 [%0], {%1, %1, %1, %1};" ::"r"(dst), "r"(0)
-                     : "memory");
-    }
-  };
-  load_q(0);
   tc_fence_before();
   load_unit<kTcMaxRows>(p, u, m);  // ends with the copies complete and __syncthreads
   tc_fence_after();
@@ -611,20 +605,20 @@ __global__ void __launch_bounds__(kThreads, 2)
   float *PART = reinterpret_cast<float *>(smem + TcSmem::part);
   volatile int *abort = &s_abort;
   // Keys that rows 32 q4 .. 32 q4 + 31 of tile mt may see: the causal
-  // limit of the last of them (row R is token R / G of the chunk), 0 when
-  // they are all past MQ.
+  // limit of the last of them below the tile's valid rows, 0 when there is
+  // none.
   auto lim_warp = [&](int mt, int q4) {
-    const int R0 = mt * kTcRows + 32 * q4;
-    if (R0 >= MQ) return 0;
-    return n0 + (min(R0 + 32, MQ) - 1) / G + 1;
+    const int toks = min(Jt, C - mt * Jt);  // the tile's tokens
+    if (32 * q4 >= toks * G) return 0;
+    return n0 + mt * Jt + min(s_dq[q4], toks - 1) + 1;
   };
   // Columns of S tile mt: its keys rounded up to whole 16-key chunks
   // (P is zero past the last row's limit, so no MMA reads further).
-  auto tile_cols = [&](int mt) {  // every tile has at least one row below MQ
-    return (n0 + (min(mt * kTcRows + kTcRows, MQ) - 1) / G + 1 + 15) & ~15;
-  };
-  auto issue_s = [&](int mt) {  // one thread
+  auto tile_cols = [&](int mt) { return (n0 + min(mt * Jt + Jt, C) + 15) & ~15; };
+  // MMA issue, one thread each (S: thread 32; PV: thread 0).
+  auto issue_s = [&](int mt) {
     const uint32_t id_s = idesc_bf16(kTcRows, tile_cols(mt), false);
+#pragma unroll
     for (int k = 0; k < 8; ++k) {  // K = 128 head-dim columns, 16 a step
       const uint32_t off = (k & 3) * 32;
       tc_mma(tm + kTcS, sdesc_sw128(aQ + (k >> 2) * (kTcRows * 128) + off, 16, 1024),
@@ -633,12 +627,19 @@ __global__ void __launch_bounds__(kThreads, 2)
     tc_commit(smem_u32(&bar_s));
   };
   const uint32_t id_o = idesc_bf16(kTcRows, 64, true);
-  auto issue_pv = [&](int hd, int NSt) {  // one thread: O half hd = P V[:, 64 hd ..]
-    for (int k = 0; k < NSt / 16; ++k) {  // K = keys, 16 a step
-      const uint64_t bv =
-          sdesc_sw128(aV + hd * (kTcMaxRows * 128) + k * 2048, kTcMaxRows * 128, 1024);
-      mma_ts_all(tm + kTcO, tm + kTcS + 16 * k, bv, id_o, k > 0);
-      mma_ts_all(tm + kTcO, tm + kTcS + 16 * k + 8, bv, id_o, true);
+  // O half hd = P V[:, 64 hd ..]; the V descriptor is formed once and
+  // stepped by adding to its address field (16-byte units).
+  auto issue_pv = [&](int hd, int NSt) {
+    const uint64_t dv = sdesc_sw128(aV + hd * (kTcMaxRows * 128), kTcMaxRows * 128, 1024);
+    const uint32_t dO = tm + kTcO;
+    uint32_t aP = tm + kTcS;
+    mma_ts_all(dO, aP, dv, id_o, false);
+    mma_ts_all(dO, aP + 8, dv, id_o, true);
+    for (int k = 1; k < NSt / 16; ++k) {  // K = keys, 16 a step (2048 bytes of V)
+      aP += 16;
+      const uint64_t bv = dv + (uint64_t)(k * 128);
+      mma_ts_all(dO, aP, bv, id_o, true);
+      mma_ts_all(dO, aP + 8, bv, id_o, true);
     }
     tc_commit(smem_u32(&bar_o));
   };
@@ -655,17 +656,31 @@ __global__ void __launch_bounds__(kThreads, 2)
     tc_fence_after();
     return all;
   };
-  // Tile 0's q rows have landed (the unit load ended with a barrier after
-  // every thread's copies completed).
+  // The issuing thread waits for a tile's q rows before its S.
+  auto wait_q = [&]() {  // thread 32
+    const int q = s_q;
+    const bool got = mbar_wait(smem_u32(&bar_q), (uint32_t)(q & 1), abort);
+    if (got) {
+      s_q = (q & 1) ^ 1;
+    } else {
+      atomicOr(c.err, ERR_TIMEOUT);
+      *abort = 1;
+    }
+    return got;
+  };
+  // K (written by the unit load) is visible to the tensor cores.
   fence_proxy_async();
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  if (tid == 0) issue_s(0);
+  if (tid == 32 && wait_q()) issue_s(0);
   for (int mt = 0; mt < n_mt && ok; ++mt) {
     // 1. S = Q K^T for the tile's keys is in tensor memory.
     if (!(ok = wait_all(&bar_s, ph_s))) break;
-    if (mt + 1 < n_mt) load_q(mt + 1);  // S has read this tile's q rows
+    if (tid == 32 && mt + 1 < n_mt) {  // S has read this tile's q rows
+      load_q(mt + 1);
+      s_q |= 2;
+    }
     const int NSt = tile_cols(mt);
     const int half = ((NSt >> 1) + 15) & ~15;
     const int c_lo = upper ? half : 0, c_hi = upper ? NSt : half;
@@ -675,9 +690,8 @@ __global__ void __launch_bounds__(kThreads, 2)
     // 2. This thread's logits (at most kTcChunks 16-column chunks) read
     // from TMEM once, exponentiated against the thread's own maximum; the
     // row's maximum and sum come from an exchange with the partner warp.
-    const int R = mt * kTcRows + r;
-    const bool valid = R < MQ;
-    const int lim = valid ? n0 + R / G + 1 : 0;  // keys the row may see
+    const bool valid = r < Jt * G && mt * Jt + r / G < C;
+    const int lim = valid ? n0 + mt * Jt + r / G + 1 : 0;  // keys the row may see
     float e[kTcChunks][16];
     float mx = -INFINITY;
 #pragma unroll
@@ -793,42 +807,36 @@ __global__ void __launch_bounds__(kThreads, 2)
     // P (hi and lo) from tensor memory, V MN-major from shared memory.
     if (tid == 0) issue_pv(0, NSt);
     // The scores: each key's column sums from the lane quarters whose
-    // chunk held it, in a fixed order.
-    if (tid < NSt && tid < n) {
+    // chunk held it, in a fixed order (warps 2 and up: warp 0 issues).
+    if (const int key = tid - 64; key >= 0 && key < NSt && key < n) {
       float sc = 0.f;
 #pragma unroll
       for (int q4 = 0; q4 < 4; ++q4)
-        if ((tid & ~15) < lim_warp(mt, q4)) sc += PART[q4 * kTcMaxRows + tid];
-      ACC[tid] += sc * inv_g;
+        if ((key & ~15) < lim_warp(mt, q4)) sc += PART[q4 * kTcMaxRows + key];
+      ACC[key] += sc * inv_g;
     }
     constexpr int osz = kOutBf16 ? 2 : 4;
     unsigned char *orow = nullptr;
     if (valid) {
-      const int j = R / G, g = R % G;
+      const int rq = r / G, tok = mt * Jt + rq, rg = r - rq * G;
       orow = reinterpret_cast<unsigned char *>(p.out) +
-             ((((u.row0 + j) * c.H + h) * G + g) * 128) * osz;
+             ((((u.row0 + tok) * c.H + h) * G + rg) * 128) * osz;
     }
     for (int hd = 0; hd < 2 && ok; ++hd) {
       if (!(ok = wait_all(&bar_o, ph_o))) break;
+      // After the second half, P has been read: the next tile's S may
+      // overwrite it while this O half drains.
+      if (hd == 1 && tid == 32 && mt + 1 < n_mt && wait_q()) issue_s(mt + 1);
       // This thread's row, 32 of the half's columns.
       float ov[2][16];
       const int c0 = (upper ? 32 : 0);
       tmem_ld16f_nowait(trow + kTcO + c0, ov[0]);
       tmem_ld16f_nowait(trow + kTcO + c0 + 16, ov[1]);
       tmem_wait_ld();
-      if (hd == 1 && mt + 1 < n_mt) {  // the next tile's q rows
-        cp_async_commit_wait_all();
-        fence_proxy_async();
-      }
       tc_fence_before();
-      __syncthreads();  // O (and, after the last half, P) has been read
+      __syncthreads();  // O has been read
       tc_fence_after();
-      if (tid == 0) {
-        if (hd == 0)
-          issue_pv(1, NSt);
-        else if (mt + 1 < n_mt)
-          issue_s(mt + 1);
-      }
+      if (hd == 0 && tid == 0) issue_pv(1, NSt);
       if (valid) {
 #pragma unroll
         for (int k = 0; k < 2; ++k) {
@@ -856,9 +864,10 @@ __global__ void __launch_bounds__(kThreads, 2)
   // completed phase and the wait returns at once.
   if (!ok) {
     volatile int never = 0;
-    if (tid == 0) {
+    if (tid == 32) {
       mbar_wait(smem_u32(&bar_s), (uint32_t)((ph_s ^ 1) & 1), &never);
       mbar_wait(smem_u32(&bar_o), (uint32_t)((ph_o ^ 1) & 1), &never);
+      if (s_q & 2) mbar_wait(smem_u32(&bar_q), (uint32_t)(s_q & 1), &never);
     }
   }
   tc_fence_before();
@@ -873,21 +882,26 @@ __global__ void __launch_bounds__(kThreads, 2)
 int absorb_max_chunk() { return kMaxChunk; }
 int absorb_max_rows() { return kMaxRows; }
 
-cudaError_t launch_absorb(const AbsorbParams &p, int kernel, cudaStream_t st) {
+cudaError_t launch_absorb(const AbsorbParams &p, int kernel, const CUtensorMap *tmQ,
+                          cudaStream_t st) {
   if (p.chunk < 1 || p.chunk > kMaxChunk || p.c.G > 8 || p.c.d != 128 ||
       !p.c.kv_bf16)
     return cudaErrorInvalidValue;
   const int units = p.c.S * p.nl * p.c.H;
   // The tensor-memory kernel stages at most kTcMaxRows rows; larger units
   // (up to kMaxRows) take the mma.sync kernel.
-  const bool tc = kernel != 1 && p.max_rows <= kTcMaxRows;
-  const int smem = tc ? TcSmem::alloc : AbsorbSmem::bytes;
-  auto kern = tc ? (p.c.out_bf16 ? absorb_tc_kernel<true> : absorb_tc_kernel<false>)
-                 : (p.c.out_bf16 ? absorb_kernel<true> : absorb_kernel<false>);
+  if (kernel != 1 && p.max_rows <= kTcMaxRows && tmQ) {
+    auto kern = p.c.out_bf16 ? absorb_tc_kernel<true> : absorb_tc_kernel<false>;
+    cudaError_t e = cudaFuncSetAttribute(
+        kern, cudaFuncAttributeMaxDynamicSharedMemorySize, TcSmem::alloc);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(kern, dim3(units), dim3(kThreads), (size_t)TcSmem::alloc, st, p, *tmQ);
+  }
+  auto kern = p.c.out_bf16 ? absorb_kernel<true> : absorb_kernel<false>;
   cudaError_t e = cudaFuncSetAttribute(
-      kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+      kern, cudaFuncAttributeMaxDynamicSharedMemorySize, AbsorbSmem::bytes);
   if (e != cudaSuccess) return e;
-  return launch_pdl(kern, dim3(units), dim3(kThreads), (size_t)smem, st, p);
+  return launch_pdl(kern, dim3(units), dim3(kThreads), (size_t)AbsorbSmem::bytes, st, p);
 }
 
 }  // namespace kvr

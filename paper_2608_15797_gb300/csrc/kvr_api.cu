@@ -183,6 +183,22 @@ bool encode_tails4(CUtensorMap *m, void *base, int nt, int tcap, size_t units,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// The chunk's queries as a 4-D tensor {128 elements, G heads, H KV heads,
+// tokens}: a box {64, G, 1, 128 / G} fetches the whole tokens that fill at
+// most 128 rows (token * G + g) of one KV head.
+bool encode_q4(CUtensorMap *m, const void *base, int G, int H, size_t tokens) {
+  auto fn = encode_tiled();
+  if (!fn || G < 1 || G > 8) return false;
+  cuuint64_t dims[4] = {128, (cuuint64_t)G, (cuuint64_t)H, (cuuint64_t)tokens};
+  cuuint64_t strides[3] = {256, (cuuint64_t)G * 256, (cuuint64_t)H * G * 256};
+  cuuint32_t box[4] = {64, (cuuint32_t)G, 1, (cuuint32_t)(128 / G)};
+  cuuint32_t estr[4] = {1, 1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(base), dims, strides,
+            box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 }  // namespace
 
 namespace {
@@ -868,7 +884,10 @@ kvr_status kvr_absorb_chunk(kvr_cache *c, int lb, int le, int chunk,
     p.evict = evict ? 1 : 0;
     p.scale_log2e = v.scale * 1.4426950408889634f;
     p.inv_g = 1.f / (float)v.G;
-    cudaError_t e = kvr::launch_absorb(p, c->absorb_kernel, as_stream(stream));
+    CUtensorMap tmq;
+    const bool have_q = encode_q4(&tmq, q, v.G, v.H, (size_t)v.S * p.nl * chunk);
+    cudaError_t e = kvr::launch_absorb(p, c->absorb_kernel, have_q ? &tmq : nullptr,
+                                       as_stream(stream));
     if (e != cudaSuccess) return cuda_fail("kvr_absorb_chunk", e);
     c->launches += 1;
     for (int j = 0; j < chunk; ++j) mirror_append(c, lb, le);

@@ -293,8 +293,11 @@ struct AbsorbParams {
 int absorb_max_chunk();
 int absorb_max_rows();
 // kernel: 0 the tensor-memory (tcgen05) kernel (units of at most 144 rows
-// after the chunk; larger ones run the other), 1 the mma.sync kernel.
-cudaError_t launch_absorb(const AbsorbParams &p, int kernel, cudaStream_t st);
+// after the chunk, given tmQ; otherwise the other), 1 the mma.sync kernel.
+// tmQ: q as a 4-D tensor {128, G, H, S * nl * chunk tokens} with boxes
+// {64, G, 1, 128 / G} and 128-byte swizzle.
+cudaError_t launch_absorb(const AbsorbParams &p, int kernel, const CUtensorMap *tmQ,
+                          cudaStream_t st);
 
 // Persistent chunked step (kvr_chunked.cu): bf16, d = 128, G <= 8, at most
 // chunk_max_rows() rows per job with the new row.  A job is one unit of the
