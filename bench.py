@@ -90,7 +90,8 @@ def parse():
                    help="--mode entropy kernel: 0 library's choice, "
                         "1 persistent streaming, 2 one CTA per piece")
     p.add_argument("--seqs", type=int, default=0,
-                   help="sequences for --mode helper/fork (0: 16 / 4)")
+                   help="sequences for --mode helper/fork/absorb/rkv "
+                        "(0: 16 / 4 / 64 / 64)")
     p.add_argument("--chunk-groups", type=int, default=0,
                    help="chunked kernel: consumer groups per SM (0 auto, -1 off)")
     p.add_argument("--chunk-stages", type=int, default=0,
@@ -1280,7 +1281,8 @@ def sub_records(args):
         r.update(metric="absorbed 64-token steps/s (7B, B=64, W=8, 64 "
                         "sequences x 28 layers a call)",
                  kernel="kvr_absorb_chunk (absorb_tc_kernel, tcgen05)",
-                 config={"workload": "7b absorb", "chunk": r["C"]})
+                 config={"workload": "7b absorb", "chunk": r["C"]},
+                 profile="absorb_7b_s64_c64")
         r_abs.update(r)
         return r
     run("absorb_7b_c64", absorb, "calls/s")
@@ -1408,7 +1410,9 @@ def main():
                 "roofline": {"bound": "hbm", "achieved": gbs,
                              "peak": float(peaks["hbm_gbs"]), "unit": "GB/s",
                              "frac": gbs / float(peaks["hbm_gbs"]),
-                             "peak_kind": peak_kind, "traffic": None,
+                             "peak_kind": peak_kind,
+                             "traffic": committed_traffic("absorb_7b_s64_c64")
+                             if r["S"] == 64 and args.absorb_kernel == 0 else None,
                              "algorithmic_bytes_per_launch": r["launch_bytes"],
                              "launch_ms": r["per_ms"],
                              "kernel": "absorb_tc_kernel (tcgen05)"
