@@ -140,6 +140,20 @@ def test_absorb_full_unit_and_128_row_tiles(path):
     harness.lockstep(c, o, w, 56, 2, w.budget, w.window, step0=400)
 
 
+@pytest.mark.parametrize("G", [2, 4, 5, 6])
+@pytest.mark.parametrize("chunk", [37, 64])
+def test_absorb_tc_tiles_of_whole_tokens(G, chunk):
+    """Each query tile of the tensor-memory kernel holds 128 // G whole
+    tokens (one q box per 64-column half): G = 5 and 6 leave the tile's last
+    rows unused (125 and 126 rows), and a 37-token chunk leaves a ragged last
+    tile whose box reaches into the next unit's tokens (or past the end of
+    q for the last unit)."""
+    w = inputs.Workload("tg", 2, 2, G, 128, "bf16", 60, 8, 72, 0, sigma=1.0)
+    c, o = _pair(w, 70 + G, 2, 72 + chunk + 1, [72, 50], "tc")
+    absorb_lockstep(c, o, w, 70 + G, chunk, w.budget, w.window)
+    harness.lockstep(c, o, w, 70 + G, 2, w.budget, w.window, step0=600)
+
+
 @pytest.mark.parametrize("G,old", [(8, 80), (7, 72), (3, 79)])
 def test_absorb_tc_largest_unit(G, old):
     """The tensor-memory kernel's largest units (old rows + a 64-token chunk
