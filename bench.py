@@ -1298,7 +1298,8 @@ def sub_records(args):
                         f"({r['rows']} rows x {r['V']} {r['dtype']} logits a "
                         f"launch)",
                  kernel="kvr_entropy_step (entropy_stream_kernel)",
-                 config={"rows": r["rows"], "vocab": r["V"]})
+                 config={"rows": r["rows"], "vocab": r["V"]},
+                 profile=f"entropy_stream_{r['rows']}x{r['V']}_{r['dtype']}")
         return r
     run("entropy_512x152064", entropy, "launches/s")
     run("helper_1p5b_16k", lambda: run_helper(a), "steps/s")
