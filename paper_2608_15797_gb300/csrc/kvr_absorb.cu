@@ -7,11 +7,16 @@
 // (TopB of Eq. 1 with the window of Sec. 4.1).  bf16, head_dim 128, G <= 8,
 // c <= 64, at most kMaxRows rows after the chunk.
 //
-// Design (GB300, sm_103a): one CTA of 8 warps per unit.
+// Design (GB300, sm_103a): one CTA of 8 warps per unit, in two kernels
+// that share the load and the selection.  absorb_tc_kernel (5th-generation
+// tensor cores, two CTAs an SM; described before it) takes units of at most
+// 144 rows after the chunk; absorb_kernel (mma.sync) takes the rest, up to
+// kMaxRows, or any unit when selected.
 //  - The unit's live K/V rows and the chunk's new rows are copied into
 //    shared memory (16-byte cp.async pieces, 128B-swizzled rows so ldmatrix
-//    is conflict-free); every later read of K and V is from there.
-//  - The c*G query rows are the M side of bf16 mma.sync (m16n8k16, fp32
+//    and the tensor-core descriptors read them conflict-free); every later
+//    read of K and V is from there.
+//  - absorb_kernel: the c*G query rows are the M side of bf16 mma.sync (m16n8k16, fp32
 //    accumulate): a warp takes 16 query rows at a time, their fragments
 //    loaded straight from global memory.  Pass 1 runs QK^T over the rows
 //    each query may see (causal bound) for the exact softmax statistics;
@@ -445,24 +450,27 @@ __global__ void __launch_bounds__(kThreads)
 // ---- the same absorb on 5th-generation tensor cores ------------------------
 //
 // Units of at most kTcMaxRows rows after the chunk, two CTAs an SM (about
-// 111 KB of shared memory and 256 tensor-memory columns each), so that one
+// 114 KB of shared memory and 256 tensor-memory columns each), so that one
 // unit's loads, selection and stores overlap the other's tensor work.
-// Query rows go in tiles of 128 (M), with the unit's keys as N (rows
-// rounded up to 16) and K = the head dimension.  Per tile:
-//   1. The tile's q rows are in shared memory (K-major, 128B swizzle; the
-//      next tile's are fetched once this tile's S is done) and one thread
-//      issues S = Q K^T into tensor memory (fp32, N columns).
-//   2. Every warp reads its rows' logits from tensor memory; warps w and
-//      w + 4 share TMEM lanes 32 (w % 4).. and take half the columns each.
-//      They form the row statistics (an exchange through shared memory),
-//      then the exact probabilities: P in place of the logits (each 16-key
-//      chunk's 16 columns take its 8 hi and 8 lo columns of bf16 pairs, the
-//      A operand of PV), and their column sums over the tile's rows (a
-//      butterfly over the warp's 32 rows, then shared-memory atomics) for
-//      the scores.
-//   3. O = P_hi V + P_lo V one 64-column half of the head dimension at a
-//      time (64 tensor-memory columns), each half stored from tensor memory
-//      before the next is computed.
+// Query rows go in tiles of 128 / G whole tokens (row token * G + g; M =
+// 128), with the unit's keys as N and K = the head dimension.  Per tile:
+//   1. The tile's q rows arrive by TMA (one 4-D box per 64-column half,
+//      K-major, 128B swizzle; the next tile's are fetched once this tile's
+//      S is done) and thread 32 issues S = Q K^T into tensor memory (fp32;
+//      N = the tile's causal limit rounded up to 16 keys).
+//   2. Every warp reads its rows' logits from tensor memory once; warps w
+//      and w + 4 share TMEM lanes 32 (w % 4).. and take half the columns
+//      each.  They form the row statistics (an exchange on a named barrier
+//      per pair), then the exact probabilities: P in place of the logits
+//      (each 16-key chunk's 16 columns take its 8 hi and 8 lo columns of
+//      bf16 pairs, the A operand of PV), and their column sums over the
+//      warp's 32 rows (a shuffle butterfly into one slot per lane quarter,
+//      summed in a fixed order) for the scores.  Chunks past a warp's last
+//      causal limit are neither read nor exponentiated.
+//   3. Thread 0 issues O = P_hi V + P_lo V one 64-column half of the head
+//      dimension at a time (64 tensor-memory columns); the second half's
+//      MMAs start once every thread has read the first, and the next
+//      tile's S once the second half is done.
 // Every mbarrier wait is bounded; tensor memory is freed before the
 // selection.
 constexpr int kTcMaxRows = 144;                    // rows this kernel stages
