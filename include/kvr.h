@@ -458,10 +458,13 @@ kvr_status kvr_entropy_launch_count(const kvr_entropy *det, uint64_t *count);
 
 void kvr_entropy_destroy(kvr_entropy *det);
 
-/* Kernel of kvr_absorb_chunk's one-launch path (results agree within
- * rounding): 0 = 5th-generation tensor cores with the logits, outputs and
- * score column sums in tensor memory (the default), 1 = mma.sync with
- * register accumulators. */
+/* Kernel of kvr_absorb_chunk's one-launch path (bf16, head_dim 128, G <= 8,
+ * chunk <= 64, at most 192 rows after the chunk, 16-byte aligned q, k_new,
+ * v_new and out; other calls run token by token).  Results agree within
+ * rounding: 0 = 5th-generation tensor cores with the logits, probabilities
+ * and outputs in tensor memory, for units of at most 144 rows after the
+ * chunk (larger ones run kernel 1; the default), 1 = mma.sync with register
+ * accumulators. */
 kvr_status kvr_cache_set_absorb_kernel(kvr_cache *cache, int kernel);
 
 /* ---- the same step for callers that cannot allocate -------------------- */
