@@ -798,6 +798,7 @@ def run_absorb(args):
     total = t0.elapsed_time(t1)
     launches = cache.launch_count() - n0
     cache.sync_status()
+    ran = cache.last_absorb_kernel()
     units = S * L * H
     m = B + Wn
     # bytes: old K/V rows read, new k/v read, kept new rows written (at most
@@ -807,15 +808,17 @@ def run_absorb(args):
                 2 * C * G * d * 2 + 8 * m + 8 * m + 16)
     # flops over the causal triangle's mean width m + C/2: the mma.sync
     # kernel runs QK^T twice and PV with hi + lo terms; the tcgen05 kernel
-    # runs QK^T once, PV with hi + lo, and the score column sums (hi + lo)
-    # as a 128-row tensor product over the same width
-    if args.absorb_kernel == 1:
-        flops = C * G * (m + C / 2.0) * d * 2 * (2 + 2)
+    # runs QK^T once and PV with hi + lo (its column sums run on the CUDA
+    # cores)
+    if ran == 0:
+        flops = C * G * (m + C / 2.0) * d * 2 * (1 + 2)
     else:
-        flops = C * G * (m + C / 2.0) * d * 2 * (1 + 2 + 2)
+        flops = C * G * (m + C / 2.0) * d * 2 * (2 + 2)
+    kernel = {0: "absorb_tc_kernel (tcgen05)", 1: "absorb_kernel (mma.sync)",
+              2: "attend_score_kernel token by token"}.get(ran, "none")
     return dict(total_ms=total, per_ms=total / max(1, launches), K=K,
                 launches=launches, launch_bytes=per_unit * units,
-                launch_flops=flops * units, S=S, C=C)
+                launch_flops=flops * units, S=S, C=C, ran=ran, kernel=kernel)
 
 
 def run_entropy(args):
@@ -1284,9 +1287,10 @@ def sub_records(args):
         r = run_absorb(a_abs)
         r.update(metric="absorbed 64-token steps/s (7B, B=64, W=8, 64 "
                         "sequences x 28 layers a call)",
-                 kernel="kvr_absorb_chunk (absorb_tc_kernel, tcgen05)",
-                 config={"workload": "7b absorb", "chunk": r["C"]},
-                 profile="absorb_7b_s64_c64")
+                 kernel=f"kvr_absorb_chunk ({r['kernel']})",
+                 config={"workload": "7b absorb", "chunk": r["C"]})
+        if r["ran"] == 0:  # the profile's kernel
+            r["profile"] = "absorb_7b_s64_c64"
         r_abs.update(r)
         return r
     run("absorb_7b_c64", absorb, "calls/s")
@@ -1417,12 +1421,10 @@ def main():
                              "frac": gbs / float(peaks["hbm_gbs"]),
                              "peak_kind": peak_kind,
                              "traffic": committed_traffic("absorb_7b_s64_c64")
-                             if r["S"] == 64 and args.absorb_kernel == 0 else None,
+                             if r["S"] == 64 and r["ran"] == 0 else None,
                              "algorithmic_bytes_per_launch": r["launch_bytes"],
                              "launch_ms": r["per_ms"],
-                             "kernel": "absorb_tc_kernel (tcgen05)"
-                             if args.absorb_kernel == 0 else
-                             "absorb_kernel (mma.sync)"},
+                             "kernel": r["kernel"]},
                 "tensor": {"achieved_tflops": tfs,
                            "peak_tflops": float(peaks.get("bf16_tflops", 0)),
                            "frac": tfs / float(peaks.get("bf16_tflops", 1)),

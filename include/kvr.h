@@ -467,6 +467,11 @@ void kvr_entropy_destroy(kvr_entropy *det);
  * accumulators. */
 kvr_status kvr_cache_set_absorb_kernel(kvr_cache *cache, int kernel);
 
+/* How the cache's last kvr_absorb_chunk ran: 0 = the tensor-memory kernel,
+ * 1 = the mma.sync kernel, 2 = token by token; -1 before the first call
+ * (or for NULL).  Host state only: no synchronisation. */
+int kvr_cache_last_absorb_kernel(const kvr_cache *cache);
+
 /* ---- the same step for callers that cannot allocate -------------------- */
 
 /* The paper has no counterpart to this call: it is a deployment variant.

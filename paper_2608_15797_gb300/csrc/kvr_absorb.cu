@@ -891,14 +891,16 @@ int absorb_max_chunk() { return kMaxChunk; }
 int absorb_max_rows() { return kMaxRows; }
 
 cudaError_t launch_absorb(const AbsorbParams &p, int kernel, const CUtensorMap *tmQ,
-                          cudaStream_t st) {
+                          cudaStream_t st, int *ran) {
   if (p.chunk < 1 || p.chunk > kMaxChunk || p.c.G > 8 || p.c.d != 128 ||
       !p.c.kv_bf16)
     return cudaErrorInvalidValue;
   const int units = p.c.S * p.nl * p.c.H;
   // The tensor-memory kernel stages at most kTcMaxRows rows; larger units
   // (up to kMaxRows) take the mma.sync kernel.
-  if (kernel != 1 && p.max_rows <= kTcMaxRows && tmQ) {
+  const bool tc = kernel != 1 && p.max_rows <= kTcMaxRows && tmQ;
+  if (ran) *ran = tc ? 0 : 1;
+  if (tc) {
     auto kern = p.c.out_bf16 ? absorb_tc_kernel<true> : absorb_tc_kernel<false>;
     cudaError_t e = cudaFuncSetAttribute(
         kern, cudaFuncAttributeMaxDynamicSharedMemorySize, TcSmem::alloc);

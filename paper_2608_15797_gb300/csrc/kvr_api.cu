@@ -105,6 +105,7 @@ struct kvr_cache {
   int chunk_groups = 0;           // chunked kernel: groups (0 auto, -1 off)
   int chunk_stages = 0;           // chunked kernel: stages per group (0 auto)
   int absorb_kernel = 0;          // 0 tcgen05, 1 mma.sync (kvr_absorb_chunk)
+  int last_absorb = -1;           // kernel of the last kvr_absorb_chunk (0, 1, 2)
   int forks = 0;                  // live forks: the cache is read-only meanwhile
   int sm_count = 0;               // of the device, queried on first use
   int smem_optin = 0;
@@ -886,9 +887,11 @@ kvr_status kvr_absorb_chunk(kvr_cache *c, int lb, int le, int chunk,
     p.inv_g = 1.f / (float)v.G;
     CUtensorMap tmq;
     const bool have_q = encode_q4(&tmq, q, v.G, v.H, (size_t)v.S * p.nl * chunk);
+    int ran = 1;
     cudaError_t e = kvr::launch_absorb(p, c->absorb_kernel, have_q ? &tmq : nullptr,
-                                       as_stream(stream));
+                                       as_stream(stream), &ran);
     if (e != cudaSuccess) return cuda_fail("kvr_absorb_chunk", e);
+    c->last_absorb = ran;
     c->launches += 1;
     for (int j = 0; j < chunk; ++j) mirror_append(c, lb, le);
     if (evict) mirror_evict(c, lb, le, budget, window);
@@ -896,6 +899,7 @@ kvr_status kvr_absorb_chunk(kvr_cache *c, int lb, int le, int chunk,
   }
   // Token by token: each launch appends token j of every unit and attends
   // over every live row, adding to the scores (eviction deferred).
+  c->last_absorb = 2;
   for (int j = 0; j < chunk; ++j) {
     StepArgs a = step_args(c, lb, le, q, k_new, v_new, out);
     a.chunk = chunk;
@@ -1561,6 +1565,8 @@ kvr_status kvr_fork_export(const kvr_fork *f, int cand, int seq,
 }
 
 int kvr_fork_last_kernel(const kvr_fork *f) { return f ? f->last_kernel : 0; }
+
+int kvr_cache_last_absorb_kernel(const kvr_cache *c) { return c ? c->last_absorb : -1; }
 
 kvr_status kvr_fork_set_kernel(kvr_fork *f, int kernel) {
   if (!f) return fail(KVR_EINVAL, "null fork");

@@ -296,8 +296,9 @@ int absorb_max_rows();
 // after the chunk, given tmQ; otherwise the other), 1 the mma.sync kernel.
 // tmQ: q as a 4-D tensor {128, G, H, S * nl * chunk tokens} with boxes
 // {64, G, 1, 128 / G} and 128-byte swizzle.
+// *ran (if given): the kernel launched, 0 tcgen05 or 1 mma.sync.
 cudaError_t launch_absorb(const AbsorbParams &p, int kernel, const CUtensorMap *tmQ,
-                          cudaStream_t st);
+                          cudaStream_t st, int *ran = nullptr);
 
 // Persistent chunked step (kvr_chunked.cu): bf16, d = 128, G <= 8, at most
 // chunk_max_rows() rows per job with the new row.  A job is one unit of the

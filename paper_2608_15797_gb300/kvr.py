@@ -81,6 +81,7 @@ _SIGS = {
     "kvr_fork_set_kernel": (_S, [_P, _I]),
     "kvr_fork_last_kernel": (_I, [_P]),
     "kvr_cache_set_absorb_kernel": (_S, [_P, _I]),
+    "kvr_cache_last_absorb_kernel": (_I, [_P]),
     "kvr_cache_scores": (_S, [_P, _P, _P, _P, _P]),
     "kvr_sync_status": (_S, [_P, _P]),
     "kvr_last_error": (ctypes.c_char_p, []),
@@ -439,6 +440,11 @@ class Cache:
         """kvr_absorb_chunk's one-launch kernel: 0 tcgen05, 1 mma.sync."""
         _check(lib.kvr_cache_set_absorb_kernel(self.handle, kernel),
                "kvr_cache_set_absorb_kernel")
+
+    def last_absorb_kernel(self) -> int:
+        """How the last absorb ran (kvr_cache_last_absorb_kernel): 0 tcgen05,
+        1 mma.sync, 2 token by token, -1 before the first."""
+        return int(lib.kvr_cache_last_absorb_kernel(self.handle))
 
     def set_fused(self, enable: bool):
         kvr_cache_set_fused(self.handle, enable)

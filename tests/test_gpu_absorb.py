@@ -67,6 +67,10 @@ def test_absorb_shapes(G, d, dtype, chunk, path):
     w = inputs.Workload("ab", 2, 2, G, d, dtype, B, W, 20, 0, sigma=1.0)
     c, o = _pair(w, 50, 3, 20 + chunk + 4, [20, 0, 9], path)
     absorb_lockstep(c, o, w, 50, chunk, B, W)
+    # The one-launch kernels take bf16 with d = 128; the rest runs token by
+    # token.
+    one_launch = d == 128 and dtype == "bf16" and path != "tokenwise"
+    assert c.last_absorb_kernel() == (PATHS[path][1] if one_launch else 2)
     harness.lockstep(c, o, w, 50, 3, B, W, step0=100)
 
 
@@ -151,6 +155,7 @@ def test_absorb_tc_tiles_of_whole_tokens(G, chunk):
     w = inputs.Workload("tg", 2, 2, G, 128, "bf16", 60, 8, 72, 0, sigma=1.0)
     c, o = _pair(w, 70 + G, 2, 72 + chunk + 1, [72, 50], "tc")
     absorb_lockstep(c, o, w, 70 + G, chunk, w.budget, w.window)
+    assert c.last_absorb_kernel() == 0
     harness.lockstep(c, o, w, 70 + G, 2, w.budget, w.window, step0=600)
 
 
@@ -163,6 +168,9 @@ def test_absorb_tc_largest_unit(G, old):
     w = inputs.Workload("tl", 2, 2, G, 128, "bf16", 60, 8, old, 0, sigma=1.0)
     c, o = _pair(w, 57 + G, 2, old + 64 + 1, [old, old - 9], "tc")
     absorb_lockstep(c, o, w, 57 + G, 64, w.budget, w.window)
+    assert c.last_absorb_kernel() == 0
     harness.lockstep(c, o, w, 57 + G, 2, w.budget, w.window, step0=500)
     c, o = _pair(w, 60 + G, 1, 146, [81], "tc")
+    assert c.last_absorb_kernel() == -1
     absorb_lockstep(c, o, w, 60 + G, 64, w.budget, w.window)
+    assert c.last_absorb_kernel() == 1
