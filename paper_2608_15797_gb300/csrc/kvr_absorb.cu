@@ -172,57 +172,77 @@ __device__ void load_unit(const AbsorbParams &p, const Unit &u,
 // and row lists of kRows rows).
 template <int kRows = kMaxRows>
 __device__ void finish_unit(const AbsorbParams &p, const Unit &u,
-                            const UnitSmem &m, int *s_base, int *s_count,
-                            int *s_wsum) {
+                            const UnitSmem &m, int *s_wsum) {
   const CacheView &c = p.c;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int n = u.n, n0 = u.n0, C = p.chunk;
   float *SC = m.sc;
   int32_t *PS = m.ps;
-  for (int r = tid; r < n; r += kThreads) SC[r] += m.acc[r];
-  __syncthreads();
+  static_assert(kRows <= kThreads, "one thread a row");
   const int B = p.budget, W = p.window;
   const bool cut = p.evict && n > B + W;
   const int wlo = u.t0 + C - 1 - W;  // a row is a candidate iff pos <= wlo
-  // TopB by rank (n <= kMaxRows <= kThreads rows, one per thread): a
-  // candidate stays iff fewer than B candidates have a larger key (keys are
-  // distinct: positions are).  Rows outside the window-free set always stay.
+  // Thread t owns row t: its final score and its TopB key.
+  const int row = tid;
+  const bool live = row < n;
   unsigned long long *KEY = m.key;
   int *KEPT = m.kept;
-  for (int r = tid; r < n; r += kThreads)
-    KEY[r] = PS[r] <= wlo ? dev::rank_key(SC[r], PS[r]) : 0ull;
-  __syncthreads();
-  for (int r = tid; r < n; r += kThreads) {
-    int k = 1;
-    if (cut && PS[r] <= wlo) {
-      const unsigned long long mine_key = KEY[r];
-      int above = 0;
-      for (int j = 0; j < n; ++j) above += KEY[j] > mine_key ? 1 : 0;
-      k = above < B ? 1 : 0;
-    }
-    KEPT[r] = k;
+  if (live) {
+    SC[row] += m.acc[row];
+    KEY[row] = PS[row] <= wlo ? dev::rank_key(SC[row], PS[row]) : 0ull;
   }
   __syncthreads();
-  auto keep = [&](int i) { return KEPT[i] != 0; };
-  if (tid == 0) *s_count = 0;
+  // TopB by rank: a candidate stays iff fewer than B candidates have a
+  // larger key (keys are distinct: positions are).  Rows outside the
+  // window-free set always stay.
+  bool kp = live;
+  if (live && cut && PS[row] <= wlo) {
+    const unsigned long long mine_key = KEY[row];
+    int above = 0;
+#pragma unroll 4
+    for (int j = 0; j < n; ++j) above += KEY[j] > mine_key ? 1 : 0;
+    kp = above < B;
+  }
+  if (live) KEPT[row] = kp ? 1 : 0;
+  // Kept count, then the holes below it and the movers above it, each from
+  // warp ballots and a prefix over the warps' counts.
+  int *s_nk = s_wsum, *s_nh = s_wsum + kWarps, *s_nm = s_wsum + 2 * kWarps;
+  const unsigned below = (1u << lane) - 1u;
+  const unsigned bk = __ballot_sync(0xffffffffu, kp);
+  if (lane == 0) s_nk[warp] = __popc(bk);
   __syncthreads();
-  int mine = 0;
-  for (int i = tid; i < n; i += kThreads) mine += keep(i) ? 1 : 0;
-  atomicAdd(s_count, mine);
-  __syncthreads();
-  const int nk = *s_count;
+  int nk = 0;
+#pragma unroll
+  for (int w = 0; w < kWarps; ++w) nk += s_nk[w];
   if (cut && nk != B + W) {
     if (tid == 0) atomicOr(c.err, ERR_LENGTH);
     return;
   }
+  const bool is_hole = live && row < nk && !kp, is_mover = live && row >= nk && kp;
+  const unsigned bh = __ballot_sync(0xffffffffu, is_hole);
+  const unsigned bm = __ballot_sync(0xffffffffu, is_mover);
+  if (lane == 0) {
+    s_nh[warp] = __popc(bh);
+    s_nm[warp] = __popc(bm);
+  }
+  __syncthreads();
+  int oh = 0, om = 0, nh = 0, nm = 0;
+#pragma unroll
+  for (int w = 0; w < kWarps; ++w) {
+    oh += w < warp ? s_nh[w] : 0;
+    om += w < warp ? s_nm[w] : 0;
+    nh += s_nh[w];
+    nm += s_nm[w];
+  }
   int *holes = m.lists, *movers = m.lists + kRows;
-  const int nh = dev::block_collect(0, nk, [&](int i) { return !keep(i); }, holes,
-                                    s_wsum, s_base);
-  const int nm = dev::block_collect(nk, n, keep, movers, s_wsum, s_base);
+  if (is_hole) holes[oh + __popc(bh & below)] = row;
+  if (is_mover) movers[om + __popc(bm & below)] = row;
   if (nh != nm) {
     if (tid == 0) atomicOr(c.err, ERR_LENGTH);
     return;
   }
+  __syncthreads();
+  auto keep = [&](int i) { return KEPT[i] != 0; };
   // Final slot of every kept row: its own below nk, a hole for a mover.
   // Rows whose bytes must be written: new rows (r >= n0) that stay below nk,
   // and every mover (all rows are in shared memory).
@@ -261,8 +281,7 @@ __global__ void __launch_bounds__(kThreads)
     absorb_kernel(const AbsorbParams p) {
   pdl_begin();
   extern __shared__ __align__(1024) unsigned char smem[];
-  __shared__ int s_base, s_count;
-  __shared__ int s_wsum[kWarps];
+  __shared__ int s_wsum[3 * kWarps];  // per-warp counts for the selection
   const CacheView &c = p.c;
   const int G = c.G, C = p.chunk;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -444,7 +463,7 @@ __global__ void __launch_bounds__(kThreads)
   }
   __syncthreads();
 
-  finish_unit(p, u, m, &s_base, &s_count, s_wsum);
+  finish_unit(p, u, m, s_wsum);
 }
 
 // ---- the same absorb on 5th-generation tensor cores ------------------------
@@ -551,8 +570,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     absorb_tc_kernel(const AbsorbParams p, const __grid_constant__ CUtensorMap tmQ) {
   pdl_begin();
   extern __shared__ __align__(1024) unsigned char smem_raw[];
-  __shared__ int s_base, s_count;
-  __shared__ int s_wsum[kWarps];
+  __shared__ int s_wsum[3 * kWarps];  // per-warp counts for the selection
   __shared__ uint32_t s_tmem;
   __shared__ int s_abort;
   __shared__ int s_q;  // thread 32's q state: bit 0 the phase to wait, bit 1 a load in flight
@@ -882,7 +900,7 @@ __global__ void __launch_bounds__(kThreads, 2)
   __syncthreads();
   if (warp == 0) tmem_dealloc(tm, kTcCols);
   if (!ok) return;
-  finish_unit<kTcMaxRows>(p, u, m, &s_base, &s_count, s_wsum);
+  finish_unit<kTcMaxRows>(p, u, m, s_wsum);
 }
 
 }  // namespace
