@@ -859,10 +859,15 @@ __global__ void __launch_bounds__(kThreads, 2)
       tmem_ld16f_nowait(trow + kTcO + c0, ov[0]);
       tmem_ld16f_nowait(trow + kTcO + c0 + 16, ov[1]);
       tmem_wait_ld();
-      tc_fence_before();
-      __syncthreads();  // O has been read
-      tc_fence_after();
-      if (hd == 0 && tid == 0) issue_pv(1, NSt);
+      // The second half's MMAs overwrite O once every thread has read the
+      // first.  (After the second half, the next writer of O is the next
+      // tile's first half, issued after that tile's fenced barrier.)
+      if (hd == 0) {
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
+        if (tid == 0) issue_pv(1, NSt);
+      }
       if (valid) {
 #pragma unroll
         for (int k = 0; k < 2; ++k) {
