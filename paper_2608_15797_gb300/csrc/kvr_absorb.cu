@@ -165,6 +165,7 @@ __device__ void load_unit(const AbsorbParams &p, const Unit &u,
     m.acc[r] = 0.f;
   }
   cp_async_commit_wait_all();
+  fence_proxy_async();  // the rows are read by the tensor cores' async proxy too
   __syncthreads();
 }
 
@@ -515,7 +516,7 @@ struct TcSmem {  // offsets from a 1024-byte aligned base
   static constexpr int bytes = part + 16 * kTcMaxRows;
   static constexpr int alloc = bytes + 1024;               // room to align
 };
-static_assert(8 * kTcMaxRows >= 8 * kTcRows, "the exchange fits in the key area");
+static_assert(8 * kTcMaxRows >= 8 * kTcRows, "the exchange fits in the key and list areas");
 // Two CTAs an SM: 228 KB less 1 KB reserved per CTA, with room for the
 // static variables.
 static_assert(TcSmem::alloc + 512 <= 113 * 1024, "two CTAs an SM");
@@ -590,7 +591,10 @@ __global__ void __launch_bounds__(kThreads, 2)
                    reinterpret_cast<int *>(smem + TcSmem::lists),
                    reinterpret_cast<unsigned long long *>(smem + TcSmem::key),
                    reinterpret_cast<int *>(smem + TcSmem::kept)};
-  float2 *s_ml = reinterpret_cast<float2 *>(smem + TcSmem::key);  // free until the selection
+  // The (max, sum) exchange of the lower and the upper warps, in areas the
+  // selection uses only after the tiles.
+  float2 *s_ml = reinterpret_cast<float2 *>(smem + TcSmem::key);
+  float2 *s_mh = reinterpret_cast<float2 *>(smem + TcSmem::lists);
   if (warp == 0) tmem_alloc(smem_u32(&s_tmem), kTcCols);
   const int n = u.n, n0 = u.n0, h = u.h;
   const uint32_t aQ = smem_u32(smem + TcSmem::q);
@@ -618,7 +622,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     load_q(0);
   }
   tc_fence_before();
-  load_unit<kTcMaxRows>(p, u, m);  // ends with the copies complete and __syncthreads
+  load_unit<kTcMaxRows>(p, u, m);  // ends with the copies complete, the async proxy fenced and a barrier
   tc_fence_after();
   const uint32_t tm = s_tmem;
   const uint32_t aK = smem_u32(m.k), aV = smem_u32(m.v);
@@ -694,11 +698,8 @@ __global__ void __launch_bounds__(kThreads, 2)
     }
     return got;
   };
-  // K (written by the unit load) is visible to the tensor cores.
-  fence_proxy_async();
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
+  // (K, written by the unit load, is visible to the tensor cores: the load
+  // fenced the async proxy before its barrier.)
   if (tid == 32 && wait_q()) issue_s(0);
   for (int mt = 0; mt < n_mt && ok; ++mt) {
     // 1. S = Q K^T for the tile's keys is in tensor memory.
@@ -767,24 +768,15 @@ __global__ void __launch_bounds__(kThreads, 2)
       sm = s0 + s1;
     }
     // Warps w and w + 4 (the same 32 rows) exchange (max, sum) through
-    // shared memory on a named barrier of their own.
+    // shared memory on a named barrier of their own; both merge the two
+    // pairs in the same order, so they agree to the bit.
     const uint32_t bar_id = 1 + wq;
-    if (upper) s_ml[r] = make_float2(mx, sm);
+    (upper ? s_mh : s_ml)[r] = make_float2(mx, sm);
     asm volatile("bar.sync %0, 64;" ::"r"(bar_id) : "memory");
-    float M = mx, L = sm;
-    if (!upper) {
-      const float2 o2 = s_ml[r];
-      M = fmaxf(mx, o2.x);
-      L = (mx == -INFINITY ? 0.f : sm * ex2(mx - M)) +
-          (o2.x == -INFINITY ? 0.f : o2.y * ex2(o2.x - M));
-      s_ml[r] = make_float2(M, L);
-    }
-    asm volatile("bar.sync %0, 64;" ::"r"(bar_id) : "memory");
-    if (upper) {
-      const float2 o2 = s_ml[r];
-      M = o2.x;
-      L = o2.y;
-    }
+    const float2 lo2 = s_ml[r], hi2 = s_mh[r];
+    const float M = fmaxf(lo2.x, hi2.x);
+    const float L = (lo2.x == -INFINITY ? 0.f : lo2.y * ex2(lo2.x - M)) +
+                    (hi2.x == -INFINITY ? 0.f : hi2.y * ex2(hi2.x - M));
     if (valid && !upper && !(L >= 1.f && L < INFINITY)) atomicOr(c.err, ERR_NONFINITE);
     // p = e * exp2(own max - row max) / row sum; rows past the tile's
     // queries have f = 0 and finite e, so exact zeros.
